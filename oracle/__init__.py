@@ -1,0 +1,204 @@
+"""CPU oracle for the keyed Poisson-race multi-draft speculative sampler.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import this
+package.  The product path (``paper_2609_21858_gb300``) never imports it and
+shares no code with it.
+
+The arithmetic lives in ``pps_oracle.c`` (plain C, fp64); this module only
+compiles it with gcc and marshals numpy arrays through ctypes.  The closed
+forms used to pin it (acceptance probabilities, the watermark pivot law) are
+in ``oracle.closed_forms``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "pps_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+DISTINCT = 0
+IID = 1
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle shared library with gcc (-O2, OpenMP)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        cmd = ["gcc", "-O2", "-std=c99", "-fPIC", "-shared", "-fopenmp", "-o", tmp, _SRC, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _P(t):
+    return ctypes.POINTER(t)
+
+
+def lib():
+    global _lib
+    with _lock:
+        if _lib is None:
+            L = ctypes.CDLL(build())
+            u32p, u64p, i32p, i64p, f32p, f64p = (_P(ctypes.c_uint32), _P(ctypes.c_uint64), _P(ctypes.c_int32),
+                                                  _P(ctypes.c_int64), _P(ctypes.c_float), _P(ctypes.c_double))
+            i64, i32, f64 = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
+            L.orc_philox4x32_10.argtypes = [u32p, u32p, u32p]
+            L.orc_philox4x32_10.restype = None
+            L.orc_word.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32, i64, i32]
+            L.orc_word.restype = ctypes.c_uint32
+            L.orc_uniform.argtypes = [ctypes.c_uint32]
+            L.orc_uniform.restype = f64
+            L.orc_exp1.argtypes = [ctypes.c_uint32]
+            L.orc_exp1.restype = f64
+            L.orc_score_word.argtypes = [ctypes.c_uint32]
+            L.orc_score_word.restype = f64
+            L.orc_race_key.argtypes = [ctypes.c_uint32, f64, f64]
+            L.orc_race_key.restype = f64
+            L.orc_target_rows.argtypes = [f32p, i64, i64, i64, f64, u64p, u64p, u32p, i32p, u32p, f64p, f64p]
+            L.orc_target_rows.restype = None
+            L.orc_draft_rows.argtypes = [f32p, i64, i64, i64, f64, u64p, u64p, u32p, i32, i32p, i32,
+                                         i32p, f64p, i32p, i32p, i32p, f64p]
+            L.orc_draft_rows.restype = None
+            L.orc_walk.argtypes = [i32, i32, i32p, i32p, i32p, i32p, i32, i32p, i32p, u32p,
+                                   i32p, i32p, i32p, f64p, f64p]
+            L.orc_walk.restype = None
+            L.orc_wm_score.argtypes = [i64, i32p, u64p, u64p, u32p, f64p, i32, i64p, f64p]
+            L.orc_wm_score.restype = None
+            L.orc_words.argtypes = [i64, i64, u64p, u64p, u32p, i32, u32p]
+            L.orc_words.restype = None
+            L.orc_set_threads.argtypes = [ctypes.c_int]
+            L.orc_set_threads.restype = ctypes.c_int
+            _lib = L
+    return _lib
+
+
+def _ptr(a, t):
+    return a.ctypes.data_as(_P(t)) if a is not None else None
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(np.asarray(a, dtype=dtype))
+
+
+def set_threads(n: int = 0) -> int:
+    """Set (n > 0) and return the number of OpenMP threads the oracle uses."""
+    return int(lib().orc_set_threads(int(n)))
+
+
+def philox4x32_10(ctr, key):
+    c = _c(ctr, np.uint32)
+    k = _c(key, np.uint32)
+    out = np.zeros(4, np.uint32)
+    lib().orc_philox4x32_10(_ptr(c, ctypes.c_uint32), _ptr(k, ctypes.c_uint32), _ptr(out, ctypes.c_uint32))
+    return out
+
+
+def word(key: int, ctx: int, pos: int, token: int, arrival: int = 1) -> int:
+    return int(lib().orc_word(key, ctx, pos, token, arrival))
+
+
+def uniform(w: int) -> float:
+    return float(lib().orc_uniform(w))
+
+
+def exp1(w: int) -> float:
+    return float(lib().orc_exp1(w))
+
+
+def score_word(w: int) -> float:
+    return float(lib().orc_score_word(w))
+
+
+def race_key(w: int, logit: float, T: float = 1.0) -> float:
+    return float(lib().orc_race_key(w, logit, T))
+
+
+def words(key, ctx, pos, vocab: int, arrival: int = 1):
+    key, ctx, pos = _c(key, np.uint64), _c(ctx, np.uint64), _c(pos, np.uint32)
+    n = key.shape[0]
+    out = np.zeros((n, vocab), np.uint32)
+    lib().orc_words(n, vocab, _ptr(key, ctypes.c_uint64), _ptr(ctx, ctypes.c_uint64), _ptr(pos, ctypes.c_uint32),
+                    arrival, _ptr(out, ctypes.c_uint32))
+    return out
+
+
+def target_rows(logits, key, ctx, pos, T: float = 1.0):
+    """Per row: (winner, word, key, margin) of the target race argmin_i E_i/P(i)."""
+    l = _c(logits, np.float32)
+    n, V = l.shape
+    key, ctx, pos = _c(key, np.uint64), _c(ctx, np.uint64), _c(pos, np.uint32)
+    win = np.zeros(n, np.int32)
+    wd = np.zeros(n, np.uint32)
+    ky = np.zeros(n, np.float64)
+    mg = np.zeros(n, np.float64)
+    lib().orc_target_rows(_ptr(l, ctypes.c_float), n, V, V, float(T), _ptr(key, ctypes.c_uint64),
+                          _ptr(ctx, ctypes.c_uint64), _ptr(pos, ctypes.c_uint32), _ptr(win, ctypes.c_int32),
+                          _ptr(wd, ctypes.c_uint32), _ptr(ky, ctypes.c_double), _ptr(mg, ctypes.c_double))
+    return win, wd, ky, mg
+
+
+def draft_rows(logits, key, ctx, pos, K: int, row_k=None, mode: int = DISTINCT, T: float = 1.0):
+    """Per row: dict(tok, key, mult, ndist, labels, min_gap) of the draft list."""
+    l = _c(logits, np.float32)
+    n, V = l.shape
+    key, ctx, pos = _c(key, np.uint64), _c(ctx, np.uint64), _c(pos, np.uint32)
+    rk = _c(row_k, np.int32) if row_k is not None else None
+    tok = np.zeros((n, K), np.int32)
+    ky = np.zeros((n, K), np.float64)
+    mult = np.zeros((n, K), np.int32)
+    nd = np.zeros(n, np.int32)
+    lab = np.zeros((n, K), np.int32)
+    gap = np.zeros(n, np.float64)
+    lib().orc_draft_rows(_ptr(l, ctypes.c_float), n, V, V, float(T), _ptr(key, ctypes.c_uint64),
+                         _ptr(ctx, ctypes.c_uint64), _ptr(pos, ctypes.c_uint32), int(K), _ptr(rk, ctypes.c_int32),
+                         int(mode), _ptr(tok, ctypes.c_int32), _ptr(ky, ctypes.c_double), _ptr(mult, ctypes.c_int32),
+                         _ptr(nd, ctypes.c_int32), _ptr(lab, ctypes.c_int32), _ptr(gap, ctypes.c_double))
+    return dict(tok=tok, key=ky, mult=mult, ndist=nd, labels=lab, min_gap=gap)
+
+
+def walk(gamma: int, seq_off, node_draft_row, draft_tok, draft_ndist, child_node, winner, word_):
+    seq_off = _c(seq_off, np.int32)
+    ndr = _c(node_draft_row, np.int32)
+    dt = _c(draft_tok, np.int32)
+    K = dt.shape[1] if dt.ndim == 2 else 1
+    dn = _c(draft_ndist, np.int32)
+    cn = _c(child_node, np.int32)
+    win = _c(winner, np.int32)
+    wd = _c(word_, np.uint32)
+    n_seq = seq_off.shape[0] - 1
+    W = gamma + 1
+    acc = np.zeros(n_seq, np.int32)
+    ne = np.zeros(n_seq, np.int32)
+    em = np.zeros((n_seq, W), np.int32)
+    sc = np.zeros((n_seq, W), np.float64)
+    ss = np.zeros(n_seq, np.float64)
+    lib().orc_walk(n_seq, gamma, _ptr(seq_off, ctypes.c_int32), _ptr(ndr, ctypes.c_int32), _ptr(dt, ctypes.c_int32),
+                   _ptr(dn, ctypes.c_int32), K, _ptr(cn, ctypes.c_int32), _ptr(win, ctypes.c_int32),
+                   _ptr(wd, ctypes.c_uint32), _ptr(acc, ctypes.c_int32), _ptr(ne, ctypes.c_int32),
+                   _ptr(em, ctypes.c_int32), _ptr(sc, ctypes.c_double), _ptr(ss, ctypes.c_double))
+    return dict(accept_len=acc, n_emitted=ne, emitted=em, score=sc, score_sum=ss)
+
+
+def wm_score(tokens, key, ctx, pos, seg_off=None):
+    t = _c(tokens, np.int32)
+    n = t.shape[0]
+    key, ctx, pos = _c(key, np.uint64), _c(ctx, np.uint64), _c(pos, np.uint32)
+    sc = np.zeros(n, np.float64)
+    so = _c(seg_off, np.int64) if seg_off is not None else None
+    n_seg = (so.shape[0] - 1) if so is not None else 1
+    sums = np.zeros(n_seg, np.float64)
+    lib().orc_wm_score(n, _ptr(t, ctypes.c_int32), _ptr(key, ctypes.c_uint64), _ptr(ctx, ctypes.c_uint64),
+                       _ptr(pos, ctypes.c_uint32), _ptr(sc, ctypes.c_double), n_seg, _ptr(so, ctypes.c_int64),
+                       _ptr(sums, ctypes.c_double))
+    return sc, sums

@@ -1,0 +1,358 @@
+/*
+ * pps_oracle.c -- plain, slow, double-precision CPU oracle for the keyed
+ * Poisson-race (exponential race) multi-draft speculative sampler of
+ * "Watermarkable Multi-Draft Speculative Sampling via Poisson Processes".
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the
+ * cpu_baseline / reference legs of bench.py may load this library.  It shares
+ * no code, header, table or constant generator with the CUDA path; it is an
+ * independent restatement of the paper's definitions, written for a reader to
+ * check by eye, not for speed.  Rows are independent, so an OpenMP loop over
+ * rows is the only concession to run time; it changes no arithmetic.
+ *
+ * What each function follows:
+ *   orc_philox4x32_10  Philox4x32-10 counter-based generator (Salmon, Moraes,
+ *                      Dror, Shaw, "Parallel random numbers: as easy as 1, 2, 3",
+ *                      SC'11): 10 rounds of the 4x32 Philox S-box with the
+ *                      published multipliers and Weyl key increments.  The
+ *                      paper only asks for a keyed pseudorandom function
+ *                      F_{ctx,k} (Sec. 3.1, Eq. 1) / keyed source G(k,c)
+ *                      (Alg. 3); Philox is this build's reading.
+ *   orc_word           the keyed source Pi_k(c): counter (token>>2, pos,
+ *                      ctx_lo, ctx_hi), key (key_lo ^ (j-1)*0x9E3779B9, key_hi)
+ *                      for arrival j, output lane token&3.
+ *   orc_exp1           E = -ln u with u = (w + 1/2) 2^-32 (first arrival time
+ *                      scaled to Exp(1), Thm A.1 Eq. "E_z = q_z S_z").
+ *   orc_race_key       s = ln E - l/T, the log of E/p up to a row constant
+ *                      (exponential race, Alg. 2; Gumbel-max equivalence,
+ *                      App. A.2).
+ *   orc_target_rows    y(c) = argmin_i E_i / P(i) (EFR, Thm A.1; target side of
+ *                      the batched direct top-k algorithm, App. B).
+ *   orc_draft_rows     DISTINCT: the K smallest E_i/Q(i) (first arrivals);
+ *                      IID: the K smallest multi-arrival scores
+ *                      G_{u,j}/Q(u), G_{u,j} = sum_{m<=j} E_{u,m}, j = 1..K,
+ *                      over every token u with Q(u) > 0 (direct finite-support
+ *                      MPFR algorithm, App. B, Thm "exactness of direct
+ *                      finite-support MPFR").
+ *   orc_walk           follow the realised target path through the context
+ *                      tree, accept while y(c*) is in D(c*), bonus token after
+ *                      gamma acceptances (Alg. 4; batched algorithm, App. B).
+ *   orc_wm_score       A_t = -ln(1 - r_t(w_t)) with pivot r_t = u of the
+ *                      emitted token (Eq. 2; App. D.1 "Gumbel watermark";
+ *                      detector algorithm, App. E).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* ------------------------------------------------------------------ */
+/* Philox4x32-10                                                       */
+/* ------------------------------------------------------------------ */
+
+/* multipliers and Weyl key increments published for Philox4x32 */
+#define ORC_PHILOX_M0 0xD2511F53u
+#define ORC_PHILOX_M1 0xCD9E8D57u
+#define ORC_PHILOX_W0 0x9E3779B9u
+#define ORC_PHILOX_W1 0xBB67AE85u
+
+void orc_philox4x32_10(const uint32_t ctr_in[4], const uint32_t key_in[2], uint32_t out[4])
+{
+    uint32_t x0 = ctr_in[0], x1 = ctr_in[1], x2 = ctr_in[2], x3 = ctr_in[3];
+    uint32_t k0 = key_in[0], k1 = key_in[1];
+    for (int round = 0; round < 10; ++round) {
+        if (round > 0) { /* key schedule: bump before every round but the first */
+            k0 += ORC_PHILOX_W0;
+            k1 += ORC_PHILOX_W1;
+        }
+        uint64_t p0 = (uint64_t)ORC_PHILOX_M0 * (uint64_t)x0;
+        uint64_t p1 = (uint64_t)ORC_PHILOX_M1 * (uint64_t)x2;
+        uint32_t hi0 = (uint32_t)(p0 >> 32), lo0 = (uint32_t)p0;
+        uint32_t hi1 = (uint32_t)(p1 >> 32), lo1 = (uint32_t)p1;
+        uint32_t y0 = hi1 ^ x1 ^ k0;
+        uint32_t y1 = lo1;
+        uint32_t y2 = hi0 ^ x3 ^ k1;
+        uint32_t y3 = lo0;
+        x0 = y0; x1 = y1; x2 = y2; x3 = y3;
+    }
+    out[0] = x0; out[1] = x1; out[2] = x2; out[3] = x3;
+}
+
+/* Keyed source: the 32-bit word of token `token`, arrival j >= 1, at the
+ * context labelled (ctx, pos) under watermark key `key`. */
+uint32_t orc_word(uint64_t key, uint64_t ctx, uint32_t pos, int64_t token, int32_t arrival)
+{
+    uint32_t ctr[4], k[2], out[4];
+    ctr[0] = (uint32_t)((uint64_t)token >> 2);
+    ctr[1] = pos;
+    ctr[2] = (uint32_t)(ctx & 0xFFFFFFFFull);
+    ctr[3] = (uint32_t)(ctx >> 32);
+    uint32_t tweak = (uint32_t)(arrival - 1) * ORC_PHILOX_W0; /* 0 for the first arrival */
+    k[0] = (uint32_t)(key & 0xFFFFFFFFull) ^ tweak;
+    k[1] = (uint32_t)(key >> 32);
+    orc_philox4x32_10(ctr, k, out);
+    return out[token & 3];
+}
+
+/* ------------------------------------------------------------------ */
+/* uniform, exponential, race key, score                               */
+/* ------------------------------------------------------------------ */
+
+/* u = (w + 1/2) 2^-32, never 0 or 1, exact in double */
+double orc_uniform(uint32_t w) { return ((double)w + 0.5) * 0x1p-32; }
+
+/* 1 - u = (~w + 1/2) 2^-32, exact in double */
+static double orc_one_minus_uniform(uint32_t w) { return ((double)(uint32_t)~w + 0.5) * 0x1p-32; }
+
+/* E = -ln u ~ Exp(1).  For u > 1/2 the same value is written through
+ * v = 1 - u so that small E keeps its relative precision. */
+double orc_exp1(uint32_t w)
+{
+    if (w < 0x80000000u) return -log(orc_uniform(w));
+    return -log1p(-orc_one_minus_uniform(w));
+}
+
+/* Aaronson per-token score A = -ln(1 - u) (Eq. 2). */
+double orc_score_word(uint32_t w)
+{
+    if (w < 0x80000000u) return -log1p(-orc_uniform(w));
+    return -log(orc_one_minus_uniform(w));
+}
+
+/* race key s = ln E - l/T.  A token with P = 0 (logit -inf) or an unusable
+ * logit (NaN) never wins: key +inf.  A logit of +inf gives -inf. */
+double orc_race_key(uint32_t w, double logit, double T)
+{
+    if (isnan(logit)) return INFINITY;
+    return log(orc_exp1(w)) - logit / T;
+}
+
+/* (key, index) lexicographic order: ties go to the smaller token index */
+static int orc_before(double ka, int64_t ia, double kb, int64_t ib)
+{
+    if (ka < kb) return 1;
+    if (ka > kb) return 0;
+    return ia < ib;
+}
+
+/* ------------------------------------------------------------------ */
+/* target winner per row                                               */
+/* ------------------------------------------------------------------ */
+
+/* winner[r] = argmin_i s_i (or -1 if every key is +inf); word[r] its first-
+ * arrival word; key[r] its key; margin[r] = s_(2) - s_(1) (+inf if < 2). */
+void orc_target_rows(const float* logits, int64_t n_rows, int64_t V, int64_t stride, double T,
+                     const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
+                     int32_t* winner, uint32_t* word, double* key_out, double* margin)
+{
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t r = 0; r < n_rows; ++r) {
+        const float* l = logits + r * stride;
+        double best = INFINITY, second = INFINITY;
+        int64_t bi = -1, si = -1;
+        for (int64_t i = 0; i < V; ++i) {
+            uint32_t w = orc_word(key[r], ctx[r], pos[r], i, 1);
+            double s = orc_race_key(w, (double)l[i], T);
+            if (s == INFINITY) continue;
+            if (bi < 0 || orc_before(s, i, best, bi)) {
+                second = best; si = bi;
+                best = s; bi = i;
+            } else if (si < 0 || orc_before(s, i, second, si)) {
+                second = s; si = i;
+            }
+        }
+        winner[r] = (int32_t)bi;
+        if (word) word[r] = bi >= 0 ? orc_word(key[r], ctx[r], pos[r], bi, 1) : 0u;
+        if (key_out) key_out[r] = best;
+        if (margin) margin[r] = (bi >= 0 && si >= 0) ? second - best : INFINITY;
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* draft lists                                                         */
+/* ------------------------------------------------------------------ */
+
+typedef struct { double s; int64_t i; int32_t j; } orc_cand;
+
+static int orc_cand_cmp(const void* a, const void* b)
+{
+    const orc_cand* x = (const orc_cand*)a;
+    const orc_cand* y = (const orc_cand*)b;
+    if (x->s < y->s) return -1;
+    if (x->s > y->s) return 1;
+    if (x->i != y->i) return x->i < y->i ? -1 : 1;
+    if (x->j != y->j) return x->j < y->j ? -1 : 1;
+    return 0;
+}
+
+/* mode 0 = DISTINCT, 1 = IID.
+ * Per row r with list length k_r = row_k ? row_k[r] : K:
+ *   tok[r*K + m]   m-th smallest first-arrival key (ascending, ties by index),
+ *                  -1 past the end of the usable tokens or past k_r;
+ *   keys[r*K + m]  its key (+inf when tok = -1);
+ *   mult[r*K + m]  DISTINCT: 1 for a valid entry; IID: how many of the k_r
+ *                  multi-arrival samples carry label tok[m];
+ *   ndist[r]       number of distinct draft tokens |D(c)|;
+ *   labels[r*K+m]  (nullable) the ordered samples: DISTINCT = tok, IID = the
+ *                  labels U_(1..k_r) of the k_r smallest scores;
+ *   min_gap[r]     (nullable) smallest gap between consecutive first-arrival
+ *                  keys s_(m+1) - s_(m), m = 1..k_r (flip accounting).
+ */
+void orc_draft_rows(const float* logits, int64_t n_rows, int64_t V, int64_t stride, double T,
+                    const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
+                    int32_t K, const int32_t* row_k, int32_t mode,
+                    int32_t* tok, double* keys, int32_t* mult, int32_t* ndist,
+                    int32_t* labels, double* min_gap)
+{
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t r = 0; r < n_rows; ++r) {
+        const float* l = logits + r * stride;
+        int32_t kr = row_k ? row_k[r] : K;
+        orc_cand* first = (orc_cand*)malloc(sizeof(orc_cand) * (size_t)V);
+        int64_t n_use = 0;
+        for (int64_t i = 0; i < V; ++i) {
+            uint32_t w = orc_word(key[r], ctx[r], pos[r], i, 1);
+            double s = orc_race_key(w, (double)l[i], T);
+            if (s == INFINITY) continue;
+            first[n_use].s = s; first[n_use].i = i; first[n_use].j = 1;
+            ++n_use;
+        }
+        qsort(first, (size_t)n_use, sizeof(orc_cand), orc_cand_cmp);
+        for (int32_t m = 0; m < K; ++m) {
+            int ok = m < kr && m < n_use;
+            tok[r * K + m] = ok ? (int32_t)first[m].i : -1;
+            if (keys) keys[r * K + m] = ok ? first[m].s : INFINITY;
+            mult[r * K + m] = 0;
+            if (labels) labels[r * K + m] = -1;
+        }
+        if (min_gap) {
+            double g = INFINITY;
+            for (int32_t m = 0; m < kr && m + 1 < n_use; ++m) {
+                double d = first[m + 1].s - first[m].s;
+                if (d < g) g = d;
+            }
+            min_gap[r] = g;
+        }
+        int32_t nvalid = kr < n_use ? kr : (int32_t)n_use;
+        if (mode == 0) {
+            for (int32_t m = 0; m < nvalid; ++m) {
+                mult[r * K + m] = 1;
+                if (labels) labels[r * K + m] = (int32_t)first[m].i;
+            }
+            ndist[r] = nvalid;
+        } else {
+            /* every usable token u contributes arrivals j = 1..k_r with score
+             * ln(G_{u,j}) - l_u/T; keep the k_r smallest */
+            int64_t nc = n_use * (int64_t)kr;
+            orc_cand* all = (orc_cand*)malloc(sizeof(orc_cand) * (size_t)(nc > 0 ? nc : 1));
+            int64_t c = 0;
+            for (int64_t i = 0; i < V; ++i) {
+                double li = (double)l[i];
+                if (isnan(li) || li == -INFINITY) continue;
+                double G = 0.0;
+                for (int32_t j = 1; j <= kr; ++j) {
+                    G += orc_exp1(orc_word(key[r], ctx[r], pos[r], i, j));
+                    all[c].s = log(G) - li / T;
+                    all[c].i = i; all[c].j = j;
+                    ++c;
+                }
+            }
+            qsort(all, (size_t)c, sizeof(orc_cand), orc_cand_cmp);
+            int32_t ns = kr < c ? kr : (int32_t)c;
+            for (int32_t m = 0; m < ns; ++m) {
+                if (labels) labels[r * K + m] = (int32_t)all[m].i;
+                for (int32_t q = 0; q < nvalid; ++q)
+                    if (tok[r * K + q] == (int32_t)all[m].i) { mult[r * K + q] += 1; break; }
+            }
+            int32_t nd = 0;
+            for (int32_t q = 0; q < nvalid; ++q) nd += mult[r * K + q] > 0;
+            ndist[r] = nd;
+            free(all);
+        }
+        free(first);
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* tree walk and per-token score                                       */
+/* ------------------------------------------------------------------ */
+
+/* Sequence b owns nodes [seq_off[b], seq_off[b+1]); its root is seq_off[b].
+ * Node c has draft row dr = node_draft_row[c] (-1 for a leaf); D(c) is
+ * draft_tok[dr*K + m] for m < draft_ndist[dr], and child_node[dr*K + m] is
+ * the node reached by that token (-1 if the caller evaluated none).
+ * Outputs per sequence: accept_len (accepted steps, 0..gamma), n_emitted,
+ * emitted[b*(gamma+1) + t], score[...] (A of each emitted token, 0 past the
+ * end, emitted = -1 past the end), score_sum[b] (sum of A). */
+void orc_walk(int32_t n_seq, int32_t gamma, const int32_t* seq_off, const int32_t* node_draft_row,
+              const int32_t* draft_tok, const int32_t* draft_ndist, int32_t K, const int32_t* child_node,
+              const int32_t* winner, const uint32_t* word,
+              int32_t* accept_len, int32_t* n_emitted, int32_t* emitted, double* score, double* score_sum)
+{
+    for (int32_t b = 0; b < n_seq; ++b) {
+        int32_t W = gamma + 1;
+        for (int32_t t = 0; t < W; ++t) { emitted[b * W + t] = -1; score[b * W + t] = 0.0; }
+        int32_t c = seq_off[b], acc = 0, ne = 0;
+        double S = 0.0;
+        int stopped = 0;
+        for (int32_t s = 0; s < gamma; ++s) {
+            int32_t y = winner[c];
+            if (y < 0) { stopped = 1; break; }
+            double A = orc_score_word(word[c]);
+            emitted[b * W + ne] = y; score[b * W + ne] = A; S += A; ++ne;
+            int32_t dr = node_draft_row[c], found = -1;
+            if (dr >= 0)
+                for (int32_t m = 0; m < draft_ndist[dr]; ++m)
+                    if (draft_tok[dr * K + m] == y) { found = m; break; }
+            if (found < 0) { stopped = 1; break; }
+            int32_t nxt = child_node[dr * K + found];
+            if (nxt < 0) { stopped = 1; break; }
+            c = nxt; ++acc;
+        }
+        if (!stopped && winner[c] >= 0) {
+            double A = orc_score_word(word[c]);
+            emitted[b * W + ne] = winner[c]; score[b * W + ne] = A; S += A; ++ne;
+        }
+        accept_len[b] = acc; n_emitted[b] = ne; score_sum[b] = S;
+    }
+}
+
+/* Detector pass: per token A_t from the regenerated first-arrival word, and
+ * per segment sums (seg_off[n_seg+1]; nullable -> one segment). */
+void orc_wm_score(int64_t n, const int32_t* tokens, const uint64_t* key, const uint64_t* ctx,
+                  const uint32_t* pos, double* score, int32_t n_seg, const int64_t* seg_off, double* sums)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t t = 0; t < n; ++t)
+        score[t] = orc_score_word(orc_word(key[t], ctx[t], pos[t], tokens[t], 1));
+    if (!sums) return;
+    if (!seg_off) { double S = 0.0; for (int64_t t = 0; t < n; ++t) S += score[t]; sums[0] = S; return; }
+    for (int32_t g = 0; g < n_seg; ++g) {
+        double S = 0.0;
+        for (int64_t t = seg_off[g]; t < seg_off[g + 1]; ++t) S += score[t];
+        sums[g] = S;
+    }
+}
+
+/* raw words of rows x vocab for a given arrival (bit-exact checks) */
+void orc_words(int64_t n_rows, int64_t V, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
+               int32_t arrival, uint32_t* out)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t r = 0; r < n_rows; ++r)
+        for (int64_t i = 0; i < V; ++i) out[r * V + i] = orc_word(key[r], ctx[r], pos[r], i, arrival);
+}
+
+int orc_set_threads(int n)
+{
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+    return omp_get_max_threads();
+#else
+    (void)n;
+    return 1;
+#endif
+}
