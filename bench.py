@@ -1,0 +1,334 @@
+"""Benchmark of the keyed-race hot path on GB300.
+
+One step = pps_draft_list over every draft row + pps_verify_tree over every
+node row (target race, tree walk, watermark scores) of one batch of
+synthetic logits.  Default workload: B=64 sequences, V=128256, K=8 drafts,
+gamma=5 (K chains of depth 5 = 41 nodes per sequence: 2,624 target rows and
+2,112 draft rows), bf16 Zipf(1.0) logits under a random vocabulary
+permutation per row, draft = target + N(0,1).  Inputs (1.21 GB) exceed L2
+(129 MB), so no flush is needed between steps.
+
+`value` counts row-passes per second (draft rows + target rows, all ranks).
+`--impl reference` times the CPU oracle on a bounded sample of the same rows.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verified rows/s and GB/s vs HBM peak at V=128256, K=8, B=64 (1xGB300)"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                p = [x.strip() for x in line.split(",")]
+                if len(p) < 9:
+                    continue
+                try:
+                    sm.append(float(p[1]))
+                    smax.append(float(p[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, p[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_init():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def oracle_sample(wl, n_draft_rows: int, n_target_rows: int, seed: int = 0):
+    """Host copies of a bounded sample of the workload's rows and a timer over them."""
+    import oracle
+    from paper_2609_21858_gb300 import synth
+    t = wl.tree
+    rng = np.random.default_rng(seed)
+    dr = np.sort(rng.choice(t.n_draft, min(n_draft_rows, t.n_draft), replace=False))
+    nr = np.sort(rng.choice(t.n_nodes, min(n_target_rows, t.n_nodes), replace=False))
+    dsel = torch.as_tensor(dr, device=wl.q_logits.device)
+    nsel = torch.as_tensor(nr, device=wl.p_logits.device)
+    q = wl.q_logits[dsel].float().cpu().numpy()
+    p = wl.p_logits[nsel].float().cpu().numpy()
+    ids_d = (synth.u64(wl.draft_key[dsel]), synth.u64(wl.draft_ctx[dsel]), synth.u32(wl.draft_pos[dsel]))
+    ids_n = (synth.u64(wl.node_key[nsel]), synth.u64(wl.node_ctx[nsel]), synth.u32(wl.node_pos[nsel]))
+    rk = t.row_k[dr]
+    cores = oracle.set_threads(0)
+
+    def run():
+        t0 = time.perf_counter()
+        oracle.draft_rows(q, *ids_d, t.K, row_k=rk)
+        oracle.target_rows(p, *ids_n)
+        return time.perf_counter() - t0
+
+    return run, len(dr), len(nr), cores
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="zipf_k8")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+
+    rank, world, local = dist_init()
+    from paper_2609_21858_gb300 import synth
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        run_reference(args, world)
+        return
+
+    from paper_2609_21858_gb300 import pps
+    pps.lib()
+    dev = torch.device("cuda", local)
+    wl = synth.make_workload(args.workload, device=dev, seed=None)
+    t = wl.tree
+    g = lambda x: torch.as_tensor(np.asarray(x)).to(dev).contiguous()
+    row_k, seq_off, ndr, child = g(t.row_k), g(t.seq_off), g(t.node_draft_row), g(t.child_node)
+    dk, dc, dp = wl.draft_key, wl.draft_ctx, wl.draft_pos
+    nk, nc, np_ = wl.node_key, wl.node_ctx, wl.node_pos
+    ws_d = pps.workspace(t.n_draft, 0, dev)
+    ws_v = pps.workspace(t.n_nodes, t.n_seq, dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    dout = dict(tok=torch.empty(t.n_draft, t.K, dtype=torch.int32, device=dev), key=None,
+                mult=torch.empty(t.n_draft, t.K, dtype=torch.int32, device=dev),
+                ndist=torch.empty(t.n_draft, dtype=torch.int32, device=dev), samples=None)
+    W = t.gamma + 1
+    vout = dict(winner=torch.empty(t.n_nodes, dtype=torch.int32, device=dev),
+                word=torch.empty(t.n_nodes, dtype=torch.int32, device=dev),
+                accept_len=torch.empty(t.n_seq, dtype=torch.int32, device=dev),
+                n_emitted=torch.empty(t.n_seq, dtype=torch.int32, device=dev),
+                emitted=torch.empty(t.n_seq, W, dtype=torch.int32, device=dev),
+                score=torch.empty(t.n_seq, W, dtype=torch.float32, device=dev),
+                score_sum=torch.empty(t.n_seq, dtype=torch.float64, device=dev))
+    stream = torch.cuda.current_stream(dev)
+
+    def step(q, p, ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        pps.draft_list(q, dk, dc, dp, t.K, row_k=row_k, ws=ws_d, status=status, out=dout, stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+        pps.verify_tree(p, nk, nc, np_, t.gamma, seq_off, ndr, dout["tok"], dout["ndist"], child, ws=ws_v,
+                        status=status, out=vout, stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+
+    q, p = wl.q_logits, wl.p_logits
+    for _ in range(max(3, args.warmup)):
+        step(q, p)
+    torch.cuda.synchronize(dev)
+    assert int(status.item()) == 0, f"status flags {int(status.item())}"
+
+    # ---- device-timed region
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk = Clocks(local)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    clk.start()
+    time.sleep(0.3)
+    start.record(stream)
+    for k in range(args.steps):
+        step(q, p, evs[k])
+    stop.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = clk.stop()
+    barrier(world)
+    ms = start.elapsed_time(stop)
+    ms = max_over_ranks(ms, world)
+    t_draft = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    t_verify = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+
+    esz = wl.p_logits.element_size()
+    rows_per_step = t.n_nodes + t.n_draft
+    bytes_verify = t.n_nodes * wl.vocab * esz
+    bytes_draft = t.n_draft * wl.vocab * esz
+    ms_step = ms / args.steps
+    value = rows_per_step * world / (ms_step / 1e3)
+    peak, peak_kind = _peaks()
+    ach_v = bytes_verify / (t_verify / 1e3) / 1e9
+    ach_d = bytes_draft / (t_draft / 1e3) / 1e9
+    ach_all = (bytes_verify + bytes_draft) / (ms_step / 1e3) / 1e9
+    emitted = float(vout["n_emitted"].sum().item())
+
+    # ---- end to end through host buffers
+    e2e = None
+    if args.e2e_steps > 0:
+        hq = torch.empty(q.shape, dtype=q.dtype, pin_memory=True)
+        hp = torch.empty(p.shape, dtype=p.dtype, pin_memory=True)
+        hq.copy_(q)
+        hp.copy_(p)
+        h_em = torch.empty(vout["emitted"].shape, dtype=torch.int32, pin_memory=True)
+        h_ne = torch.empty(t.n_seq, dtype=torch.int32, pin_memory=True)
+        h_ss = torch.empty(t.n_seq, dtype=torch.float64, pin_memory=True)
+        dq, dp2 = torch.empty_like(q), torch.empty_like(p)
+
+        def e2e_step():
+            dq.copy_(hq, non_blocking=True)
+            dp2.copy_(hp, non_blocking=True)
+            step(dq, dp2)
+            h_em.copy_(vout["emitted"], non_blocking=True)
+            h_ne.copy_(vout["n_emitted"], non_blocking=True)
+            h_ss.copy_(vout["score_sum"], non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        e_ms = max_over_ranks(e0.elapsed_time(e1) / args.e2e_steps, world)
+        e2e = {"value": rows_per_step * world / (e_ms / 1e3), "unit": "rows/s",
+               "h2d_bytes_per_step": int(hq.numel() * esz + hp.numel() * esz),
+               "d2h_bytes_per_step": int(h_em.numel() * 4 + h_ne.numel() * 4 + h_ss.numel() * 8),
+               "ms_per_step": e_ms}
+        del hq, hp, dq, dp2
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        run, nd, nn, cores = oracle_sample(wl, 8, 8)
+        dt = run()
+        reps = max(1, int(args.cpu_seconds / max(dt, 1e-3)))
+        tot = sum(run() for _ in range(reps))
+        cpu = {"value": reps * (nd + nn) / tot, "unit": "rows/s", "cores": cores, "kind": "oracle",
+               "sample": f"{nd} draft + {nn} target rows of the same workload, x{reps} repetitions, "
+                         f"{tot:.1f} s on {cores} threads"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if wl.dtype == torch.bfloat16 else "f32",
+            "data": "synthetic (seeded Zipf-rank logits; no model, no dataset)",
+            "config": {"workload": f"{args.workload}: B={t.n_seq}, V={wl.vocab}, K={t.K}, gamma={t.gamma}, "
+                                   f"{t.n_nodes} target rows + {t.n_draft} draft rows per step",
+                       "rows_per_step": rows_per_step, "l2": "inputs (1.21 GB) larger than L2, no flush",
+                       "parallelism": f"replicas x{world}"},
+            "gb_per_s": ach_all, "tokens_per_s": emitted * world / (ms_step / 1e3),
+            "roofline": {"bound": "hbm", "achieved": ach_v, "peak": peak, "unit": "GB/s", "frac": ach_v / peak,
+                         "traffic": None, "kernel": "race_kernel<bf16, verify> (pps_verify_tree)",
+                         "peak_kind": peak_kind, "algorithmic_bytes": bytes_verify, "ms": t_verify},
+            "roofline_draft": {"achieved": ach_d, "frac": ach_d / peak, "ms": t_draft, "algorithmic_bytes": bytes_draft},
+            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": 2 * args.steps, "clocks": clocks,
+            "mean_accept_len": float(vout["accept_len"].float().mean().item()),
+        }
+        print(json.dumps(line))
+
+
+def run_reference(args, world):
+    """The CPU oracle on a bounded sample per step, on this host's cores."""
+    from paper_2609_21858_gb300 import synth
+    wl = synth.make_workload(args.workload, device="cuda" if torch.cuda.is_available() else "cpu")
+    t = wl.tree
+    run, nd, nn, cores = oracle_sample(wl, 4, 4)
+    for _ in range(max(1, min(args.warmup, 2))):
+        run()
+    times = [run() for _ in range(args.steps)]
+    tot = sum(times)
+    value = args.steps * (nd + nn) / tot
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{args.workload}: B={t.n_seq}, V={wl.vocab}, K={t.K}, gamma={t.gamma}",
+                   "rows_per_step": nd + nn},
+        "cpu_baseline": {"value": value, "unit": "rows/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{nd} draft + {nn} target rows per step"},
+        "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,189 @@
+/*
+ * pps.h -- C ABI of libpps, the GB300 (sm_103a) implementation of the keyed
+ * Poisson-race multi-draft speculative sampler of "Watermarkable Multi-Draft
+ * Speculative Sampling via Poisson Processes".
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every pointer argument is DEVICE memory on the current CUDA device, owned
+ *   by the caller, unless the comment says otherwise.  The library never
+ *   allocates device memory and keeps no state between calls.
+ * - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *   stream).  A non-PPS_OK return from argument validation is synchronous and
+ *   launches nothing.  PPS_ERR_CUDA reports a failed launch (cudaGetLastError
+ *   after the launch); the CUDA error itself stays readable through the CUDA
+ *   runtime.  Outputs are undefined unless the call returned PPS_OK.
+ * - Logits rows are `row_stride` elements apart (row_stride >= vocab),
+ *   row-major, fp32 or bf16.  Rows whose start is 16-byte aligned are
+ *   streamed with 128-bit loads; other layouts take a slower scalar path.
+ * - Row identities (pps_row_ids) label the keyed Poisson source G(k, c) of the
+ *   paper (Sec. 3.3, Alg. 3 and 4, detector algorithm of App. E): a 64-bit
+ *   watermark key, a 64-bit context label Lambda(c) and a 32-bit position.
+ * - `status` (nullable) is a device word the kernels OR flags into
+ *   (PPS_FLAG_*); clear it before the call if you read it.
+ *
+ * The keyed source (this library's reading; the paper fixes only a keyed
+ * pseudorandom function, Sec. 3.1 Eq. 1, and G(k, c), Alg. 3):
+ *   word w(i, j) of token i, arrival j >= 1 = lane (i & 3) of
+ *   Philox4x32-10(counter = (i >> 2, pos, ctx_lo, ctx_hi),
+ *                 key = (key_lo ^ (j - 1) * 0x9E3779B9, key_hi)),
+ *   u = (w + 1/2) 2^-32, E = -ln u ~ Exp(1) (first arrival, Thm A.1).
+ *   Race key of token i at temperature T: s_i = ln E_i - logit_i / T
+ *   (argmin s = argmin E/P, Alg. 2 and App. A.2); NaN logits never win.
+ *   Ties in s go to the smaller token index.
+ */
+#ifndef PPS_H
+#define PPS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* pps_stream_t; /* identical to cudaStream_t */
+
+typedef enum {
+    PPS_OK = 0,
+    PPS_ERR_INVALID_ARG = 1, /* null pointer, size out of range, K > vocab, stride < vocab, T <= 0 ... */
+    PPS_ERR_UNSUPPORTED = 2, /* dtype or mode not implemented                                        */
+    PPS_ERR_WORKSPACE = 3,   /* workspace null or smaller than pps_workspace_size()                    */
+    PPS_ERR_CUDA = 4         /* a kernel launch or CUDA call failed                                    */
+} pps_status;
+
+typedef enum { PPS_F32 = 0, PPS_BF16 = 1 } pps_dtype;
+
+typedef enum {
+    PPS_DRAFT_DISTINCT = 0, /* the K smallest first-arrival keys (K distinct tokens)                 */
+    PPS_DRAFT_IID = 1       /* the K smallest multi-arrival scores (direct finite-support MPFR, App. B) */
+} pps_draft_mode;
+
+/* per-row identities, each an array of n_rows (device) */
+typedef struct {
+    const uint64_t* key;      /* watermark key k                         */
+    const uint64_t* ctx_hash; /* context label Lambda(c)                 */
+    const uint32_t* pos;      /* position of the context                 */
+} pps_row_ids;
+
+/* bits OR-ed into *status */
+#define PPS_FLAG_GUARD 1u       /* fp32 streaming filter could not prove a row's candidate set complete */
+#define PPS_FLAG_LOGIT_RANGE 2u /* |logit / T| too large for the fp32 filter's error bound (> 2^16)      */
+
+#define PPS_MAX_K 32
+
+/* Library version string and a text for a status code (host pointers, static). */
+const char* pps_version(void);
+const char* pps_status_string(pps_status s);
+
+/* Bytes of workspace pps_draft_list / pps_verify_tree need for n_rows rows and
+ * n_seq sequences (n_seq = 0 for pps_draft_list).  The workspace holds
+ * per-row partial candidate lists and arrival counters; it must be zeroed once
+ * before its first use (pps_workspace_clear or cudaMemset) and is left zeroed
+ * by every call that returns PPS_OK and runs to completion.  One workspace
+ * must not be used by two calls that run concurrently. */
+size_t pps_workspace_size(int64_t n_rows, int64_t vocab, int32_t K, int32_t n_seq);
+pps_status pps_workspace_clear(void* ws, size_t ws_bytes, pps_stream_t stream);
+
+/*
+ * pps_draft_list -- the drafter's list at every context row (MPFR(Q(.|c),
+ * Pi(c), nu(c)), Eq. 4; direct finite-support MPFR algorithm and the draft
+ * side of the batched direct top-k algorithm, App. B; draft-tree step of
+ * Alg. 4).
+ *
+ * q_logits     [n_rows, row_stride] draft logits (dtype), row r = context c_r
+ * ids          identities of the n_rows contexts
+ * temperature  T > 0, applied as logit / T
+ * K            list stride and largest list length, 1 <= K <= min(32, vocab)
+ * row_k        nullable [n_rows]: list length nu(c_r) of each row, 1..K
+ *              (NULL = K for every row)
+ * mode         PPS_DRAFT_DISTINCT or PPS_DRAFT_IID
+ * out_tok      [n_rows, K] tokens of the k_r smallest first-arrival keys in
+ *              ascending key order; -1 past k_r or past the row's usable tokens
+ * out_key      nullable [n_rows, K] their keys s (fp32 estimate, natural log)
+ * out_mult     [n_rows, K] DISTINCT: 1 per valid entry; IID: how many of the
+ *              k_r samples carry the label out_tok[r, m]
+ * out_ndistinct [n_rows] |D(c_r)|, the number of distinct draft tokens; they
+ *              are out_tok[r, 0 .. out_ndistinct[r]-1] in both modes
+ * out_samples  nullable [n_rows, K] the ordered samples (DISTINCT: = out_tok;
+ *              IID: labels of the k_r smallest multi-arrival scores)
+ * ws, ws_bytes workspace of pps_workspace_size(n_rows, vocab, K, 0) bytes
+ */
+pps_status pps_draft_list(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t row_stride,
+                          pps_row_ids ids, float temperature, int32_t K, const int32_t* row_k, pps_draft_mode mode,
+                          int32_t* out_tok, float* out_key, int32_t* out_mult, int32_t* out_ndistinct,
+                          int32_t* out_samples, uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream);
+
+/*
+ * pps_verify_tree -- target race at every node of the draft trees, then the
+ * walk along the realised target path with the watermark score of every
+ * emitted token (batched-target evaluation and "follow the realised target
+ * path" of the batched direct top-k algorithm, App. B; Alg. 4; score Eq. 2).
+ *
+ * p_logits     [n_nodes, row_stride] target logits, one row per tree node
+ * ids          identities of the n_nodes contexts (the same labels the draft
+ *              rows of those contexts used)
+ * n_seq, gamma sequences and block length (1 <= gamma <= 64)
+ * seq_off      [n_seq+1] sequence b owns nodes seq_off[b] .. seq_off[b+1]-1,
+ *              its root is node seq_off[b] (non-decreasing, seq_off[0] = 0,
+ *              seq_off[n_seq] = n_nodes)
+ * node_draft_row [n_nodes] draft row of node c, -1 for a leaf
+ * n_draft      number of draft rows
+ * draft_tok, draft_ndistinct  pps_draft_list outputs for the draft rows
+ *              ([n_draft, K], [n_draft]); D(c) = draft_tok[dr, 0..ndist-1]
+ *              The walk treats a draft row outside [0, n_draft) as a leaf, a
+ *              child outside [0, n_nodes) as not evaluated, and clamps ndist
+ *              to K, so an inconsistent tree cannot make it read out of bounds;
+ *              every sequence must own at least its root node, otherwise its
+ *              outputs are not written.
+ * K            stride of draft_tok and child_node
+ * child_node   [n_draft, K] node reached from draft row dr by list slot m
+ *              (the context c || draft_tok[dr, m]); -1 = not evaluated
+ * out_winner   [n_nodes] y(c) = argmin_i s_i, -1 if no token is usable
+ * out_word     [n_nodes] first-arrival word of y(c) (0 if none)
+ * out_accept_len [n_seq] accepted steps (0..gamma)
+ * out_n_emitted  [n_seq] emitted tokens (accept_len + 1, unless a winner was -1)
+ * out_emitted  [n_seq, gamma+1] emitted tokens, -1 past the end
+ * out_score    [n_seq, gamma+1] A = -ln(1 - u_y) of each emitted token, 0 past the end
+ * out_score_sum [n_seq] sum of A (fp64)
+ * ws, ws_bytes workspace of pps_workspace_size(n_nodes, vocab, 1, n_seq) bytes
+ */
+pps_status pps_verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_nodes, int64_t vocab, int64_t row_stride,
+                           pps_row_ids ids, float temperature, int32_t n_seq, int32_t gamma, const int32_t* seq_off,
+                           const int32_t* node_draft_row, int64_t n_draft, const int32_t* draft_tok,
+                           const int32_t* draft_ndistinct, int32_t K, const int32_t* child_node, int32_t* out_winner, uint32_t* out_word,
+                           int32_t* out_accept_len, int32_t* out_n_emitted, int32_t* out_emitted, float* out_score,
+                           double* out_score_sum, uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream);
+
+/*
+ * pps_wm_score -- detector pass (detector algorithm of App. E; Eq. 2):
+ * regenerate the first-arrival word of every observed token under its
+ * context's identity and score it, A_t = -ln(1 - u_t).
+ *
+ * tokens       [n] observed tokens (0 <= token < 2^34)
+ * ids          [n] identity of the context each token was emitted in
+ * n_seg, seg_off  nullable seg_off [n_seg+1]: segment g = tokens
+ *              seg_off[g] .. seg_off[g+1]-1 (non-decreasing, seg_off[0] = 0,
+ *              seg_off[n_seg] = n); NULL = one segment of all n tokens
+ * out_score    nullable [n] A_t (fp32)
+ * out_sum      nullable [n_seg] (or [1]) S_A per segment (fp64); zeroed by the call
+ */
+pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,
+                        float* out_score, double* out_sum, pps_stream_t stream);
+
+/* Raw words w(i, arrival) for i < vocab of n_rows rows -> out [n_rows, vocab]
+ * (bit-exact check of the keyed source). */
+pps_status pps_philox_words(pps_row_ids ids, int64_t n_rows, int64_t vocab, int32_t arrival, uint32_t* out,
+                            pps_stream_t stream);
+
+/* Self-test of the fp32 key transform used by the streaming filter: over
+ * every 32-bit word w in [w_begin, w_end) it compares the fp32 value of
+ * log2(-log2 u(w)) with an fp64 evaluation and writes the largest absolute
+ * difference to out_max_err[0] (device float, must hold 0 before the call). */
+pps_status pps_selftest_key_error(uint64_t w_begin, uint64_t w_end, float* out_max_err, pps_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PPS_H */

@@ -1,0 +1,190 @@
+// pps_api.cu -- extern "C" entry points of libpps: argument validation,
+// workspace layout and launches.  Every entry point returns before launching
+// anything when an argument is invalid.
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+
+#include "pps.h"
+#include "pps_internal.h"
+
+namespace pps {
+
+static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+size_t workspace_bytes(int64_t n_rows, int32_t n_seq) {
+    return align256(sizeof(Partial) * (size_t)(n_rows + kGridMax)) + align256(sizeof(uint32_t) * (size_t)n_rows) +
+           align256(sizeof(uint32_t) * (size_t)(n_seq > 0 ? n_seq : 0));
+}
+
+void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials, uint32_t** row_cnt,
+                     uint32_t** seq_cnt) {
+    char* p = static_cast<char*>(ws);
+    *partials = reinterpret_cast<Partial*>(p);
+    p += align256(sizeof(Partial) * (size_t)(n_rows + kGridMax));
+    *row_cnt = reinterpret_cast<uint32_t*>(p);
+    p += align256(sizeof(uint32_t) * (size_t)n_rows);
+    *seq_cnt = reinterpret_cast<uint32_t*>(p);
+}
+
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+static pps_status check_rows(const void* logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t stride,
+                             const pps_row_ids& ids, float T) {
+    if (dtype != PPS_F32 && dtype != PPS_BF16) return PPS_ERR_UNSUPPORTED;
+    if (n_rows < 0 || vocab < 1 || vocab > (int64_t(1) << 31) - 1 || stride < vocab) return PPS_ERR_INVALID_ARG;
+    if (n_rows > 0 && (!logits || !ids.key || !ids.ctx_hash || !ids.pos)) return PPS_ERR_INVALID_ARG;
+    if (!(T > 0.0f) || !std::isfinite(T)) return PPS_ERR_INVALID_ARG;
+    return PPS_OK;
+}
+
+static bool vec_ok(const void* logits, pps_dtype dtype, int64_t stride) {
+    size_t esz = dtype == PPS_BF16 ? 2 : 4;
+    return aligned16(logits) && ((size_t)stride * esz) % 16 == 0;
+}
+
+static RaceArgs base_args(const void* logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t stride,
+                          const pps_row_ids& ids, float T) {
+    RaceArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.logits = logits;
+    a.n_rows = n_rows;
+    a.V = vocab;
+    a.stride = stride;
+    a.key = ids.key;
+    a.ctx = ids.ctx_hash;
+    a.pos = ids.pos;
+    a.T = T;
+    a.c = (float)(1.4426950408889634074 / (double)T);
+    int vw = dtype == PPS_BF16 ? 8 : 4;
+    a.nv = (vocab + vw - 1) / vw;
+    a.total = n_rows * a.nv;
+    return a;
+}
+
+}  // namespace pps
+
+using namespace pps;
+
+extern "C" {
+
+const char* pps_version(void) { return "libpps 0.1 (sm_103a)"; }
+
+const char* pps_status_string(pps_status s) {
+    switch (s) {
+        case PPS_OK: return "ok";
+        case PPS_ERR_INVALID_ARG: return "invalid argument";
+        case PPS_ERR_UNSUPPORTED: return "unsupported dtype or mode";
+        case PPS_ERR_WORKSPACE: return "workspace missing or too small";
+        case PPS_ERR_CUDA: return "CUDA launch failed";
+    }
+    return "unknown status";
+}
+
+size_t pps_workspace_size(int64_t n_rows, int64_t vocab, int32_t K, int32_t n_seq) {
+    (void)vocab;
+    (void)K;
+    if (n_rows < 0) n_rows = 0;
+    return workspace_bytes(n_rows, n_seq);
+}
+
+pps_status pps_workspace_clear(void* ws, size_t ws_bytes, pps_stream_t stream) {
+    if (!ws && ws_bytes) return PPS_ERR_INVALID_ARG;
+    if (ws_bytes == 0) return PPS_OK;
+    return cudaMemsetAsync(ws, 0, ws_bytes, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_draft_list(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t row_stride,
+                          pps_row_ids ids, float temperature, int32_t K, const int32_t* row_k, pps_draft_mode mode,
+                          int32_t* out_tok, float* out_key, int32_t* out_mult, int32_t* out_ndistinct,
+                          int32_t* out_samples, uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream) {
+    pps_status st = check_rows(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature);
+    if (st != PPS_OK) return st;
+    if (mode != PPS_DRAFT_DISTINCT && mode != PPS_DRAFT_IID) return PPS_ERR_UNSUPPORTED;
+    if (K < 1 || K > PPS_MAX_K || K > vocab) return PPS_ERR_INVALID_ARG;
+    if (n_rows == 0) return PPS_OK;
+    if (!out_tok || !out_mult || !out_ndistinct) return PPS_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < workspace_bytes(n_rows, 0)) return PPS_ERR_WORKSPACE;
+    RaceArgs a = base_args(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature);
+    a.K = K;
+    a.row_k = row_k;
+    a.iid = mode == PPS_DRAFT_IID;
+    a.out_tok = out_tok;
+    a.out_key = out_key;
+    a.out_mult = out_mult;
+    a.out_nd = out_ndistinct;
+    a.out_samples = out_samples;
+    a.status = status;
+    workspace_carve(ws, n_rows, 0, &a.partials, &a.row_cnt, &a.seq_cnt);
+    const int dt = dtype == PPS_BF16 ? 1 : 0;
+    const bool vec = vec_ok(q_logits, dtype, row_stride);
+    a.G = race_grid(a.total, dt, false, vec);
+    return launch_race(a, dt, false, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_nodes, int64_t vocab, int64_t row_stride,
+                           pps_row_ids ids, float temperature, int32_t n_seq, int32_t gamma, const int32_t* seq_off,
+                           const int32_t* node_draft_row, int64_t n_draft, const int32_t* draft_tok,
+                           const int32_t* draft_ndistinct, int32_t K, const int32_t* child_node, int32_t* out_winner, uint32_t* out_word,
+                           int32_t* out_accept_len, int32_t* out_n_emitted, int32_t* out_emitted, float* out_score,
+                           double* out_score_sum, uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream) {
+    pps_status st = check_rows(p_logits, dtype, n_nodes, vocab, row_stride, ids, temperature);
+    if (st != PPS_OK) return st;
+    if (n_seq < 0 || gamma < 1 || gamma > 64 || K < 1 || K > PPS_MAX_K || n_draft < 0) return PPS_ERR_INVALID_ARG;
+    if (n_nodes == 0 || n_seq == 0) return n_nodes == 0 && n_seq == 0 ? PPS_OK : PPS_ERR_INVALID_ARG;
+    if (n_nodes < n_seq) return PPS_ERR_INVALID_ARG;
+    if (!seq_off || !node_draft_row || !draft_tok || !draft_ndistinct || !child_node || !out_winner || !out_word ||
+        !out_accept_len || !out_n_emitted || !out_emitted || !out_score || !out_score_sum)
+        return PPS_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < workspace_bytes(n_nodes, n_seq)) return PPS_ERR_WORKSPACE;
+    RaceArgs a = base_args(p_logits, dtype, n_nodes, vocab, row_stride, ids, temperature);
+    a.K = 1;
+    a.n_seq = n_seq;
+    a.gamma = gamma;
+    a.seq_off = seq_off;
+    a.node_draft_row = node_draft_row;
+    a.n_draft = n_draft;
+    a.draft_tok = draft_tok;
+    a.draft_nd = draft_ndistinct;
+    a.Kd = K;
+    a.child_node = child_node;
+    a.out_winner = out_winner;
+    a.out_word = out_word;
+    a.out_acc = out_accept_len;
+    a.out_ne = out_n_emitted;
+    a.out_em = out_emitted;
+    a.out_sc = out_score;
+    a.out_ss = out_score_sum;
+    a.status = status;
+    workspace_carve(ws, n_nodes, n_seq, &a.partials, &a.row_cnt, &a.seq_cnt);
+    const int dt = dtype == PPS_BF16 ? 1 : 0;
+    const bool vec = vec_ok(p_logits, dtype, row_stride);
+    a.G = race_grid(a.total, dt, true, vec);
+    return launch_race(a, dt, true, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,
+                        float* out_score, double* out_sum, pps_stream_t stream) {
+    if (n < 0) return PPS_ERR_INVALID_ARG;
+    if (seg_off && n_seg < 1) return PPS_ERR_INVALID_ARG;
+    if (n > 0 && (!tokens || !ids.key || !ids.ctx_hash || !ids.pos)) return PPS_ERR_INVALID_ARG;
+    if (!out_score && !out_sum) return PPS_ERR_INVALID_ARG;
+    cudaError_t e = launch_wm_score(tokens, ids.key, ids.ctx_hash, ids.pos, n, seg_off ? n_seg : 1, seg_off, out_score,
+                                    out_sum, (cudaStream_t)stream);
+    return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_philox_words(pps_row_ids ids, int64_t n_rows, int64_t vocab, int32_t arrival, uint32_t* out,
+                            pps_stream_t stream) {
+    if (n_rows < 0 || vocab < 1 || arrival < 1) return PPS_ERR_INVALID_ARG;
+    if (n_rows > 0 && (!ids.key || !ids.ctx_hash || !ids.pos || !out)) return PPS_ERR_INVALID_ARG;
+    cudaError_t e = launch_words(ids.key, ids.ctx_hash, ids.pos, n_rows, vocab, arrival, out, (cudaStream_t)stream);
+    return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_selftest_key_error(uint64_t w_begin, uint64_t w_end, float* out_max_err, pps_stream_t stream) {
+    if (!out_max_err || w_end > (uint64_t(1) << 32) || w_begin > w_end) return PPS_ERR_INVALID_ARG;
+    return launch_selftest(w_begin, w_end, out_max_err, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,217 @@
+// pps_device.cuh -- device primitives of the keyed Poisson race (sm_103a).
+//
+// Keyed source: Philox4x32-10 (Salmon et al., SC'11) evaluated in registers,
+// one block of four 32-bit words per four consecutive tokens.  Counter
+// (token >> 2, pos, ctx_lo, ctx_hi), key (key_lo ^ (j-1) * 0x9E3779B9, key_hi)
+// for arrival j; the word of token i is lane i & 3.  u = (w + 1/2) 2^-32,
+// E = -ln u (first arrival scaled to Exp(1), Thm A.1).
+//
+// Keys.  The streaming kernels order tokens by the fp32 key
+//     k(i) = log2(-log2 u_i) - logit_i * log2(e) / T
+//          = log2(e) * (ln E_i - logit_i / T) + log2(log2 e),
+// an increasing affine map of the paper's race key s = ln E - l/T (Alg. 2,
+// App. A.2), so the order and the argmin are the same.  The fp32 value carries
+// an error bounded by key_err_bound(); pairs closer than the sum of their
+// bounds are re-ordered with the fp64 key s.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace pps {
+
+constexpr uint32_t kPhiloxM0 = 0xD2511F53u;
+constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;
+constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;
+constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr double kLn2 = 0.69314718055994530942;
+// log2(ln 2): converts the filter bound E < 2^(theta + l c) ln 2 into base-2 exponents
+constexpr float kLog2Ln2 = -0.52876637294589f;
+// bound on |k_fp32 - k_exact| is kErrAbs + kErrRel * (|k| + kErrSpan); the
+// self-test measures the transform part (largest |x32 - x64| over all 2^32 words)
+constexpr float kErrAbs = 3.0e-6f;
+constexpr float kErrRel = 1.2e-7f;  // ~2^-23: rounding of c = log2(e)/T and of the fused multiply-add
+constexpr float kErrSpan = 40.0f;   // |log2(-log2 u)| <= 34.9 for every 32-bit word
+// the filter may only drop a token whose fp32 key is >= theta; it tests
+// E >= v with theta raised by this margin (log2 units), which covers the
+// approximate ex2, the rounding of z and the key error for |theta| < 2^16
+constexpr float kFilterMargin = 0.015625f;
+
+__device__ __forceinline__ float key_err_bound(float k) { return kErrAbs + kErrRel * (fabsf(k) + kErrSpan); }
+
+// ------------------------------------------------------------------ Philox
+
+__device__ __forceinline__ void mulhilo(uint32_t a, uint32_t b, uint32_t& hi, uint32_t& lo) {
+    uint64_t p = (uint64_t)a * (uint64_t)b;
+    hi = (uint32_t)(p >> 32);
+    lo = (uint32_t)p;
+}
+
+// full Philox4x32-10 on counter (x0..x3), key (k0, k1)
+__device__ __forceinline__ uint4 philox(uint32_t x0, uint32_t x1, uint32_t x2, uint32_t x3, uint32_t k0, uint32_t k1) {
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        if (r) {
+            k0 += kPhiloxW0;
+            k1 += kPhiloxW1;
+        }
+        uint32_t hi0, lo0, hi1, lo1;
+        mulhilo(kPhiloxM0, x0, hi0, lo0);
+        mulhilo(kPhiloxM1, x2, hi1, lo1);
+        uint32_t y0 = hi1 ^ x1 ^ k0, y2 = hi0 ^ x3 ^ k1;
+        x0 = y0;
+        x1 = lo1;
+        x2 = y2;
+        x3 = lo0;
+    }
+    return make_uint4(x0, x1, x2, x3);
+}
+
+__device__ __forceinline__ uint32_t lane_of(uint4 v, uint32_t lane) {
+    return lane == 0 ? v.x : lane == 1 ? v.y : lane == 2 ? v.z : v.w;
+}
+
+// word of token i, arrival j (generic path: epilogues, helpers)
+__device__ __forceinline__ uint32_t word_of(uint64_t key, uint64_t ctx, uint32_t pos, int64_t i, int j) {
+    uint32_t k0 = (uint32_t)key ^ ((uint32_t)(j - 1) * kPhiloxW0);
+    uint4 b = philox((uint32_t)((uint64_t)i >> 2), pos, (uint32_t)ctx, (uint32_t)(ctx >> 32), k0, (uint32_t)(key >> 32));
+    return lane_of(b, (uint32_t)(i & 3));
+}
+
+// Row-specialised Philox for the streaming loop (first arrival, fixed row).
+// Only counter word 0 (token >> 2) varies along a row, so the products of
+// the constant words in rounds 1-2 are hoisted per row: round 1 needs one
+// multiply, round 2 one multiply, rounds 3-10 the usual two.
+struct RowPhilox {
+    uint32_t r1_c3k;     // ctx_hi ^ key_hi                         (round 1, word 2)
+    uint32_t r2_hi0;     // hi(M0 * y0) with y0 = hi(M1*ctx_lo) ^ pos ^ k0   (round 2)
+    uint32_t r2_f;       // lo(M1 * ctx_lo) ^ (k0 + W0)             (round 2, word 0 xor term)
+    uint32_t r2_g;       // k1 + W1                                 (round 2, word 2 xor term)
+    uint32_t r2_lo0;     // lo(M0 * y0)                             (round 2, word 3)
+    uint32_t rk0[8], rk1[8];  // keys of rounds 3..10
+
+    __device__ __forceinline__ void init(uint64_t key, uint64_t ctx, uint32_t pos) {
+        uint32_t k0 = (uint32_t)key, k1 = (uint32_t)(key >> 32);
+        uint32_t c2 = (uint32_t)ctx, c3 = (uint32_t)(ctx >> 32);
+        uint32_t hi1, lo1;
+        mulhilo(kPhiloxM1, c2, hi1, lo1);
+        uint32_t y0 = hi1 ^ pos ^ k0;  // round-1 word 0
+        r1_c3k = c3 ^ k1;
+        uint32_t hi, lo;
+        mulhilo(kPhiloxM0, y0, hi, lo);
+        r2_hi0 = hi;
+        r2_lo0 = lo;
+        r2_f = lo1 ^ (k0 + kPhiloxW0);
+        r2_g = k1 + kPhiloxW1;
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+            rk0[r] = k0 + (uint32_t)(r + 2) * kPhiloxW0;
+            rk1[r] = k1 + (uint32_t)(r + 2) * kPhiloxW1;
+        }
+    }
+
+    // the four words of block c0 (tokens 4*c0 .. 4*c0+3)
+    __device__ __forceinline__ uint4 block(uint32_t c0) const {
+        uint32_t hi0, lo0;
+        mulhilo(kPhiloxM0, c0, hi0, lo0);
+        // round 1: (y0, y1) constant, y2 = hi0 ^ c3 ^ k1, y3 = lo0
+        uint32_t y2 = hi0 ^ r1_c3k;
+        uint32_t y3 = lo0;
+        // round 2: M0*y0 constant
+        uint32_t h1, l1;
+        mulhilo(kPhiloxM1, y2, h1, l1);
+        uint32_t x0 = h1 ^ r2_f;
+        uint32_t x1 = l1;
+        uint32_t x2 = r2_hi0 ^ y3 ^ r2_g;
+        uint32_t x3 = r2_lo0;
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+            uint32_t a0, b0, a1, b1;
+            mulhilo(kPhiloxM0, x0, a0, b0);
+            mulhilo(kPhiloxM1, x2, a1, b1);
+            uint32_t n0 = a1 ^ x1 ^ rk0[r], n2 = a0 ^ x3 ^ rk1[r];
+            x0 = n0;
+            x1 = b1;
+            x2 = n2;
+            x3 = b0;
+        }
+        return make_uint4(x0, x1, x2, x3);
+    }
+};
+
+// ------------------------------------------------------------------ transforms
+
+// y = -log2 u = E log2(e), accurate fp32 (u <= 1/2 through u, u > 1/2 through v = 1-u)
+__device__ __forceinline__ float neg_log2_u(uint32_t w) {
+    if (w < 0x80000000u) {
+        float u = fmaf((float)w, 0x1p-32f, 0x1p-33f);
+        return -log2f(u);
+    }
+    float v = fmaf((float)(~w), 0x1p-32f, 0x1p-33f);
+    return -log1pf(-v) * kLog2e;
+}
+
+// x = log2(-log2 u), the word part of the fp32 key
+__device__ __forceinline__ float key_x32(uint32_t w) { return log2f(neg_log2_u(w)); }
+
+// fp32 key k = x - l * c with c = log2(e) / T; NaN logits map to +inf
+__device__ __forceinline__ float key32(uint32_t w, float l, float c) {
+    float k = fmaf(-l, c, key_x32(w));
+    return k != k ? __int_as_float(0x7f800000) : k;
+}
+
+// fp64 race key s = ln E - l / T (the paper's definition, used for near-ties)
+__device__ __forceinline__ double exp1_f64(uint32_t w) {
+    if (w < 0x80000000u) return -log(((double)w + 0.5) * 0x1p-32);
+    return -log1p(-(((double)(~w) + 0.5) * 0x1p-32));
+}
+__device__ __forceinline__ double key64(uint32_t w, float l, float T) {
+    double ld = (double)l;
+    if (ld != ld) return __longlong_as_double(0x7ff0000000000000ll);
+    return log(exp1_f64(w)) - ld / (double)T;
+}
+
+// Aaronson score A = -ln(1 - u) (Eq. 2), fp64 and accurate fp32
+__device__ __forceinline__ double score64(uint32_t w) {
+    if (w < 0x80000000u) return -log1p(-(((double)w + 0.5) * 0x1p-32));
+    return -log(((double)(~w) + 0.5) * 0x1p-32);
+}
+__device__ __forceinline__ float score32(uint32_t w) {
+    if (w < 0x80000000u) return -log1pf(-fmaf((float)w, 0x1p-32f, 0x1p-33f));
+    return -logf(fmaf((float)(~w), 0x1p-32f, 0x1p-33f));
+}
+
+// fp32 key (log2 units, shifted) -> s (natural log units)
+__device__ __forceinline__ float key_to_s(float k) { return (k + 0.52876637294589f) * 0.69314718055994530942f; }
+
+// ------------------------------------------------------------------ filter
+//
+// A token can enter a list only if its fp32 key is below theta.  Since
+// E = -ln(1 - v) >= v with v = 1 - u = (~w + 1/2) 2^-32, a key below theta
+// needs v < e_z := 2^(theta + l c) ln 2.  With a = (~w) >> 9 that holds only if
+// a <= round(2^(theta + margin + l c + log2(ln 2) + 23)).  tz carries
+// theta + margin + log2(ln 2) + 23 (+inf while the list is not full).
+// The comparison is done on float bit patterns: 2^23 + a has the bits
+// 0x4b000000 | a, and T + 2^23 rounds T to an integer in the low bits for
+// T < 2^23 (and is larger than every 0x4b000000 | a otherwise).
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ bool filter_pass(uint32_t w, float l, float c, float tz) {
+    float T = ex2_approx(fmaf(l, c, tz));
+    uint32_t tb = __float_as_uint(T + 8388608.0f);
+    uint32_t ab = (~(w >> 9) & 0x007fffffu) | 0x4b000000u;
+    return ab <= tb;
+}
+__device__ __forceinline__ float filter_tz(float theta) {
+    return theta + (kFilterMargin + kLog2Ln2 + 23.0f);
+}
+
+// bf16 -> fp32 (exact)
+__device__ __forceinline__ float bf16_lo(uint32_t x) { return __uint_as_float(x << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t x) { return __uint_as_float(x & 0xffff0000u); }
+
+}  // namespace pps

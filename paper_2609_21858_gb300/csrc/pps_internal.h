@@ -1,0 +1,82 @@
+// pps_internal.h -- host/device structures shared by the libpps translation units.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace pps {
+
+constexpr int kThreads = 256;           // threads per CTA of the streaming kernels
+constexpr int kWarps = kThreads / 32;
+constexpr int kGridMax = 4096;          // upper bound on the streaming grid (sizes the workspace)
+constexpr int64_t kMinVecsPerCta = 2048;  // 16-byte vectors per CTA below which the grid shrinks
+
+// one partial candidate list of a row segment (sorted ascending by (key, idx))
+struct alignas(16) Partial {
+    float key[32];
+    int32_t idx[32];
+    float theta_drop;  // every token of the segment left out has an fp32 key >= theta_drop
+    int32_t n;
+    int32_t pad[2];
+};
+
+struct RaceArgs {
+    const void* logits;
+    int64_t n_rows, V, stride;
+    const uint64_t* key;
+    const uint64_t* ctx;
+    const uint32_t* pos;
+    float T;  // temperature
+    float c;  // log2(e) / T
+    // draft side
+    int K;
+    const int32_t* row_k;
+    int iid;
+    int32_t* out_tok;
+    float* out_key;
+    int32_t* out_mult;
+    int32_t* out_nd;
+    int32_t* out_samples;
+    // target side + walk
+    int n_seq, gamma;
+    const int32_t* seq_off;
+    const int32_t* node_draft_row;
+    int64_t n_draft;
+    const int32_t* draft_tok;
+    const int32_t* draft_nd;
+    int Kd;
+    const int32_t* child_node;
+    int32_t* out_winner;
+    uint32_t* out_word;
+    int32_t* out_acc;
+    int32_t* out_ne;
+    int32_t* out_em;
+    float* out_sc;
+    double* out_ss;
+    uint32_t* status;
+    // partition of the flattened (row, vector) range over the grid
+    int64_t nv;     // 16-byte vectors per row (last one may be partial)
+    int64_t total;  // n_rows * nv
+    int G;
+    // workspace
+    Partial* partials;   // [n_rows + kGridMax]
+    uint32_t* row_cnt;   // [n_rows]
+    uint32_t* seq_cnt;   // [n_seq]
+};
+
+size_t workspace_bytes(int64_t n_rows, int32_t n_seq);
+void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials, uint32_t** row_cnt,
+                     uint32_t** seq_cnt);
+
+// launchers (pps_race.cu)
+cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
+int race_grid(int64_t total, int dtype, bool verify, bool vec);
+
+// launchers (pps_misc.cu)
+cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
+                            int64_t n, int32_t n_seg, const int64_t* seg_off, float* out_score, double* out_sum,
+                            cudaStream_t stream);
+cudaError_t launch_words(const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int64_t n_rows, int64_t V,
+                         int32_t arrival, uint32_t* out, cudaStream_t stream);
+cudaError_t launch_selftest(uint64_t w_begin, uint64_t w_end, float* out, cudaStream_t stream);
+
+}  // namespace pps

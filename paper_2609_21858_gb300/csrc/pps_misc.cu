@@ -1,0 +1,162 @@
+// pps_misc.cu -- detector pass, raw keyed words, and the fp32 key self-test.
+#include <climits>
+#include <cstdint>
+
+#include "pps_device.cuh"
+#include "pps_internal.h"
+
+namespace pps {
+
+#define FULL 0xffffffffu
+
+// Detector (App. E): every warp takes a contiguous chunk of tokens; lane t of
+// an iteration scores token base + t.  Segment sums: a segmented warp scan
+// over the 32 consecutive tokens of an iteration, with the open segment
+// carried to the next iteration, so a warp issues one fp64 atomic per
+// segment end it sees (plus one at the end of its chunk).
+constexpr int kScoreChunk = 32 * 64;
+
+__global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict__ tokens,
+                                                       const uint64_t* __restrict__ key,
+                                                       const uint64_t* __restrict__ ctx,
+                                                       const uint32_t* __restrict__ pos, int64_t n, int32_t n_seg,
+                                                       const int64_t* __restrict__ seg_off, float* out_score,
+                                                       double* out_sum) {
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t c0 = gw * kScoreChunk;
+    if (c0 >= n) return;
+    const int64_t c1 = min(n, c0 + (int64_t)kScoreChunk);
+    // segment of the chunk's first token (binary search, lane 0)
+    int seg = 0;
+    if (out_sum && seg_off) {
+        if (lane == 0) {
+            int lo = 0, hi = n_seg;  // seg_off[lo] <= c0 < seg_off[hi]
+            while (hi - lo > 1) {
+                int mid = (lo + hi) >> 1;
+                if (seg_off[mid] <= c0)
+                    lo = mid;
+                else
+                    hi = mid;
+            }
+            seg = lo;
+        }
+        seg = __shfl_sync(FULL, seg, 0);
+    }
+    double carry = 0.0;  // running sum of the open segment `seg` (warp-uniform)
+    for (int64_t base = c0; base < c1; base += 32) {
+        const int64_t t = base + lane;
+        float A = 0.0f;
+        if (t < c1) {
+            int64_t tok = tokens[t];
+            A = score32(word_of(key[t], ctx[t], pos[t], tok, 1));
+            if (out_score) out_score[t] = A;
+        }
+        if (!out_sum) continue;
+        if (!seg_off) {
+            double v = A;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
+            carry += v;
+            continue;
+        }
+        // segment of my token, advanced from the warp's open segment (segments are contiguous)
+        int my = INT_MAX;
+        if (t < c1) {
+            my = seg;
+            while (my + 1 < n_seg && seg_off[my + 1] <= t) ++my;
+        }
+        // segmented inclusive scan over the lanes of each segment run
+        double v = A;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            double ov = __shfl_up_sync(FULL, v, o);
+            int os = __shfl_up_sync(FULL, my, o);
+            if (lane >= o && os == my) v += ov;
+        }
+        // the carried segment ended before this iteration's first run: flush it
+        const int s0 = __shfl_sync(FULL, my, 0);
+        if (s0 != seg) {
+            if (lane == 0 && carry != 0.0) atomicAdd(out_sum + seg, carry);
+            carry = 0.0;
+            seg = s0;
+        }
+        const int nxt = __shfl_down_sync(FULL, my, 1);
+        const bool more = base + 32 < c1;
+        if (t < c1 && (lane == 31 || nxt != my)) {
+            const bool open = lane == 31 && more;  // may continue into the next iteration
+            if (!open) atomicAdd(out_sum + my, v + (my == seg ? carry : 0.0));
+        }
+        if (more) {
+            const double v31 = __shfl_sync(FULL, v, 31);
+            const int s31 = __shfl_sync(FULL, my, 31);
+            carry = v31 + (s31 == seg ? carry : 0.0);
+            seg = s31;
+        } else {
+            carry = 0.0;
+        }
+    }
+    if (out_sum && !seg_off && lane == 0) atomicAdd(out_sum, carry);
+}
+
+__global__ void words_kernel(const uint64_t* __restrict__ key, const uint64_t* __restrict__ ctx,
+                             const uint32_t* __restrict__ pos, int64_t n_rows, int64_t V, int32_t arrival,
+                             uint32_t* __restrict__ out) {
+    const int64_t total = n_rows * V;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
+        int64_t r = t / V, i = t - r * V;
+        out[t] = word_of(key[r], ctx[r], pos[r], i, arrival);
+    }
+}
+
+// largest |x32(w) - log2(-log2 u(w))| over a word range; the fp64 reference
+// uses E = -ln u through u for u <= 1/2 and through v = 1 - u above
+__global__ void selftest_kernel(uint64_t w0, uint64_t w1, float* out) {
+    float worst = 0.0f;
+    for (uint64_t w = w0 + (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; w < w1;
+         w += (uint64_t)gridDim.x * blockDim.x) {
+        uint32_t x = (uint32_t)w;
+        float x32 = key_x32(x);
+        double xd = log2(exp1_f64(x) * 1.4426950408889634074);
+        float d = (float)fabs((double)x32 - xd);
+        worst = fmaxf(worst, d);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) worst = fmaxf(worst, __shfl_xor_sync(FULL, worst, o));
+    if ((threadIdx.x & 31) == 0) atomicMax(reinterpret_cast<unsigned int*>(out), __float_as_uint(worst));
+}
+
+cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
+                            int64_t n, int32_t n_seg, const int64_t* seg_off, float* out_score, double* out_sum,
+                            cudaStream_t stream) {
+    if (out_sum) {
+        cudaError_t e = cudaMemsetAsync(out_sum, 0, sizeof(double) * (size_t)(seg_off ? n_seg : 1), stream);
+        if (e != cudaSuccess) return e;
+    }
+    if (n == 0) return cudaSuccess;
+    int64_t warps = (n + kScoreChunk - 1) / kScoreChunk;
+    int64_t blocks = (warps * 32 + 255) / 256;
+    wm_score_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, key, ctx, pos, n, n_seg, seg_off, out_score, out_sum);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_words(const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int64_t n_rows, int64_t V,
+                         int32_t arrival, uint32_t* out, cudaStream_t stream) {
+    int64_t total = n_rows * V;
+    if (total == 0) return cudaSuccess;
+    int64_t blocks = (total + 255) / 256;
+    if (blocks > 65535 * 8) blocks = 65535 * 8;
+    words_kernel<<<(unsigned)blocks, 256, 0, stream>>>(key, ctx, pos, n_rows, V, arrival, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_selftest(uint64_t w_begin, uint64_t w_end, float* out, cudaStream_t stream) {
+    if (w_end <= w_begin) return cudaSuccess;
+    uint64_t n = w_end - w_begin;
+    uint64_t blocks = (n + 255) / 256;
+    if (blocks > 152 * 64) blocks = 152 * 64;
+    selftest_kernel<<<(unsigned)blocks, 256, 0, stream>>>(w_begin, w_end, out);
+    return cudaGetLastError();
+}
+
+}  // namespace pps

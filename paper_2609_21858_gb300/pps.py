@@ -1,0 +1,213 @@
+"""ctypes binding of libpps (include/pps.h): same entry-point names, argument
+marshalling only.  Torch supplies device memory and the current stream; every
+step of the computation runs in the library's CUDA kernels.  There is no CPU
+fallback: a missing or unloadable libpps.so raises immediately.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libpps.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
+F32, BF16 = 0, 1
+DISTINCT, IID = 0, 1
+FLAG_GUARD, FLAG_LOGIT_RANGE = 1, 2
+MAX_K = 32
+
+_lock = threading.Lock()
+_lib = None
+
+
+class RowIds(ctypes.Structure):
+    _fields_ = [("key", ctypes.c_void_p), ("ctx_hash", ctypes.c_void_p), ("pos", ctypes.c_void_p)]
+
+
+class PPSError(RuntimeError):
+    def __init__(self, fn, code):
+        super().__init__(f"{fn} failed: {code} ({status_string(code)})")
+        self.code = code
+
+
+def lib():
+    """Load libpps.so (raises if it was not built)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(f"libpps.so not found at {LIB_PATH}; build it with "
+                                   "`python -c 'import __graft_entry__ as g; g.build()'`")
+            L = ctypes.CDLL(LIB_PATH)
+            vp, i64, i32, f32, u64, sz = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_float,
+                                          ctypes.c_uint64, ctypes.c_size_t)
+            L.pps_version.restype = ctypes.c_char_p
+            L.pps_status_string.argtypes = [ctypes.c_int]
+            L.pps_status_string.restype = ctypes.c_char_p
+            L.pps_workspace_size.argtypes = [i64, i64, i32, i32]
+            L.pps_workspace_size.restype = sz
+            L.pps_workspace_clear.argtypes = [vp, sz, vp]
+            L.pps_workspace_clear.restype = ctypes.c_int
+            L.pps_draft_list.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, i32, vp, ctypes.c_int,
+                                         vp, vp, vp, vp, vp, vp, vp, sz, vp]
+            L.pps_draft_list.restype = ctypes.c_int
+            L.pps_verify_tree.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, i32, i32, vp, vp, i64, vp,
+                                          vp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+            L.pps_verify_tree.restype = ctypes.c_int
+            L.pps_wm_score.argtypes = [vp, RowIds, i64, i32, vp, vp, vp, vp]
+            L.pps_wm_score.restype = ctypes.c_int
+            L.pps_philox_words.argtypes = [RowIds, i64, i64, i32, vp, vp]
+            L.pps_philox_words.restype = ctypes.c_int
+            L.pps_selftest_key_error.argtypes = [u64, u64, vp, vp]
+            L.pps_selftest_key_error.restype = ctypes.c_int
+            _lib = L
+    return _lib
+
+
+def version() -> str:
+    return lib().pps_version().decode()
+
+
+def status_string(code: int) -> str:
+    return lib().pps_status_string(int(code)).decode()
+
+
+def _check(fn, code):
+    if code != OK:
+        raise PPSError(fn, code)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return F32
+    raise TypeError(f"logits must be bfloat16 or float32, got {t.dtype}")
+
+
+def _ids(key, ctx, pos):
+    for name, t, dt in (("key", key, torch.int64), ("ctx", ctx, torch.int64), ("pos", pos, torch.int32)):
+        if not t.is_cuda or t.dtype != dt or not t.is_contiguous():
+            raise TypeError(f"{name} must be a contiguous CUDA {dt} tensor (bit pattern of the unsigned id)")
+    return RowIds(key.data_ptr(), ctx.data_ptr(), pos.data_ptr())
+
+
+def _rows(logits):
+    if not logits.is_cuda or logits.dim() != 2 or logits.stride(1) != 1:
+        raise TypeError("logits must be a 2-D CUDA tensor with unit stride along the vocabulary")
+    return logits.shape[0], logits.shape[1], logits.stride(0)
+
+
+def workspace_size(n_rows: int, vocab: int = 0, K: int = 1, n_seq: int = 0) -> int:
+    return int(lib().pps_workspace_size(n_rows, vocab, K, n_seq))
+
+
+def workspace(n_rows: int, n_seq: int = 0, device=None) -> torch.Tensor:
+    """A zeroed workspace (reusable across calls of the same or smaller size)."""
+    nb = workspace_size(n_rows, 0, 1, n_seq)
+    return torch.zeros(nb, dtype=torch.uint8, device=device or "cuda")
+
+
+def workspace_clear(ws: torch.Tensor, stream=None):
+    _check("pps_workspace_clear", lib().pps_workspace_clear(_ptr(ws), ws.numel(), _stream(stream)))
+
+
+def draft_list(q_logits, key, ctx, pos, K: int, row_k=None, mode: int = DISTINCT, temperature: float = 1.0,
+               ws=None, status=None, out=None, keys: bool = True, samples: bool = True, stream=None):
+    """pps_draft_list.  Returns dict(tok, key, mult, ndist, samples) of CUDA tensors."""
+    n, V, stride = _rows(q_logits)
+    dev = q_logits.device
+    if out is None:
+        out = dict(tok=torch.empty(n, K, dtype=torch.int32, device=dev),
+                   key=torch.empty(n, K, dtype=torch.float32, device=dev) if keys else None,
+                   mult=torch.empty(n, K, dtype=torch.int32, device=dev),
+                   ndist=torch.empty(n, dtype=torch.int32, device=dev),
+                   samples=torch.empty(n, K, dtype=torch.int32, device=dev) if samples else None)
+    if ws is None:
+        ws = workspace(n, 0, dev)
+    if row_k is not None and (row_k.dtype != torch.int32 or not row_k.is_cuda):
+        raise TypeError("row_k must be a CUDA int32 tensor")
+    code = lib().pps_draft_list(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
+                                float(temperature), int(K), _ptr(row_k), int(mode), _ptr(out["tok"]),
+                                _ptr(out.get("key")), _ptr(out["mult"]), _ptr(out["ndist"]), _ptr(out.get("samples")),
+                                _ptr(status), _ptr(ws), ws.numel(), _stream(stream))
+    _check("pps_draft_list", code)
+    return out
+
+
+def verify_tree(p_logits, key, ctx, pos, gamma: int, seq_off, node_draft_row, draft_tok, draft_ndist, child_node,
+                temperature: float = 1.0, ws=None, status=None, out=None, stream=None):
+    """pps_verify_tree.  Returns dict(winner, word, accept_len, n_emitted, emitted, score, score_sum)."""
+    n, V, stride = _rows(p_logits)
+    dev = p_logits.device
+    n_seq = seq_off.numel() - 1
+    K = draft_tok.shape[1]
+    W = gamma + 1
+    if out is None:
+        out = dict(winner=torch.empty(n, dtype=torch.int32, device=dev),
+                   word=torch.empty(n, dtype=torch.int32, device=dev),
+                   accept_len=torch.empty(n_seq, dtype=torch.int32, device=dev),
+                   n_emitted=torch.empty(n_seq, dtype=torch.int32, device=dev),
+                   emitted=torch.empty(n_seq, W, dtype=torch.int32, device=dev),
+                   score=torch.empty(n_seq, W, dtype=torch.float32, device=dev),
+                   score_sum=torch.empty(n_seq, dtype=torch.float64, device=dev))
+    if ws is None:
+        ws = workspace(n, n_seq, dev)
+    for name, t in (("seq_off", seq_off), ("node_draft_row", node_draft_row), ("draft_tok", draft_tok),
+                    ("draft_ndist", draft_ndist), ("child_node", child_node)):
+        if not t.is_cuda or t.dtype != torch.int32 or not t.is_contiguous():
+            raise TypeError(f"{name} must be a contiguous CUDA int32 tensor")
+    code = lib().pps_verify_tree(_ptr(p_logits), _dtype_code(p_logits), n, V, stride, _ids(key, ctx, pos),
+                                 float(temperature), n_seq, int(gamma), _ptr(seq_off), _ptr(node_draft_row),
+                                 draft_tok.shape[0], _ptr(draft_tok), _ptr(draft_ndist), int(K), _ptr(child_node), _ptr(out["winner"]),
+                                 _ptr(out["word"]), _ptr(out["accept_len"]), _ptr(out["n_emitted"]),
+                                 _ptr(out["emitted"]), _ptr(out["score"]), _ptr(out["score_sum"]), _ptr(status),
+                                 _ptr(ws), ws.numel(), _stream(stream))
+    _check("pps_verify_tree", code)
+    return out
+
+
+def wm_score(tokens, key, ctx, pos, seg_off=None, out_score=None, out_sum=None, want_scores=True, stream=None):
+    """pps_wm_score.  Returns (scores or None, sums)."""
+    n = tokens.numel()
+    dev = tokens.device
+    n_seg = seg_off.numel() - 1 if seg_off is not None else 1
+    if out_score is None and want_scores:
+        out_score = torch.empty(n, dtype=torch.float32, device=dev)
+    if out_sum is None:
+        out_sum = torch.empty(n_seg, dtype=torch.float64, device=dev)
+    if tokens.dtype != torch.int32 or not tokens.is_cuda:
+        raise TypeError("tokens must be a CUDA int32 tensor")
+    if seg_off is not None and (seg_off.dtype != torch.int64 or not seg_off.is_cuda):
+        raise TypeError("seg_off must be a CUDA int64 tensor")
+    code = lib().pps_wm_score(_ptr(tokens), _ids(key, ctx, pos), n, n_seg, _ptr(seg_off), _ptr(out_score),
+                              _ptr(out_sum), _stream(stream))
+    _check("pps_wm_score", code)
+    return out_score, out_sum
+
+
+def philox_words(key, ctx, pos, vocab: int, arrival: int = 1, stream=None):
+    n = key.numel()
+    out = torch.empty(n, vocab, dtype=torch.int32, device=key.device)
+    _check("pps_philox_words", lib().pps_philox_words(_ids(key, ctx, pos), n, vocab, arrival, _ptr(out),
+                                                      _stream(stream)))
+    return out
+
+
+def selftest_key_error(w_begin: int = 0, w_end: int = 1 << 32, stream=None) -> float:
+    out = torch.zeros(1, dtype=torch.float32, device="cuda")
+    _check("pps_selftest_key_error", lib().pps_selftest_key_error(w_begin, w_end, _ptr(out), _stream(stream)))
+    return float(out.item())

@@ -1,0 +1,90 @@
+"""C-ABI checks that need no GPU: the library loads, exports every entry point
+include/pps.h declares, and rejects invalid arguments before launching anything."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_21858_gb300 import pps
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    txt = open(os.path.join(ROOT, "include", "pps.h")).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"\b(pps_[a-z0-9_]+)\s*\(", txt)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ("pps_draft_list", "pps_verify_tree", "pps_wm_score", "pps_workspace_size", "pps_philox_words"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol():
+    L = pps.lib()
+    for n in _declared():
+        assert hasattr(L, n), n
+    assert "sm_103a" in pps.version()
+
+
+def _ids0():
+    return pps.RowIds(None, None, None)
+
+
+def test_validation_rejects_bad_arguments_without_a_gpu():
+    L = pps.lib()
+    fake = ctypes.c_void_p(256)  # never dereferenced: every call below fails validation first
+    ids = pps.RowIds(256, 256, 256)
+    ws = 1 << 30
+
+    def draft(**kw):
+        a = dict(logits=fake, dtype=pps.BF16, n=4, V=100, stride=100, ids=ids, T=1.0, K=4, mode=pps.DISTINCT,
+                 tok=fake, mult=fake, nd=fake, ws=fake, wsb=ws)
+        a.update(kw)
+        return L.pps_draft_list(a["logits"], a["dtype"], a["n"], a["V"], a["stride"], a["ids"], a["T"], a["K"], None,
+                                a["mode"], a["tok"], None, a["mult"], a["nd"], None, None, a["ws"], a["wsb"], None)
+
+    assert draft(K=0) == pps.ERR_INVALID_ARG
+    assert draft(K=33) == pps.ERR_INVALID_ARG
+    assert draft(K=8, V=5, stride=5) == pps.ERR_INVALID_ARG
+    assert draft(stride=99) == pps.ERR_INVALID_ARG
+    assert draft(T=0.0) == pps.ERR_INVALID_ARG
+    assert draft(T=float("nan")) == pps.ERR_INVALID_ARG
+    assert draft(dtype=7) == pps.ERR_UNSUPPORTED
+    assert draft(mode=5) == pps.ERR_UNSUPPORTED
+    assert draft(ids=_ids0()) == pps.ERR_INVALID_ARG
+    assert draft(tok=None) == pps.ERR_INVALID_ARG
+    assert draft(ws=None) == pps.ERR_WORKSPACE
+    assert draft(wsb=16) == pps.ERR_WORKSPACE
+    assert draft(n=0) == pps.OK  # nothing to do, nothing launched
+
+    def verify(**kw):
+        a = dict(n=10, V=100, gamma=2, n_seq=2, K=2, ws=fake, wsb=ws, seq=fake)
+        a.update(kw)
+        return L.pps_verify_tree(fake, pps.F32, a["n"], a["V"], a["V"], ids, 1.0, a["n_seq"], a["gamma"], a["seq"],
+                                 fake, a.get("nd", 4), fake, fake, a["K"], fake, fake, fake, fake, fake, fake, fake, fake, None,
+                                 a["ws"], a["wsb"], None)
+
+    assert verify(gamma=0) == pps.ERR_INVALID_ARG
+    assert verify(gamma=65) == pps.ERR_INVALID_ARG
+    assert verify(n_seq=11) == pps.ERR_INVALID_ARG
+    assert verify(K=0) == pps.ERR_INVALID_ARG
+    assert verify(seq=None) == pps.ERR_INVALID_ARG
+    assert verify(nd=-1) == pps.ERR_INVALID_ARG
+    assert verify(wsb=0) == pps.ERR_WORKSPACE
+    assert L.pps_wm_score(fake, ids, -1, 1, None, fake, None, None) == pps.ERR_INVALID_ARG
+    assert L.pps_wm_score(fake, ids, 10, 1, None, None, None, None) == pps.ERR_INVALID_ARG
+    assert L.pps_wm_score(fake, ids, 10, 0, fake, fake, None, None) == pps.ERR_INVALID_ARG
+    assert L.pps_philox_words(ids, 1, 10, 0, fake, None) == pps.ERR_INVALID_ARG
+    assert L.pps_selftest_key_error(0, (1 << 32) + 1, fake, None) == pps.ERR_INVALID_ARG
+
+
+def test_workspace_size_grows_with_rows_and_sequences():
+    a = pps.workspace_size(100, 1000, 8, 0)
+    b = pps.workspace_size(200, 1000, 8, 0)
+    c = pps.workspace_size(200, 1000, 8, 50)
+    assert 0 < a < b <= c
+    assert pps.status_string(pps.ERR_WORKSPACE) == "workspace missing or too small"
