@@ -182,8 +182,8 @@ __device__ __forceinline__ float score32(uint32_t w) {
     return -logf(fmaf((float)(~w), 0x1p-32f, 0x1p-33f));
 }
 
-// fp32 key (log2 units, shifted) -> s (natural log units)
-__device__ __forceinline__ float key_to_s(float k) { return (k + 0.52876637294589f) * 0.69314718055994530942f; }
+// fp32 key k = log2(E) + log2(log2 e) - l log2(e)/T  ->  s = ln E - l/T = (k - log2(log2 e)) ln 2
+__device__ __forceinline__ float key_to_s(float k) { return (k + kLog2Ln2) * 0.69314718055994530942f; }
 
 // ------------------------------------------------------------------ filter
 //

@@ -81,11 +81,15 @@ __device__ __forceinline__ void warp_sort(float& k, int& i, int lane) {
     }
 }
 
-// merge a sorted list (lk, li) with a sorted batch (ok, oi); keep the kp smallest
-__device__ __forceinline__ void warp_merge(float& lk, int& li, float ok, int oi, int kp, int lane) {
+// merge a sorted list (lk, li) with a sorted batch (ok, oi); keep the kp smallest.
+// Returns (warp-uniform) the smallest key it discards: the (kp+1)-th of the union.
+template <bool TRACK>
+__device__ __forceinline__ float warp_merge(float& lk, int& li, float ok, int oi, int kp, int lane) {
     float rk = __shfl_sync(FULL, ok, 31 - lane);
     int ri = __shfl_sync(FULL, oi, 31 - lane);
+    float dropk = rk;
     if (lex_less(rk, ri, lk, li)) {
+        dropk = lk;
         lk = rk;
         li = ri;
     }
@@ -101,10 +105,16 @@ __device__ __forceinline__ void warp_merge(float& lk, int& li, float ok, int oi,
             li = xi;
         }
     }
+    if (TRACK) {
+        if (kp < 32) dropk = fminf(dropk, __shfl_sync(FULL, lk, kp & 31));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) dropk = fminf(dropk, __shfl_xor_sync(FULL, dropk, o));
+    }
     if (lane >= kp) {
         lk = kInf;
         li = INT_MAX;
     }
+    return dropk;
 }
 
 __device__ __forceinline__ void warp_sort_d(double& k, int& i, int lane) {
@@ -200,7 +210,7 @@ __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], in
             float ok = valid ? bk : kInf;
             int oi = valid ? bi : INT_MAX;
             warp_sort(ok, oi, lane);
-            warp_merge(L.lk, L.li, ok, oi, L.kp, lane);
+            warp_merge<false>(L.lk, L.li, ok, oi, L.kp, lane);
         }
         if (valid) {
 #pragma unroll
@@ -530,11 +540,12 @@ __global__ void __launch_bounds__(kThreads, 3) race_kernel(const RaceArgs a) {
             float lk = L.lk;
             int li = L.li;
             float theta_drop = s_theta[0];
+            // every token left out of the merged list has a key >= theta_drop: the warps
+            // dropped only keys >= their final kp-th key, the merges drop what they return
             for (int w = 1; w < kWarps; ++w) {
-                warp_merge(lk, li, s_key[w][lane], s_idx[w][lane], kp, lane);
-                theta_drop = fminf(theta_drop, s_theta[w]);
+                float dk = warp_merge<true>(lk, li, s_key[w][lane], s_idx[w][lane], kp, lane);
+                theta_drop = fminf(theta_drop, fminf(s_theta[w], dk));
             }
-            theta_drop = fminf(theta_drop, __shfl_sync(FULL, lk, kp - 1));
             bool final_here = v0 == 0 && v1 == nv;
             if (!final_here) {
                 // publish this segment's list; the last CTA of the row merges all segments
@@ -560,10 +571,9 @@ __global__ void __launch_bounds__(kThreads, 3) race_kernel(const RaceArgs a) {
                     theta_drop = kInf;
                     for (int64_t bb = first_cta; bb <= last_cta; ++bb) {
                         const Partial* Q = a.partials + (bb + r);
-                        warp_merge(lk, li, __ldcg(Q->key + lane), __ldcg(Q->idx + lane), kp, lane);
-                        theta_drop = fminf(theta_drop, __ldcg(&Q->theta_drop));
+                        float dk = warp_merge<true>(lk, li, __ldcg(Q->key + lane), __ldcg(Q->idx + lane), kp, lane);
+                        theta_drop = fminf(theta_drop, fminf(__ldcg(&Q->theta_drop), dk));
                     }
-                    theta_drop = fminf(theta_drop, __shfl_sync(FULL, lk, kp - 1));
                 }
             }
             if (final_here) {
