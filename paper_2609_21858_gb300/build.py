@@ -36,6 +36,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
     os.makedirs(OUT, exist_ok=True)
     hdrs = [os.path.join(CSRC, h) for h in HEADERS] + [os.path.join(ROOT, "include", "pps.h")]
     flags = ["-std=c++17", "-O3", "-lineinfo", "-Xcompiler", "-fPIC", "-I" + os.path.join(ROOT, "include")] + ARCH
+    flags += os.environ.get("PPS_NVCC_FLAGS", "").split()  # extra flags for experiments (e.g. -DPPS_RACE_MIN_BLOCKS=4)
 
     def compile_one(src):
         s = os.path.join(CSRC, src)

@@ -13,7 +13,7 @@ namespace pps {
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 size_t workspace_bytes(int64_t n_rows, int32_t n_seq) {
-    return align256(sizeof(Partial) * (size_t)(n_rows + kGridMax)) + align256(sizeof(uint32_t) * (size_t)n_rows) +
+    return align256(sizeof(Partial) * (size_t)(n_rows + (int64_t)kGridMax)) + align256(sizeof(uint32_t) * (size_t)n_rows) +
            align256(sizeof(uint32_t) * (size_t)(n_seq > 0 ? n_seq : 0));
 }
 
@@ -21,7 +21,7 @@ void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials
                      uint32_t** seq_cnt) {
     char* p = static_cast<char*>(ws);
     *partials = reinterpret_cast<Partial*>(p);
-    p += align256(sizeof(Partial) * (size_t)(n_rows + kGridMax));
+    p += align256(sizeof(Partial) * (size_t)(n_rows + (int64_t)kGridMax));
     *row_cnt = reinterpret_cast<uint32_t*>(p);
     p += align256(sizeof(uint32_t) * (size_t)n_rows);
     *seq_cnt = reinterpret_cast<uint32_t*>(p);

@@ -84,26 +84,24 @@ __device__ __forceinline__ uint32_t word_of(uint64_t key, uint64_t ctx, uint32_t
 // the constant words in rounds 1-2 are hoisted per row: round 1 needs one
 // multiply, round 2 one multiply, rounds 3-10 the usual two.
 struct RowPhilox {
-    uint32_t r1_c3k;     // ctx_hi ^ key_hi                         (round 1, word 2)
-    uint32_t r2_hi0;     // hi(M0 * y0) with y0 = hi(M1*ctx_lo) ^ pos ^ k0   (round 2)
-    uint32_t r2_f;       // lo(M1 * ctx_lo) ^ (k0 + W0)             (round 2, word 0 xor term)
-    uint32_t r2_g;       // k1 + W1                                 (round 2, word 2 xor term)
-    uint32_t r2_lo0;     // lo(M0 * y0)                             (round 2, word 3)
+    uint32_t r1_c3k;          // ctx_hi ^ key_hi                         (round 1, word 2)
+    uint32_t r2_f;            // lo(M1 * ctx_lo) ^ (k0 + W0)             (round 2, word 0 xor term)
+    uint32_t r2_gh;           // hi(M0 * y0) ^ (k1 + W1), y0 = hi(M1*ctx_lo) ^ pos ^ k0   (round 2, word 2)
+    uint32_t r2_lo0;          // lo(M0 * y0)                             (round 2, word 3)
     uint32_t rk0[8], rk1[8];  // keys of rounds 3..10
 
     __device__ __forceinline__ void init(uint64_t key, uint64_t ctx, uint32_t pos) {
-        uint32_t k0 = (uint32_t)key, k1 = (uint32_t)(key >> 32);
-        uint32_t c2 = (uint32_t)ctx, c3 = (uint32_t)(ctx >> 32);
+        const uint32_t k0 = (uint32_t)key, k1 = (uint32_t)(key >> 32);
+        const uint32_t c2 = (uint32_t)ctx, c3 = (uint32_t)(ctx >> 32);
         uint32_t hi1, lo1;
         mulhilo(kPhiloxM1, c2, hi1, lo1);
-        uint32_t y0 = hi1 ^ pos ^ k0;  // round-1 word 0
+        const uint32_t y0 = hi1 ^ pos ^ k0;  // round-1 word 0
         r1_c3k = c3 ^ k1;
         uint32_t hi, lo;
         mulhilo(kPhiloxM0, y0, hi, lo);
-        r2_hi0 = hi;
         r2_lo0 = lo;
         r2_f = lo1 ^ (k0 + kPhiloxW0);
-        r2_g = k1 + kPhiloxW1;
+        r2_gh = hi ^ (k1 + kPhiloxW1);
 #pragma unroll
         for (int r = 0; r < 8; ++r) {
             rk0[r] = k0 + (uint32_t)(r + 2) * kPhiloxW0;
@@ -116,21 +114,21 @@ struct RowPhilox {
         uint32_t hi0, lo0;
         mulhilo(kPhiloxM0, c0, hi0, lo0);
         // round 1: (y0, y1) constant, y2 = hi0 ^ c3 ^ k1, y3 = lo0
-        uint32_t y2 = hi0 ^ r1_c3k;
-        uint32_t y3 = lo0;
+        const uint32_t y2 = hi0 ^ r1_c3k;
+        const uint32_t y3 = lo0;
         // round 2: M0*y0 constant
         uint32_t h1, l1;
         mulhilo(kPhiloxM1, y2, h1, l1);
         uint32_t x0 = h1 ^ r2_f;
         uint32_t x1 = l1;
-        uint32_t x2 = r2_hi0 ^ y3 ^ r2_g;
+        uint32_t x2 = y3 ^ r2_gh;
         uint32_t x3 = r2_lo0;
 #pragma unroll
         for (int r = 0; r < 8; ++r) {
             uint32_t a0, b0, a1, b1;
             mulhilo(kPhiloxM0, x0, a0, b0);
             mulhilo(kPhiloxM1, x2, a1, b1);
-            uint32_t n0 = a1 ^ x1 ^ rk0[r], n2 = a0 ^ x3 ^ rk1[r];
+            const uint32_t n0 = a1 ^ x1 ^ rk0[r], n2 = a0 ^ x3 ^ rk1[r];
             x0 = n0;
             x1 = b1;
             x2 = n2;
@@ -142,18 +140,32 @@ struct RowPhilox {
 
 // ------------------------------------------------------------------ transforms
 
-// y = -log2 u = E log2(e), accurate fp32 (u <= 1/2 through u, u > 1/2 through v = 1-u)
+// y = -log2 u = E log2(e) in fp32 with two MUFU operations at most:
+//   u <= 1/2:          y = -lg2(u), u rounded to fp32 (relative error 2^-24, y >= 1);
+//   1/2 < u, v >= 1/16: y = -lg2(1 - v) with 1 - v = u rounded to fp32 (y >= 0.093);
+//   v < 1/16:          y = v log2(e) (1 + v/2 + v^2/3 + v^3/4 + v^4/5 + v^5/6), the
+//                      Taylor series of -ln(1 - v) (truncation below v^6/7 < 2^-26.8).
+// The largest |log2(y32) - log2(y)| over all 2^32 words is measured by
+// pps_selftest_key_error and must stay below kErrAbs.
+__device__ __forceinline__ float lg2_approx(float x) {
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
 __device__ __forceinline__ float neg_log2_u(uint32_t w) {
-    if (w < 0x80000000u) {
-        float u = fmaf((float)w, 0x1p-32f, 0x1p-33f);
-        return -log2f(u);
-    }
-    float v = fmaf((float)(~w), 0x1p-32f, 0x1p-33f);
-    return -log1pf(-v) * kLog2e;
+    if (w < 0x80000000u) return -lg2_approx(fmaf((float)w, 0x1p-32f, 0x1p-33f));
+    const float v = fmaf((float)(~w), 0x1p-32f, 0x1p-33f);
+    if (v >= 0.0625f) return -lg2_approx(fmaf((float)w, 0x1p-32f, 0x1p-33f));
+    float p = fmaf(v, 1.0f / 6.0f, 0.2f);
+    p = fmaf(v, p, 0.25f);
+    p = fmaf(v, p, 1.0f / 3.0f);
+    p = fmaf(v, p, 0.5f);
+    p = fmaf(v, p, 1.0f);
+    return v * kLog2e * p;
 }
 
 // x = log2(-log2 u), the word part of the fp32 key
-__device__ __forceinline__ float key_x32(uint32_t w) { return log2f(neg_log2_u(w)); }
+__device__ __forceinline__ float key_x32(uint32_t w) { return lg2_approx(neg_log2_u(w)); }
 
 // fp32 key k = x - l * c with c = log2(e) / T; NaN logits map to +inf
 __device__ __forceinline__ float key32(uint32_t w, float l, float c) {
@@ -189,22 +201,28 @@ __device__ __forceinline__ float key_to_s(float k) { return (k + kLog2Ln2) * 0.6
 //
 // A token can enter a list only if its fp32 key is below theta.  Since
 // E = -ln(1 - v) >= v with v = 1 - u = (~w + 1/2) 2^-32, a key below theta
-// needs v < e_z := 2^(theta + l c) ln 2.  With a = (~w) >> 9 that holds only if
-// a <= round(2^(theta + margin + l c + log2(ln 2) + 23)).  tz carries
-// theta + margin + log2(ln 2) + 23 (+inf while the list is not full).
-// The comparison is done on float bit patterns: 2^23 + a has the bits
-// 0x4b000000 | a, and T + 2^23 rounds T to an integer in the low bits for
-// T < 2^23 (and is larger than every 0x4b000000 | a otherwise).
+// needs v < e_z := 2^(theta + l c) ln 2, i.e. (with a = (~w) >> 9, so that
+// ~w >= 512 a) a < T := e_z 2^23.  With b = w >> 9, a = 2^23 - 1 - b, so the
+// token can be dropped when T + 2^23 + b <= 2^24 - 1.  The sum is formed in
+// fp32 from the bit pattern 0x4b000000 + b (= 2^23 + b exactly, one mad.hi
+// on the multiply pipe) plus T; its rounding error is below 1, so testing
+// S >= 2^24 - 2 never drops a token that could enter.  tz carries
+// theta + margin + log2(ln 2) + 23 (+inf while the list is not full); NaN
+// logits give S = NaN and are dropped.
 __device__ __forceinline__ float ex2_approx(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
-__device__ __forceinline__ bool filter_pass(uint32_t w, float l, float c, float tz) {
+__device__ __forceinline__ float filter_sum(uint32_t w, float l, float c, float tz) {
     float T = ex2_approx(fmaf(l, c, tz));
-    uint32_t tb = __float_as_uint(T + 8388608.0f);
-    uint32_t ab = (~(w >> 9) & 0x007fffffu) | 0x4b000000u;
-    return ab <= tb;
+    uint32_t bb;
+    asm("mad.hi.u32 %0, %1, %2, %3;" : "=r"(bb) : "r"(w), "r"(1u << 23), "r"(0x4b000000u));
+    return T + __uint_as_float(bb);
+}
+constexpr float kFilterCut = 16777214.0f;  // 2^24 - 2
+__device__ __forceinline__ bool filter_pass(uint32_t w, float l, float c, float tz) {
+    return filter_sum(w, l, c, tz) >= kFilterCut;
 }
 __device__ __forceinline__ float filter_tz(float theta) {
     return theta + (kFilterMargin + kLog2Ln2 + 23.0f);

@@ -5,10 +5,10 @@
 
 namespace pps {
 
-constexpr int kThreads = 256;           // threads per CTA of the streaming kernels
+constexpr int kThreads = 32;            // one warp per CTA: per-row values are CTA-uniform
 constexpr int kWarps = kThreads / 32;
-constexpr int kGridMax = 4096;          // upper bound on the streaming grid (sizes the workspace)
-constexpr int64_t kMinVecsPerCta = 2048;  // 16-byte vectors per CTA below which the grid shrinks
+constexpr int kGridMax = 16384;         // upper bound on the streaming grid (one-warp CTAs)
+constexpr int64_t kMinVecsPerWarp = 256;  // 16-byte vectors per warp below which the grid shrinks
 
 // one partial candidate list of a row segment (sorted ascending by (key, idx))
 struct alignas(16) Partial {
@@ -58,7 +58,7 @@ struct RaceArgs {
     int64_t total;  // n_rows * nv
     int G;
     // workspace
-    Partial* partials;   // [n_rows + kGridMax]
+    Partial* partials;   // [n_rows + kGridMax]: slot (warp + row)
     uint32_t* row_cnt;   // [n_rows]
     uint32_t* seq_cnt;   // [n_seq]
 };

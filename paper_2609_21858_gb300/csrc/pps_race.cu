@@ -2,20 +2,24 @@
 // target winners) with the tree walk fused behind a per-sequence ticket.
 //
 // Work split.  The n_rows x vocab logits are viewed as one flattened range of
-// 16-byte vectors (8 bf16 or 4 fp32 tokens); CTA b of G streams the slice
-// [b*total/G, (b+1)*total/G), i.e. whole rows plus at most two partial rows.
-// A row cut between CTAs is finished by the CTA that arrives last at the
-// row's counter (no CTA ever waits on another).
+// 16-byte vectors (8 bf16 or 4 fp32 tokens).  A CTA is a single warp; warp gw
+// of NW streams the slice [gw*total/NW, (gw+1)*total/NW), i.e. a few whole
+// rows plus at most two partial rows.  A row cut between warps is merged and
+// finished by the warp that arrives last at the row's counter; a sequence's
+// walk is run by the warp that finishes its last node.  No warp ever waits
+// for another and the kernel has no block-wide barrier.  One-warp CTAs also
+// make every per-row value warp-uniform, so the Philox round keys of a row
+// can live in uniform registers.
 //
-// Per token (hot loop): the Philox word (row-specialised), the logit, and a
+// Per token (fast loop): the Philox word (row-specialised), the logit, and a
 // conservative fp32 filter that rejects almost every token with one ex2 and
-// an integer compare (pps_device.cuh).  Survivors get the accurate fp32 key
-// and enter a per-warp sorted list of kp = min(32, 2k+2) entries (one entry
-// per lane).  Lists are merged per CTA and per row with warp bitonic merges.
-// The finished list proves its own completeness (every dropped token has a
-// key above the k-th key plus both error bounds) and re-orders near-ties
-// with the fp64 key s = ln E - l/T, so the selected tokens and their order
-// are those of the exact definition (Alg. 2, Eq. 4, App. B algorithms).
+// a few multiply-pipe operations (pps_device.cuh).  Survivors get the fp32 key
+// and enter a per-warp sorted list of kp = min(32, 2k+1) entries (one per
+// lane).  Lists of a row are merged with warp bitonic merges.  The finished
+// list proves its own completeness (every dropped token has a key above the
+// k-th key plus both error bounds) and re-orders near-ties with the fp64 key
+// s = ln E - l/T, so the selected tokens and their order are those of the
+// exact definition (Alg. 2, Eq. 4, App. B algorithms).
 #include <cfloat>
 #include <climits>
 #include <cstdint>
@@ -23,6 +27,16 @@
 #include "pps.h"
 #include "pps_device.cuh"
 #include "pps_internal.h"
+
+#ifndef PPS_UNITS
+#define PPS_UNITS 2  // 8-token units per lane per fast-loop iteration (2 Philox blocks each)
+#endif
+#ifndef PPS_PREFETCH
+#define PPS_PREFETCH 0  // 1: load the next iteration's vectors one iteration ahead (costs registers)
+#endif
+#ifndef PPS_RACE_MIN_BLOCKS
+#define PPS_RACE_MIN_BLOCKS 16  // one-warp CTAs resident per SM: 128 registers, no spills
+#endif
 
 namespace pps {
 
@@ -155,14 +169,61 @@ __device__ __forceinline__ uint4 ldg_stream(const void* p) {
     return r;
 }
 
-// ---------------------------------------------------------------- per-warp stream state
+// scalar load of the tokens of vector v (i < V), packed like a 16-byte vector
+template <int DT>
+__device__ __forceinline__ uint4 load_scalar(const char* row, int64_t v, int64_t V) {
+    constexpr int VW = DT == 1 ? 8 : 4;
+    uint32_t t[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int e = 0; e < VW; ++e) {
+        int64_t i = v * VW + e;
+        if (i < V) {
+            if constexpr (DT == 1) {
+                uint32_t h = __ldg(reinterpret_cast<const unsigned short*>(row) + i);
+                t[e >> 1] |= h << (16 * (e & 1));
+            } else {
+                t[e] = __float_as_uint(__ldg(reinterpret_cast<const float*>(row) + i));
+            }
+        }
+    }
+    return make_uint4(t[0], t[1], t[2], t[3]);
+}
+
+// Counter offset of block b of a lane's fast-loop iteration: bf16 blocks come
+// in pairs (2v, 2v+1) of one vector v, vectors 32 apart; fp32 blocks are
+// single vectors 32 apart.
+template <int DT>
+__device__ __forceinline__ uint32_t block_offset(int b) {
+    return DT == 1 ? (uint32_t)((b >> 1) * 64 + (b & 1)) : (uint32_t)(32 * b);
+}
+
+// the four logits of block b of an iteration's vectors d[]
+template <int DT>
+__device__ __forceinline__ void block_logits(const uint4 (&d)[4], int b, float (&l)[4]) {
+    if constexpr (DT == 1) {
+        const uint4 v = d[b >> 1];
+        const uint32_t x0 = (b & 1) ? v.z : v.x, x1 = (b & 1) ? v.w : v.y;
+        l[0] = bf16_lo(x0);
+        l[1] = bf16_hi(x0);
+        l[2] = bf16_lo(x1);
+        l[3] = bf16_hi(x1);
+    } else {
+        const uint4 v = d[b];
+        l[0] = __uint_as_float(v.x);
+        l[1] = __uint_as_float(v.y);
+        l[2] = __uint_as_float(v.z);
+        l[3] = __uint_as_float(v.w);
+    }
+}
+
+// ---------------------------------------------------------------- per-warp list state
 
 struct WarpList {
-    float lk;   // this lane's entry
+    float lk;  // this lane's entry
     int li;
-    float th;   // key of entry kp-1 (+inf while not full)
+    float th;  // key of entry kp-1 (+inf while not full)
     int thi;
-    float tz;   // filter threshold (pps_device.cuh)
+    float tz;  // filter threshold (pps_device.cuh)
     int kp;
 
     __device__ __forceinline__ void reset(int kp_) {
@@ -180,7 +241,11 @@ struct WarpList {
     }
 };
 
-// Offer the survivors of one vector (keys pk[e], token i0 + e) to the warp list.
+// Offer the keyed survivors of one lane (pk[e] for token i0 + e, +inf = none)
+// to the warp list: each round every lane offers its smallest remaining key
+// below the threshold; up to three offers are inserted one by one, more are
+// sorted across the warp and merged.  Ends when no lane has a key below it,
+// so the threshold is always current.
 template <int VW>
 __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], int64_t i0, int lane) {
     while (true) {
@@ -194,16 +259,16 @@ __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], in
                 be = e;
             }
         }
-        bool valid = be >= 0 && bk < kInf && lex_less(bk, bi, L.th, L.thi);
-        unsigned vm = __ballot_sync(FULL, valid);
+        const bool valid = be >= 0 && bk < kInf && lex_less(bk, bi, L.th, L.thi);
+        const unsigned vm = __ballot_sync(FULL, valid);
         if (vm == 0) break;
         if (__popc(vm) <= 3) {
             unsigned m = vm;
             while (m) {
-                int src = __ffs(m) - 1;
+                const int src = __ffs(m) - 1;
                 m &= m - 1;
-                float ck = __shfl_sync(FULL, bk, src);
-                int ci = __shfl_sync(FULL, bi, src);
+                const float ck = __shfl_sync(FULL, bk, src);
+                const int ci = __shfl_sync(FULL, bi, src);
                 list_insert(L.lk, L.li, ck, ci, L.kp, lane);
             }
         } else {
@@ -212,45 +277,199 @@ __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], in
             warp_sort(ok, oi, lane);
             warp_merge<false>(L.lk, L.li, ok, oi, L.kp, lane);
         }
-        if (valid) {
+        // every offer of this round is now in the list or above its threshold
 #pragma unroll
-            for (int e = 0; e < VW; ++e)
-                if (e == be) pk[e] = kInf;
-        }
+        for (int e = 0; e < VW; ++e)
+            if (e == be) pk[e] = kInf;
         L.refresh();
     }
 }
 
-// Process one 16-byte vector of tokens [i0, i0+VW) with words from RowPhilox.
+// Filter, key and offer the 4 tokens of one Philox block (counter cb, tokens
+// 4cb..4cb+3, logits l[]) for the lanes with `mine`.
+__device__ __forceinline__ void block_survivors(WarpList& L, const RowPhilox& rp, bool mine, uint32_t cb,
+                                                const float (&l)[4], unsigned valid, float c, int lane) {
+    float pk[4] = {kInf, kInf, kInf, kInf};
+    if (mine) {
+        const uint4 q = rp.block(cb);
+        const uint32_t wq[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            if (((valid >> e) & 1u) && filter_pass(wq[e], l[e], c, L.tz)) pk[e] = key32(wq[e], l[e], c);
+    }
+    offer_survivors<4>(L, pk, (int64_t)4 * cb, lane);
+}
+
+// ---------------------------------------------------------------- rare paths (out of line)
+
+struct SlowState {
+    WarpList L;
+};
+
+// Slow path of the fast loop: the blocks flagged in bm (bit b = block b of
+// this lane's iteration) have a token over the filter cut; regenerate their
+// words and offer their survivors.  The fast loop keeps no per-token state.
+template <int DT, int NB>
+__device__ __noinline__ SlowState slow_blocks(SlowState st, uint64_t key, uint64_t ctx, uint32_t pos, unsigned bm,
+                                              uint32_t cl, uint4 d0, uint4 d1, uint4 d2, uint4 d3, float c) {
+    const int lane = threadIdx.x & 31;
+    RowPhilox rp;
+    rp.init(key, ctx, pos);
+    const uint4 d[4] = {d0, d1, d2, d3};
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        if (__any_sync(FULL, (bm >> b) & 1u)) {
+            float l[4];
+            block_logits<DT>(d, b, l);
+            block_survivors(st.L, rp, (bm >> b) & 1u, cl + block_offset<DT>(b), l, 0xfu, c, lane);
+        }
+    }
+    return st;
+}
+
+// Scalar-load path, one vector per lane at a time: the last partial
+// iteration of a segment, the ragged vector of a row, and unaligned rows.
 template <int DT>
-__device__ __forceinline__ void process_vector(WarpList& L, const RowPhilox& rp, uint4 d, int64_t vidx, int nvalid,
-                                               float c, int lane) {
+__device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64_t V, int64_t base, int64_t v1,
+                                            float c, uint64_t key, uint64_t ctx, uint32_t pos) {
     constexpr int VW = DT == 1 ? 8 : 4;
-    const int64_t i0 = vidx * VW;
-    uint32_t w[VW];
-    float l[VW];
-    if constexpr (DT == 1) {
-        uint4 b0 = rp.block((uint32_t)(2 * vidx));
-        uint4 b1 = rp.block((uint32_t)(2 * vidx + 1));
-        w[0] = b0.x; w[1] = b0.y; w[2] = b0.z; w[3] = b0.w;
-        w[4] = b1.x; w[5] = b1.y; w[6] = b1.z; w[7] = b1.w;
-        l[0] = bf16_lo(d.x); l[1] = bf16_hi(d.x); l[2] = bf16_lo(d.y); l[3] = bf16_hi(d.y);
-        l[4] = bf16_lo(d.z); l[5] = bf16_hi(d.z); l[6] = bf16_lo(d.w); l[7] = bf16_hi(d.w);
-    } else {
-        uint4 b0 = rp.block((uint32_t)vidx);
-        w[0] = b0.x; w[1] = b0.y; w[2] = b0.z; w[3] = b0.w;
-        l[0] = __uint_as_float(d.x); l[1] = __uint_as_float(d.y);
-        l[2] = __uint_as_float(d.z); l[3] = __uint_as_float(d.w);
-    }
-    unsigned m = 0;
+    const int lane = threadIdx.x & 31;
+    RowPhilox rp;
+    rp.init(key, ctx, pos);
+    for (; base < v1; base += 32) {
+        const int64_t v = base + lane;
+        uint4 dv = make_uint4(0, 0, 0, 0);
+        unsigned valid = 0;
+        if (v < v1) {
+            dv = load_scalar<DT>(row, v, V);
+            const int64_t nt = min((int64_t)VW, V - v * VW);
+            valid = (1u << nt) - 1u;
+        }
+        const uint4 d[4] = {dv, dv, dv, dv};
+        // the vector's blocks: bf16 2 (counters 2v, 2v+1), fp32 1 (counter v)
 #pragma unroll
-    for (int e = 0; e < VW; ++e) m |= (unsigned)(filter_pass(w[e], l[e], c, L.tz) && e < nvalid) << e;
-    if (__any_sync(FULL, m != 0)) {
-        float pk[VW];
+        for (int h = 0; h < (DT == 1 ? 2 : 1); ++h) {
+            const unsigned vh = (valid >> (4 * h)) & 0xfu;
+            float l[4];
+            block_logits<DT>(d, h, l);
+            const uint32_t cb = DT == 1 ? (uint32_t)(2 * v + h) : (uint32_t)v;
+            // any token of the block over the cut?
+            bool pass = false;
+            if (vh) {
+                const uint4 q = rp.block(cb);
+                const uint32_t wq[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
-        for (int e = 0; e < VW; ++e) pk[e] = (m >> e & 1u) ? key32(w[e], l[e], c) : kInf;
-        offer_survivors<VW>(L, pk, i0, lane);
+                for (int e = 0; e < 4; ++e) pass |= ((vh >> e) & 1u) && filter_pass(wq[e], l[e], c, st.L.tz);
+            }
+            if (__any_sync(FULL, pass)) block_survivors(st.L, rp, pass, cb, l, vh, c, lane);
+        }
     }
+    return st;
+}
+
+// ---------------------------------------------------------------- the fast loop
+
+struct ScanStop {
+    int64_t it;   // iteration with a survivor (n_it when the scan ran to the end)
+    unsigned bm;  // its blocks over the filter cut (this lane)
+    uint32_t cl;  // its block counter base (this lane)
+    uint4 d0, d1, d2, d3;
+};
+
+// Fast scan over iterations [it0, n_it) of the full vectors starting at
+// vector v0 of a row.  Each iteration covers PPS_UNITS x 32 (bf16) or x 64
+// (fp32) vectors; every lane takes PPS_UNITS units of 8 tokens = 2 x
+// PPS_UNITS Philox blocks with counters cl + block_offset(b), cl advancing by
+// 64 x PPS_UNITS, so that many independent multiply chains are in flight per
+// lane.  A lane keeps only the per-block maxima of the filter sums.  The scan
+// makes no calls: it stops at the first iteration in which some lane has a
+// block over the cut and hands that iteration back, so that nothing the loop
+// keeps in registers (the row's round keys above all) lives across a call.
+template <int DT>
+__device__ __forceinline__ ScanStop fast_scan(const RowPhilox& rp, const char* row, int64_t v0, int64_t it0,
+                                              int64_t n_it, float c, float tz) {
+    constexpr int NB = 2 * PPS_UNITS;          // Philox blocks per lane per iteration
+    constexpr int ND = DT == 1 ? NB / 2 : NB;  // 16-byte vectors per lane per iteration
+    constexpr int STEP = 32 * ND;              // vectors per iteration
+    const int lane = threadIdx.x & 31;
+    const uint4* p = reinterpret_cast<const uint4*>(row) + v0 + it0 * STEP + lane;
+    uint32_t cl = (DT == 1 ? (uint32_t)(2 * (v0 + lane)) : (uint32_t)(v0 + lane)) + (uint32_t)(it0 * 64 * PPS_UNITS);
+    ScanStop out;
+    out.it = n_it;
+#if PPS_PREFETCH
+    uint4 nx[ND];
+#pragma unroll
+    for (int k = 0; k < ND; ++k) nx[k] = ldg_stream(p + 32 * k);
+#endif
+    for (int64_t it = it0; it < n_it; ++it) {
+        uint4 d[4];
+#if PPS_PREFETCH
+#pragma unroll
+        for (int k = 0; k < ND; ++k) d[k] = nx[k];
+        p += STEP;
+        if (it + 1 < n_it) {
+#pragma unroll
+            for (int k = 0; k < ND; ++k) nx[k] = ldg_stream(p + 32 * k);
+        }
+#else
+#pragma unroll
+        for (int k = 0; k < ND; ++k) d[k] = ldg_stream(p + 32 * k);
+        p += STEP;
+#endif
+#pragma unroll
+        for (int k = ND; k < 4; ++k) d[k] = d[0];
+        unsigned bm = 0;
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            const uint4 q = rp.block(cl + block_offset<DT>(b));
+            float l[4];
+            block_logits<DT>(d, b, l);
+            const float m01 = fmaxf(filter_sum(q.x, l[0], c, tz), filter_sum(q.y, l[1], c, tz));
+            const float m23 = fmaxf(filter_sum(q.z, l[2], c, tz), filter_sum(q.w, l[3], c, tz));
+            bm |= (unsigned)(fmaxf(m01, m23) >= kFilterCut) << b;
+        }
+        if (__any_sync(FULL, bm != 0)) {
+            out.it = it;
+            out.bm = bm;
+            out.cl = cl;
+            out.d0 = d[0];
+            out.d1 = d[1];
+            out.d2 = d[2];
+            out.d3 = d[3];
+            break;
+        }
+        cl += 64 * PPS_UNITS;
+    }
+    return out;
+}
+
+// Stream vectors [v0, v1) of one row through the warp's list: full
+// iterations through the fast loop, the rest through the scalar tail.
+template <int DT, bool VEC>
+__device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int64_t V, int64_t v0, int64_t v1,
+                                               float c, uint64_t key, uint64_t ctx, uint32_t pos) {
+    constexpr int VW = DT == 1 ? 8 : 4;
+    constexpr int STEP = (DT == 1 ? 32 : 64) * PPS_UNITS;  // vectors per fast-loop iteration
+    const int64_t nfull = V / VW;                           // vectors holding VW tokens
+    const int64_t vend = VEC ? min(v1, nfull) : v0;
+    const int64_t n_it = vend > v0 ? (vend - v0) / STEP : 0;
+    SlowState st{L};
+    int64_t base = v0;
+    if (n_it > 0) {
+        constexpr int NB = 2 * PPS_UNITS;
+        int64_t it = 0;
+        while (true) {
+            RowPhilox rp;
+            rp.init(key, ctx, pos);
+            const ScanStop sp = fast_scan<DT>(rp, row, v0, it, n_it, c, st.L.tz);
+            if (sp.it >= n_it) break;
+            st = slow_blocks<DT, NB>(st, key, ctx, pos, sp.bm, sp.cl, sp.d0, sp.d1, sp.d2, sp.d3, c);
+            it = sp.it + 1;
+        }
+        base = v0 + n_it * STEP;
+    }
+    if (base < v1) st = tail_loop<DT>(st, row, V, base, v1, c, key, ctx, pos);
+    L = st.L;
 }
 
 // ---------------------------------------------------------------- finalize
@@ -265,8 +484,8 @@ __device__ void walk_sequence(const RaceArgs& a, int s);
 
 // Warp 0 finishes row r from its complete list (lk, li) and the drop bound.
 template <int DT, bool VERIFY>
-__device__ void finalize_row(const RaceArgs& a, int64_t r, float lk, int li, float theta_drop, int kr, int kp,
-                             int lane) {
+__device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk, int li, float theta_drop, int kr,
+                                          int kp, int lane) {
     const int nvalid = __popc(__ballot_sync(FULL, lane < kp && lk < kInf));
     const float tau = nvalid >= kr ? __shfl_sync(FULL, lk, kr - 1) : kInf;
     bool complete;
@@ -366,9 +585,9 @@ __device__ void finalize_row(const RaceArgs& a, int64_t r, float lk, int li, flo
     if (lane == 0) a.out_nd[r] = nd;
 }
 
-__device__ __forceinline__ int64_t cta_of(int64_t g, int64_t total, int G) {
-    // largest b with floor(b*total/G) <= g
-    return ((g + 1) * (int64_t)G - 1) / total;
+__device__ __forceinline__ int64_t warp_of(int64_t g, int64_t total, int64_t NW) {
+    // largest w with floor(w*total/NW) <= g
+    return ((g + 1) * NW - 1) / total;
 }
 
 __device__ __forceinline__ int seq_of_node(const int32_t* seq_off, int n_seq, int64_t r) {
@@ -383,7 +602,7 @@ __device__ __forceinline__ int seq_of_node(const int32_t* seq_off, int n_seq, in
     return lo;
 }
 
-__device__ void walk_sequence(const RaceArgs& a, int s) {
+__device__ __noinline__ void walk_sequence(const RaceArgs& a, int s) {
     const int W = a.gamma + 1;
     int c = __ldg(a.seq_off + s);
     if (c < 0 || c >= a.n_rows) return;
@@ -441,162 +660,105 @@ __device__ void walk_sequence(const RaceArgs& a, int s) {
     a.out_ss[s] = S;
 }
 
+// End of a row segment: publish the warp's list, or merge the row's lists if
+// this warp is the last to finish the row, then finish the row (and the walk
+// of its sequence when it is the sequence's last node).  Out of line.
+template <int DT, bool VERIFY>
+__device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_t gw, int64_t NW, int64_t v0,
+                                        int64_t v1, const WarpList L, int kr, int kp) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nv = a.nv;
+    float lk = L.lk;
+    int li = L.li;
+    // every token of the segment left out of the list has a key >= theta_drop
+    float theta_drop = L.th;
+    bool final_here = v0 == 0 && v1 == nv;
+    if (!final_here) {
+        // publish this segment's list; the last warp of the row merges all segments
+        Partial* P = a.partials + (gw + r);
+        P->key[lane] = lk;
+        P->idx[lane] = li;
+        if (lane == 0) P->theta_drop = theta_drop;
+        __threadfence();
+        __syncwarp();
+        const int64_t first_w = warp_of(r * nv, a.total, NW);
+        const int64_t last_w = warp_of(r * nv + nv - 1, a.total, NW);
+        unsigned last = 0;
+        if (lane == 0) {
+            unsigned t = atomicAdd(a.row_cnt + r, 1u);
+            last = t == (unsigned)(last_w - first_w);
+            if (last) a.row_cnt[r] = 0u;
+        }
+        final_here = __shfl_sync(FULL, last, 0) != 0;
+        if (final_here) {
+            __threadfence();
+            lk = kInf;
+            li = INT_MAX;
+            theta_drop = kInf;
+            for (int64_t ww = first_w; ww <= last_w; ++ww) {
+                const Partial* Q = a.partials + (ww + r);
+                float dk = warp_merge<true>(lk, li, __ldcg(Q->key + lane), __ldcg(Q->idx + lane), kp, lane);
+                theta_drop = fminf(theta_drop, fminf(__ldcg(&Q->theta_drop), dk));
+            }
+        }
+    }
+    if (final_here) {
+        finalize_row<DT, VERIFY>(a, r, lk, li, theta_drop, kr, kp, lane);
+        if constexpr (VERIFY) {
+            // sequence ticket: the warp that finishes a sequence's last node walks it
+            __threadfence();
+            if (lane == 0) {
+                int s = seq_of_node(a.seq_off, a.n_seq, r);
+                int nn = __ldg(a.seq_off + s + 1) - __ldg(a.seq_off + s);
+                unsigned t = atomicAdd(a.seq_cnt + s, 1u);
+                if (t == (unsigned)(nn - 1)) {
+                    a.seq_cnt[s] = 0u;
+                    __threadfence();
+                    walk_sequence(a, s);
+                }
+            }
+            __syncwarp();
+        }
+    }
+}
+
 // ---------------------------------------------------------------- the kernel
+//
+// Every warp is an independent worker: warp gw of NW streams the flattened
+// vector slice [gw*total/NW, (gw+1)*total/NW).  A row cut between warps is
+// merged and finished by the warp that arrives last at the row's counter; a
+// sequence's walk is run by the warp that finishes its last node.  No warp
+// ever waits for another and the kernel has no block-wide barrier.
 
 template <int DT, bool VERIFY, bool VEC>
-__global__ void __launch_bounds__(kThreads, 3) race_kernel(const RaceArgs a) {
-    constexpr int VW = DT == 1 ? 8 : 4;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    __shared__ float s_key[kWarps][32];
-    __shared__ int s_idx[kWarps][32];
-    __shared__ float s_theta[kWarps];
-
-    const int64_t b = blockIdx.x;
-    const int64_t g0 = b * a.total / a.G, g1 = (b + 1) * a.total / a.G;
-    if (g0 >= g1) return;
+__global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(const RaceArgs a) {
+    const int64_t NW = a.G;
+    const int64_t gw = blockIdx.x;
+    const int64_t g0 = gw * a.total / NW, g1 = (gw + 1) * a.total / NW;
     const float c = a.c;
     const int64_t nv = a.nv;
-    const int tail = (int)(a.V - (nv - 1) * VW);  // tokens in the last vector of a row (1..VW)
     const size_t esz = DT == 1 ? 2 : 4;
 
-    for (int64_t r = g0 / nv; r < a.n_rows && r * nv < g1; ++r) {
+    for (int64_t r = g0 / nv; g0 < g1 && r < a.n_rows && r * nv < g1; ++r) {
         const int64_t v0 = max(g0, r * nv) - r * nv, v1 = min(g1, (r + 1) * nv) - r * nv;
         int kr = 1;
         if (!VERIFY) {
             kr = a.row_k ? __ldg(a.row_k + r) : a.K;
             kr = max(1, min(kr, a.K));
         }
-        const int kp = min(32, 2 * kr + 2);
-        RowPhilox rp;
-        rp.init(__ldg(a.key + r), __ldg(a.ctx + r), __ldg(a.pos + r));
+        const int kp = min(32, 2 * kr + 1);
+        const uint64_t key = __ldg(a.key + r), ctx = __ldg(a.ctx + r);
+        const uint32_t pos = __ldg(a.pos + r);
         const char* row = reinterpret_cast<const char*>(a.logits) + (size_t)r * (size_t)a.stride * esz;
 
         WarpList L;
         L.reset(kp);
-        // stream: thread t takes vectors v0 + t, v0 + t + kThreads, ...
-        int64_t v = v0 + threadIdx.x;
-        if (VEC) {
-            const int64_t vfull_end = (tail == VW) ? v1 : min(v1, nv - 1);
-            uint4 cur = make_uint4(0, 0, 0, 0), nxt = cur;
-            if (v < vfull_end) cur = ldg_stream(row + (size_t)v * 16);
-            // warps iterate in lockstep while any lane has work
-            while (__any_sync(FULL, v < vfull_end)) {
-                int64_t vn = v + kThreads;
-                if (vn < vfull_end) nxt = ldg_stream(row + (size_t)vn * 16);
-                int nvld = v < vfull_end ? VW : 0;
-                process_vector<DT>(L, rp, cur, v < vfull_end ? v : 0, nvld, c, lane);
-                cur = nxt;
-                v = vn;
-            }
-            // ragged last vector of the row (scalar loads)
-            if (vfull_end < v1) {
-                int64_t vl = nv - 1;
-                uint4 d = make_uint4(0, 0, 0, 0);
-                int nvld = 0;
-                if (threadIdx.x == (int)((vl - v0) % kThreads) && vl >= v0) {
-                    uint32_t tmp[4] = {0u, 0u, 0u, 0u};
-                    for (int e = 0; e < tail; ++e) {
-                        int64_t i = vl * VW + e;
-                        if (DT == 1) {
-                            uint32_t h = __ldg(reinterpret_cast<const unsigned short*>(row) + i);
-                            tmp[e >> 1] |= h << (16 * (e & 1));
-                        } else {
-                            tmp[e] = __float_as_uint(__ldg(reinterpret_cast<const float*>(row) + i));
-                        }
-                    }
-                    d = make_uint4(tmp[0], tmp[1], tmp[2], tmp[3]);
-                    nvld = tail;
-                }
-                process_vector<DT>(L, rp, d, nvld ? vl : 0, nvld, c, lane);
-            }
-        } else {
-            // unaligned rows: scalar loads for every token
-            while (__any_sync(FULL, v < v1)) {
-                uint32_t tmp[4] = {0u, 0u, 0u, 0u};
-                int nvld = 0;
-                if (v < v1) {
-                    nvld = (v == nv - 1) ? tail : VW;
-                    for (int e = 0; e < nvld; ++e) {
-                        int64_t i = v * VW + e;
-                        if (DT == 1) {
-                            uint32_t h = __ldg(reinterpret_cast<const unsigned short*>(row) + i);
-                            tmp[e >> 1] |= h << (16 * (e & 1));
-                        } else {
-                            tmp[e] = __float_as_uint(__ldg(reinterpret_cast<const float*>(row) + i));
-                        }
-                    }
-                }
-                process_vector<DT>(L, rp, make_uint4(tmp[0], tmp[1], tmp[2], tmp[3]), nvld ? v : 0, nvld, c, lane);
-                v += kThreads;
-            }
-        }
+        stream_segment<DT, VEC>(L, row, a.V, v0, v1, c, key, ctx, pos);
 
-        // ---- merge the warp lists of this CTA
-        s_key[warp][lane] = L.lk;
-        s_idx[warp][lane] = L.li;
-        if (lane == 0) s_theta[warp] = L.th;
-        __syncthreads();
-        if (warp == 0) {
-            float lk = L.lk;
-            int li = L.li;
-            float theta_drop = s_theta[0];
-            // every token left out of the merged list has a key >= theta_drop: the warps
-            // dropped only keys >= their final kp-th key, the merges drop what they return
-            for (int w = 1; w < kWarps; ++w) {
-                float dk = warp_merge<true>(lk, li, s_key[w][lane], s_idx[w][lane], kp, lane);
-                theta_drop = fminf(theta_drop, fminf(s_theta[w], dk));
-            }
-            bool final_here = v0 == 0 && v1 == nv;
-            if (!final_here) {
-                // publish this segment's list; the last CTA of the row merges all segments
-                Partial* P = a.partials + (b + r);
-                P->key[lane] = lk;
-                P->idx[lane] = li;
-                if (lane == 0) P->theta_drop = theta_drop;
-                __threadfence();
-                __syncwarp();
-                const int64_t first_cta = cta_of(r * nv, a.total, a.G);
-                const int64_t last_cta = cta_of(r * nv + nv - 1, a.total, a.G);
-                unsigned last = 0;
-                if (lane == 0) {
-                    unsigned t = atomicAdd(a.row_cnt + r, 1u);
-                    last = t == (unsigned)(last_cta - first_cta);
-                    if (last) a.row_cnt[r] = 0u;
-                }
-                final_here = __shfl_sync(FULL, last, 0) != 0;
-                if (final_here) {
-                    __threadfence();
-                    lk = kInf;
-                    li = INT_MAX;
-                    theta_drop = kInf;
-                    for (int64_t bb = first_cta; bb <= last_cta; ++bb) {
-                        const Partial* Q = a.partials + (bb + r);
-                        float dk = warp_merge<true>(lk, li, __ldcg(Q->key + lane), __ldcg(Q->idx + lane), kp, lane);
-                        theta_drop = fminf(theta_drop, fminf(__ldcg(&Q->theta_drop), dk));
-                    }
-                }
-            }
-            if (final_here) {
-                finalize_row<DT, VERIFY>(a, r, lk, li, theta_drop, kr, kp, lane);
-                if constexpr (VERIFY) {
-                    // sequence ticket: the CTA that finishes a sequence's last node walks it
-                    __threadfence();
-                    if (lane == 0) {
-                        int s = seq_of_node(a.seq_off, a.n_seq, r);
-                        int nn = __ldg(a.seq_off + s + 1) - __ldg(a.seq_off + s);
-                        unsigned t = atomicAdd(a.seq_cnt + s, 1u);
-                        if (t == (unsigned)(nn - 1)) {
-                            a.seq_cnt[s] = 0u;
-                            __threadfence();
-                            walk_sequence(a, s);
-                        }
-                    }
-                }
-            }
-        }
-        __syncthreads();
+        finish_segment<DT, VERIFY>(a, r, gw, NW, v0, v1, L, kr, kp);
     }
 }
+
 
 int race_grid(int64_t total, int dtype, bool verify, bool vec) {
     static int sms = 0, occ[2][2][2] = {};
@@ -619,7 +781,7 @@ int race_grid(int64_t total, int dtype, bool verify, bool vec) {
         if (o <= 0) o = 1;
     }
     int64_t g = (int64_t)sms * o;
-    int64_t by_size = (total + kMinVecsPerCta - 1) / kMinVecsPerCta;
+    int64_t by_size = (total + kMinVecsPerWarp - 1) / kMinVecsPerWarp;
     if (by_size < g) g = by_size;
     if (g > kGridMax) g = kGridMax;
     if (g < 1) g = 1;
