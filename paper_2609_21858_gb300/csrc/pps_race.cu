@@ -29,13 +29,13 @@
 #include "pps_internal.h"
 
 #ifndef PPS_UNITS
-#define PPS_UNITS 2  // 8-token units per lane per fast-loop iteration (2 Philox blocks each)
+#define PPS_UNITS 3  // 8-token units per lane per fast-loop iteration (2 Philox blocks each)
 #endif
 #ifndef PPS_PREFETCH
 #define PPS_PREFETCH 0  // 1: load the next iteration's vectors one iteration ahead (costs registers)
 #endif
 #ifndef PPS_RACE_MIN_BLOCKS
-#define PPS_RACE_MIN_BLOCKS 16  // one-warp CTAs resident per SM: 128 registers, no spills
+#define PPS_RACE_MIN_BLOCKS 12  // one-warp CTAs resident per SM (register budget 168, no spills)
 #endif
 
 namespace pps {
@@ -198,8 +198,8 @@ __device__ __forceinline__ uint32_t block_offset(int b) {
 }
 
 // the four logits of block b of an iteration's vectors d[]
-template <int DT>
-__device__ __forceinline__ void block_logits(const uint4 (&d)[4], int b, float (&l)[4]) {
+template <int DT, int N>
+__device__ __forceinline__ void block_logits(const uint4 (&d)[N], int b, float (&l)[4]) {
     if constexpr (DT == 1) {
         const uint4 v = d[b >> 1];
         const uint32_t x0 = (b & 1) ? v.z : v.x, x1 = (b & 1) ? v.w : v.y;
@@ -306,24 +306,42 @@ struct SlowState {
     WarpList L;
 };
 
-// Slow path of the fast loop: the blocks flagged in bm (bit b = block b of
-// this lane's iteration) have a token over the filter cut; regenerate their
-// words and offer their survivors.  The fast loop keeps no per-token state.
-template <int DT, int NB>
-__device__ __noinline__ SlowState slow_blocks(SlowState st, uint64_t key, uint64_t ctx, uint32_t pos, unsigned bm,
-                                              uint32_t cl, uint4 d0, uint4 d1, uint4 d2, uint4 d3, float c) {
+// Blocks flagged by the fast scan wait in a per-warp queue of Philox block
+// counters in shared memory (one iteration adds at most 32 x 2 x PPS_UNITS).
+constexpr int kQueueCap = 32 + 32 * 2 * PPS_UNITS;
+
+// Work off the queue: lane j regenerates the words of queued block j (32 at
+// a time), reloads its four logits, keys the tokens over the filter cut and
+// offers them.  Out of line; the fast scan itself makes no calls.
+template <int DT>
+__device__ __noinline__ SlowState flush_queue(SlowState st, const uint32_t* q, int qn, const char* row, float c,
+                                              uint64_t key, uint64_t ctx, uint32_t pos) {
     const int lane = threadIdx.x & 31;
     RowPhilox rp;
     rp.init(key, ctx, pos);
-    const uint4 d[4] = {d0, d1, d2, d3};
-#pragma unroll
-    for (int b = 0; b < NB; ++b) {
-        if (__any_sync(FULL, (bm >> b) & 1u)) {
-            float l[4];
-            block_logits<DT>(d, b, l);
-            block_survivors(st.L, rp, (bm >> b) & 1u, cl + block_offset<DT>(b), l, 0xfu, c, lane);
+    __syncwarp();
+    for (int base = 0; base < qn; base += 32) {
+        const bool mine = base + lane < qn;
+        const uint32_t cb = mine ? q[base + lane] : 0u;
+        float l[4] = {0.f, 0.f, 0.f, 0.f};
+        if (mine) {
+            if constexpr (DT == 1) {
+                const uint2 v = __ldg(reinterpret_cast<const uint2*>(row) + cb);
+                l[0] = bf16_lo(v.x);
+                l[1] = bf16_hi(v.x);
+                l[2] = bf16_lo(v.y);
+                l[3] = bf16_hi(v.y);
+            } else {
+                const uint4 v = __ldg(reinterpret_cast<const uint4*>(row) + cb);
+                l[0] = __uint_as_float(v.x);
+                l[1] = __uint_as_float(v.y);
+                l[2] = __uint_as_float(v.z);
+                l[3] = __uint_as_float(v.w);
+            }
         }
+        block_survivors(st.L, rp, mine, cb, l, 0xfu, c, lane);
     }
+    __syncwarp();
     return st;
 }
 
@@ -345,7 +363,7 @@ __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64
             const int64_t nt = min((int64_t)VW, V - v * VW);
             valid = (1u << nt) - 1u;
         }
-        const uint4 d[4] = {dv, dv, dv, dv};
+        const uint4 d[2] = {dv, dv};
         // the vector's blocks: bf16 2 (counters 2v, 2v+1), fp32 1 (counter v)
 #pragma unroll
         for (int h = 0; h < (DT == 1 ? 2 : 1); ++h) {
@@ -369,40 +387,32 @@ __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64
 
 // ---------------------------------------------------------------- the fast loop
 
-struct ScanStop {
-    int64_t it;   // iteration with a survivor (n_it when the scan ran to the end)
-    unsigned bm;  // its blocks over the filter cut (this lane)
-    uint32_t cl;  // its block counter base (this lane)
-    uint4 d0, d1, d2, d3;
-};
-
 // Fast scan over iterations [it0, n_it) of the full vectors starting at
 // vector v0 of a row.  Each iteration covers PPS_UNITS x 32 (bf16) or x 64
 // (fp32) vectors; every lane takes PPS_UNITS units of 8 tokens = 2 x
 // PPS_UNITS Philox blocks with counters cl + block_offset(b), cl advancing by
 // 64 x PPS_UNITS, so that many independent multiply chains are in flight per
-// lane.  A lane keeps only the per-block maxima of the filter sums.  The scan
-// makes no calls: it stops at the first iteration in which some lane has a
-// block over the cut and hands that iteration back, so that nothing the loop
-// keeps in registers (the row's round keys above all) lives across a call.
+// lane.  A lane keeps only the per-block maxima of the filter sums; a block
+// with a token over the cut is appended to the warp's queue.  The scan makes
+// no calls: it returns the iteration after which the queue holds 32 or more
+// blocks (n_it when it ran to the end), so that nothing it keeps in
+// registers (the row's round keys above all) lives across a call.
 template <int DT>
-__device__ __forceinline__ ScanStop fast_scan(const RowPhilox& rp, const char* row, int64_t v0, int64_t it0,
-                                              int64_t n_it, float c, float tz) {
+__device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* row, int64_t v0, int64_t it0,
+                                             int64_t n_it, float c, float tz, uint32_t* q, int& qn) {
     constexpr int NB = 2 * PPS_UNITS;          // Philox blocks per lane per iteration
     constexpr int ND = DT == 1 ? NB / 2 : NB;  // 16-byte vectors per lane per iteration
     constexpr int STEP = 32 * ND;              // vectors per iteration
     const int lane = threadIdx.x & 31;
     const uint4* p = reinterpret_cast<const uint4*>(row) + v0 + it0 * STEP + lane;
     uint32_t cl = (DT == 1 ? (uint32_t)(2 * (v0 + lane)) : (uint32_t)(v0 + lane)) + (uint32_t)(it0 * 64 * PPS_UNITS);
-    ScanStop out;
-    out.it = n_it;
 #if PPS_PREFETCH
     uint4 nx[ND];
 #pragma unroll
     for (int k = 0; k < ND; ++k) nx[k] = ldg_stream(p + 32 * k);
 #endif
     for (int64_t it = it0; it < n_it; ++it) {
-        uint4 d[4];
+        uint4 d[ND];
 #if PPS_PREFETCH
 #pragma unroll
         for (int k = 0; k < ND; ++k) d[k] = nx[k];
@@ -416,38 +426,43 @@ __device__ __forceinline__ ScanStop fast_scan(const RowPhilox& rp, const char* r
         for (int k = 0; k < ND; ++k) d[k] = ldg_stream(p + 32 * k);
         p += STEP;
 #endif
-#pragma unroll
-        for (int k = ND; k < 4; ++k) d[k] = d[0];
         unsigned bm = 0;
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
-            const uint4 q = rp.block(cl + block_offset<DT>(b));
+            const uint4 w = rp.block(cl + block_offset<DT>(b));
             float l[4];
             block_logits<DT>(d, b, l);
-            const float m01 = fmaxf(filter_sum(q.x, l[0], c, tz), filter_sum(q.y, l[1], c, tz));
-            const float m23 = fmaxf(filter_sum(q.z, l[2], c, tz), filter_sum(q.w, l[3], c, tz));
+            const float m01 = fmaxf(filter_sum(w.x, l[0], c, tz), filter_sum(w.y, l[1], c, tz));
+            const float m23 = fmaxf(filter_sum(w.z, l[2], c, tz), filter_sum(w.w, l[3], c, tz));
             bm |= (unsigned)(fmaxf(m01, m23) >= kFilterCut) << b;
         }
         if (__any_sync(FULL, bm != 0)) {
-            out.it = it;
-            out.bm = bm;
-            out.cl = cl;
-            out.d0 = d[0];
-            out.d1 = d[1];
-            out.d2 = d[2];
-            out.d3 = d[3];
-            break;
+            // append this lane's flagged blocks at its offset in the warp's batch
+            const int n = __popc(bm);
+            int off = n;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int t = __shfl_up_sync(FULL, off, o);
+                if (lane >= o) off += t;
+            }
+            const int total = __shfl_sync(FULL, off, 31);
+            off += qn - n;
+#pragma unroll
+            for (int b = 0; b < NB; ++b)
+                if ((bm >> b) & 1u) q[off++] = cl + block_offset<DT>(b);
+            qn += total;
+            if (qn >= 32) return it + 1;
         }
         cl += 64 * PPS_UNITS;
     }
-    return out;
+    return n_it;
 }
 
 // Stream vectors [v0, v1) of one row through the warp's list: full
 // iterations through the fast loop, the rest through the scalar tail.
 template <int DT, bool VEC>
 __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int64_t V, int64_t v0, int64_t v1,
-                                               float c, uint64_t key, uint64_t ctx, uint32_t pos) {
+                                               float c, uint64_t key, uint64_t ctx, uint32_t pos, uint32_t* q) {
     constexpr int VW = DT == 1 ? 8 : 4;
     constexpr int STEP = (DT == 1 ? 32 : 64) * PPS_UNITS;  // vectors per fast-loop iteration
     const int64_t nfull = V / VW;                           // vectors holding VW tokens
@@ -456,15 +471,14 @@ __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int
     SlowState st{L};
     int64_t base = v0;
     if (n_it > 0) {
-        constexpr int NB = 2 * PPS_UNITS;
         int64_t it = 0;
-        while (true) {
+        int qn = 0;
+        while (it < n_it) {
             RowPhilox rp;
             rp.init(key, ctx, pos);
-            const ScanStop sp = fast_scan<DT>(rp, row, v0, it, n_it, c, st.L.tz);
-            if (sp.it >= n_it) break;
-            st = slow_blocks<DT, NB>(st, key, ctx, pos, sp.bm, sp.cl, sp.d0, sp.d1, sp.d2, sp.d3, c);
-            it = sp.it + 1;
+            it = fast_scan<DT>(rp, row, v0, it, n_it, c, st.L.tz, q, qn);
+            if (qn > 0) st = flush_queue<DT>(st, q, qn, row, c, key, ctx, pos);
+            qn = 0;
         }
         base = v0 + n_it * STEP;
     }
@@ -732,6 +746,7 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
 
 template <int DT, bool VERIFY, bool VEC>
 __global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(const RaceArgs a) {
+    __shared__ uint32_t s_queue[kQueueCap];
     const int64_t NW = a.G;
     const int64_t gw = blockIdx.x;
     const int64_t g0 = gw * a.total / NW, g1 = (gw + 1) * a.total / NW;
@@ -753,7 +768,7 @@ __global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(con
 
         WarpList L;
         L.reset(kp);
-        stream_segment<DT, VEC>(L, row, a.V, v0, v1, c, key, ctx, pos);
+        stream_segment<DT, VEC>(L, row, a.V, v0, v1, c, key, ctx, pos, s_queue);
 
         finish_segment<DT, VERIFY>(a, r, gw, NW, v0, v1, L, kr, kp);
     }
