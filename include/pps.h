@@ -49,7 +49,8 @@ typedef enum {
     PPS_ERR_INVALID_ARG = 1, /* null pointer, size out of range, K > vocab, stride < vocab, T <= 0 ... */
     PPS_ERR_UNSUPPORTED = 2, /* dtype or mode not implemented                                        */
     PPS_ERR_WORKSPACE = 3,   /* workspace null or smaller than pps_workspace_size()                    */
-    PPS_ERR_CUDA = 4         /* a kernel launch or CUDA call failed                                    */
+    PPS_ERR_CUDA = 4,        /* a kernel launch or CUDA call failed                                    */
+    PPS_ERR_SIZE = 5         /* problem larger than the fixed scratch of pps_draft_list_noalloc        */
 } pps_status;
 
 typedef enum { PPS_F32 = 0, PPS_BF16 = 1 } pps_dtype;
@@ -170,6 +171,37 @@ pps_status pps_verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_node
  */
 pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,
                         float* out_score, double* out_sum, pps_stream_t stream);
+
+/*
+ * pps_draft_list_noalloc -- pps_draft_list for callers that must not
+ * allocate device memory per call and cannot hand the library a workspace:
+ * code running under an allocator that forbids new allocations once serving
+ * has started, plugin or callback hooks of an inference engine that receive
+ * only their input and output buffers, or deployments that must size every
+ * device buffer up front.  The paper has no counterpart; this is a packaging
+ * variant of the draft-list entry point, with the same arguments minus the
+ * workspace and the same outputs.
+ *
+ * Its scratch (per-row partial lists and arrival counters) is one file-scope
+ * device array of PPS_NOALLOC_SCRATCH_BYTES (about 1.8 MB) that every GPU
+ * which loads libpps holds until the process exits.  It serves at most
+ * PPS_NOALLOC_MAX_ROWS rows per call (larger n_rows returns PPS_ERR_SIZE)
+ * and caps the kernel grid at PPS_NOALLOC_MAX_WARPS warps.  The first call
+ * on a device looks the array's device address up (a CUDA runtime query, no
+ * allocation); make that first call before any stream capture.  Each call
+ * clears the counters it uses with an asynchronous memset on `stream` and
+ * allocates nothing.  All calls share the one array and it keeps the last
+ * call's contents: calls whose executions overlap on the GPU (on different
+ * streams, or from different threads without ordering) race on it, so the
+ * caller must serialise them.
+ */
+#define PPS_NOALLOC_MAX_ROWS 4096
+#define PPS_NOALLOC_MAX_WARPS 2432
+pps_status pps_draft_list_noalloc(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab,
+                                  int64_t row_stride, pps_row_ids ids, float temperature, int32_t K,
+                                  const int32_t* row_k, pps_draft_mode mode, int32_t* out_tok, float* out_key,
+                                  int32_t* out_mult, int32_t* out_ndistinct, int32_t* out_samples, uint32_t* status,
+                                  pps_stream_t stream);
 
 /* Raw words w(i, arrival) for i < vocab of n_rows rows -> out [n_rows, vocab]
  * (bit-exact check of the keyed source). */

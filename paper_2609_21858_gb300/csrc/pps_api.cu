@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <mutex>
 
 #include "pps.h"
 #include "pps_internal.h"
@@ -62,6 +63,38 @@ static RaceArgs base_args(const void* logits, pps_dtype dtype, int64_t n_rows, i
     return a;
 }
 
+// ---------------------------------------------------------------- fixed scratch of the no-alloc entry point
+//
+// The array below is the whole scratch of pps_draft_list_noalloc: partial
+// lists for PPS_NOALLOC_MAX_ROWS rows plus one per warp of a grid capped at
+// PPS_NOALLOC_MAX_WARPS warps (slot = warp + row), then one arrival counter
+// per row.  In host code its name is only a stand-in for the symbol, not a
+// device address; the address is looked up per device with
+// cudaGetSymbolAddress and cached.
+constexpr size_t kNoAllocPartialBytes = sizeof(Partial) * (size_t)(PPS_NOALLOC_MAX_ROWS + PPS_NOALLOC_MAX_WARPS);
+constexpr size_t kNoAllocCounterBytes = sizeof(uint32_t) * (size_t)PPS_NOALLOC_MAX_ROWS;
+constexpr size_t kNoAllocScratchBytes = kNoAllocPartialBytes + kNoAllocCounterBytes;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+static std::mutex g_noalloc_mu;
+static void* g_noalloc_ptr[kMaxDevices];
+
+// Device address of the scratch on the current device (set up on first use).
+static pps_status noalloc_scratch(void** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PPS_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices) return PPS_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return PPS_ERR_CUDA;
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return PPS_OK;
+}
+
 }  // namespace pps
 
 using namespace pps;
@@ -77,6 +110,7 @@ const char* pps_status_string(pps_status s) {
         case PPS_ERR_UNSUPPORTED: return "unsupported dtype or mode";
         case PPS_ERR_WORKSPACE: return "workspace missing or too small";
         case PPS_ERR_CUDA: return "CUDA launch failed";
+        case PPS_ERR_SIZE: return "problem larger than the no-alloc scratch";
     }
     return "unknown status";
 }
@@ -161,6 +195,46 @@ pps_status pps_verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_node
     const bool vec = vec_ok(p_logits, dtype, row_stride);
     a.G = race_grid(a.total, dt, true, vec);
     return launch_race(a, dt, true, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_draft_list_noalloc(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab,
+                                  int64_t row_stride, pps_row_ids ids, float temperature, int32_t K,
+                                  const int32_t* row_k, pps_draft_mode mode, int32_t* out_tok, float* out_key,
+                                  int32_t* out_mult, int32_t* out_ndistinct, int32_t* out_samples, uint32_t* status,
+                                  pps_stream_t stream) {
+    pps_status st = check_rows(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature);
+    if (st != PPS_OK) return st;
+    if (mode != PPS_DRAFT_DISTINCT && mode != PPS_DRAFT_IID) return PPS_ERR_UNSUPPORTED;
+    if (K < 1 || K > PPS_MAX_K || K > vocab) return PPS_ERR_INVALID_ARG;
+    if (n_rows == 0) return PPS_OK;
+    if (!out_tok || !out_mult || !out_ndistinct) return PPS_ERR_INVALID_ARG;
+    if (n_rows > PPS_NOALLOC_MAX_ROWS) return PPS_ERR_SIZE;
+    void* scratch = nullptr;
+    st = noalloc_scratch(&scratch);
+    if (st != PPS_OK) return st;
+    char* base = static_cast<char*>(scratch);
+    uint32_t* row_cnt = reinterpret_cast<uint32_t*>(base + kNoAllocPartialBytes);
+    // the arrival counters must start at zero; the partial lists need no clearing
+    if (cudaMemsetAsync(row_cnt, 0, sizeof(uint32_t) * (size_t)n_rows, (cudaStream_t)stream) != cudaSuccess)
+        return PPS_ERR_CUDA;
+    RaceArgs a = base_args(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature);
+    a.K = K;
+    a.row_k = row_k;
+    a.iid = mode == PPS_DRAFT_IID;
+    a.out_tok = out_tok;
+    a.out_key = out_key;
+    a.out_mult = out_mult;
+    a.out_nd = out_ndistinct;
+    a.out_samples = out_samples;
+    a.status = status;
+    a.partials = reinterpret_cast<Partial*>(base);
+    a.row_cnt = row_cnt;
+    a.seq_cnt = nullptr;
+    const int dt = dtype == PPS_BF16 ? 1 : 0;
+    const bool vec = vec_ok(q_logits, dtype, row_stride);
+    a.G = race_grid(a.total, dt, false, vec);
+    if (a.G > PPS_NOALLOC_MAX_WARPS) a.G = PPS_NOALLOC_MAX_WARPS;
+    return launch_race(a, dt, false, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
 }
 
 pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,

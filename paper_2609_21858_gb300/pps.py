@@ -14,7 +14,8 @@ import torch
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", "libpps.so")
 
-OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_SIZE = 0, 1, 2, 3, 4, 5
+NOALLOC_MAX_ROWS = 4096
 F32, BF16 = 0, 1
 DISTINCT, IID = 0, 1
 FLAG_GUARD, FLAG_LOGIT_RANGE = 1, 2
@@ -58,6 +59,9 @@ def lib():
             L.pps_verify_tree.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, i32, i32, vp, vp, i64, vp,
                                           vp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
             L.pps_verify_tree.restype = ctypes.c_int
+            L.pps_draft_list_noalloc.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, i32, vp, ctypes.c_int,
+                                                 vp, vp, vp, vp, vp, vp, vp]
+            L.pps_draft_list_noalloc.restype = ctypes.c_int
             L.pps_wm_score.argtypes = [vp, RowIds, i64, i32, vp, vp, vp, vp]
             L.pps_wm_score.restype = ctypes.c_int
             L.pps_philox_words.argtypes = [RowIds, i64, i64, i32, vp, vp]
@@ -145,6 +149,29 @@ def draft_list(q_logits, key, ctx, pos, K: int, row_k=None, mode: int = DISTINCT
                                 _ptr(out.get("key")), _ptr(out["mult"]), _ptr(out["ndist"]), _ptr(out.get("samples")),
                                 _ptr(status), _ptr(ws), ws.numel(), _stream(stream))
     _check("pps_draft_list", code)
+    return out
+
+
+def draft_list_noalloc(q_logits, key, ctx, pos, K: int, row_k=None, mode: int = DISTINCT, temperature: float = 1.0,
+                       status=None, out=None, keys: bool = True, samples: bool = True, stream=None):
+    """pps_draft_list_noalloc: pps_draft_list without a workspace, for callers
+    that cannot allocate device memory per call (the library's built-in
+    scratch serves up to NOALLOC_MAX_ROWS rows; calls must not overlap on the GPU)."""
+    n, V, stride = _rows(q_logits)
+    dev = q_logits.device
+    if out is None:
+        out = dict(tok=torch.empty(n, K, dtype=torch.int32, device=dev),
+                   key=torch.empty(n, K, dtype=torch.float32, device=dev) if keys else None,
+                   mult=torch.empty(n, K, dtype=torch.int32, device=dev),
+                   ndist=torch.empty(n, dtype=torch.int32, device=dev),
+                   samples=torch.empty(n, K, dtype=torch.int32, device=dev) if samples else None)
+    if row_k is not None and (row_k.dtype != torch.int32 or not row_k.is_cuda):
+        raise TypeError("row_k must be a CUDA int32 tensor")
+    code = lib().pps_draft_list_noalloc(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
+                                        float(temperature), int(K), _ptr(row_k), int(mode), _ptr(out["tok"]),
+                                        _ptr(out.get("key")), _ptr(out["mult"]), _ptr(out["ndist"]),
+                                        _ptr(out.get("samples")), _ptr(status), _stream(stream))
+    _check("pps_draft_list_noalloc", code)
     return out
 
 
