@@ -29,6 +29,53 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "verified rows/s and GB/s vs HBM peak at V=128256, K=8, B=64 (1xGB300)"
+WIDE_MULS_PER_TOKEN = 4.5
+WIDE_MULS_PER_SM_CLK = 32
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "race_kernel_zipf_k8_traffic.txt")
+
+
+def kernel_source_digest() -> str:
+    """sha1 over the CUDA sources of libpps (a recorded ncu figure is stale once this changes)."""
+    import hashlib
+    h = hashlib.sha1()
+    csrc = os.path.join(ROOT, "paper_2609_21858_gb300", "csrc")
+    for name in ("pps_race.cu", "pps_device.cuh", "pps_internal.h"):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + b"\0" + f.read())
+    return h.hexdigest()
+
+
+def philox_only_rate(dev) -> float:
+    """Tokens per second of the keyed source alone (4 tokens per Philox block)."""
+    from paper_2609_21858_gb300 import pps
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    out_len = sms * 8 * 256
+    n_blocks = out_len * 512
+    for _ in range(3):
+        pps.selftest_philox_rate(n_blocks, out_len)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(5):
+        pps.selftest_philox_rate(n_blocks, out_len)
+    e1.record()
+    torch.cuda.synchronize(dev)
+    return 5 * 4 * n_blocks / (e0.elapsed_time(e1) / 1e3)
+
+
+def _traffic(which: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current kernel."""
+    try:
+        kv = {}
+        with open(TRAFFIC_FILE) as f:
+            for line in f:
+                if "=" in line and not line.startswith("#"):
+                    k, v = line.strip().split("=", 1)
+                    kv[k.strip()] = v.strip()
+        if kv.get("kernel_source_sha1") != kernel_source_digest():
+            return None
+        return float(kv[f"{which}_dram_bytes_per_launch"])
+    except Exception:
+        return None
 
 
 def _peaks():
@@ -152,6 +199,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="zipf_k8")
+    ap.add_argument("--n-seq", type=int, default=None, help="override the number of sequences (smaller profiling cases)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -169,7 +217,7 @@ def main():
     from paper_2609_21858_gb300 import pps
     pps.lib()
     dev = torch.device("cuda", local)
-    wl = synth.make_workload(args.workload, device=dev, seed=None)
+    wl = synth.make_workload(args.workload, device=dev, n_seq=args.n_seq)
     t = wl.tree
     g = lambda x: torch.as_tensor(np.asarray(x)).to(dev).contiguous()
     row_k, seq_off, ndr, child = g(t.row_k), g(t.seq_off), g(t.node_draft_row), g(t.child_node)
@@ -238,6 +286,15 @@ def main():
     ach_v = bytes_verify / (t_verify / 1e3) / 1e9
     ach_d = bytes_draft / (t_draft / 1e3) / 1e9
     ach_all = (bytes_verify + bytes_draft) / (ms_step / 1e3) / 1e9
+    # integer-multiply roof: 18 wide 32x32->64 multiplies per Philox4x32-10 block (rounds 1-2 of a
+    # row share two products) = 4.5 per token; the multiply pipe retires 32 per SM per clock
+    tok_verify = t.n_nodes * wl.vocab
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    clk = (clocks.get("sm_mhz") or 2070.0) * 1e6
+    mul_peak = sms * WIDE_MULS_PER_SM_CLK * clk / 1e12
+    mul_ach = tok_verify * WIDE_MULS_PER_TOKEN / (t_verify / 1e3) / 1e12
+    traffic = _traffic("verify")
+    philox_tok_s = philox_only_rate(dev) if rank == 0 else None
     emitted = float(vout["n_emitted"].sum().item())
 
     # ---- end to end through host buffers
@@ -297,10 +354,18 @@ def main():
                        "rows_per_step": rows_per_step, "l2": "inputs (1.21 GB) larger than L2, no flush",
                        "parallelism": f"replicas x{world}"},
             "gb_per_s": ach_all, "tokens_per_s": emitted * world / (ms_step / 1e3),
-            "roofline": {"bound": "hbm", "achieved": ach_v, "peak": peak, "unit": "GB/s", "frac": ach_v / peak,
-                         "traffic": None, "kernel": "race_kernel<bf16, verify> (pps_verify_tree)",
-                         "peak_kind": peak_kind, "algorithmic_bytes": bytes_verify, "ms": t_verify},
-            "roofline_draft": {"achieved": ach_d, "frac": ach_d / peak, "ms": t_draft, "algorithmic_bytes": bytes_draft},
+            "roofline": {"bound": "alu", "achieved": mul_ach, "peak": mul_peak, "unit": "T wide-mul/s",
+                         "frac": mul_ach / mul_peak, "traffic": traffic,
+                         "kernel": "race_kernel (pps_verify_tree)", "ms": t_verify,
+                         "peak_kind": f"derived: {sms} SMs x {WIDE_MULS_PER_SM_CLK} 32x32->64 multiplies/clk x "
+                                      f"{clk / 1e6:.0f} MHz (median sampled SM clock)",
+                         "work": f"{WIDE_MULS_PER_TOKEN} wide multiplies per token x {tok_verify} tokens",
+                         "philox_only_tok_s": philox_tok_s,
+                         "tok_s": tok_verify / (t_verify / 1e3)},
+            "roofline_hbm": {"bound": "hbm", "achieved": ach_v, "peak": peak, "unit": "GB/s", "frac": ach_v / peak,
+                             "peak_kind": peak_kind, "algorithmic_bytes": bytes_verify, "traffic": traffic},
+            "roofline_draft": {"achieved_gbs": ach_d, "frac_hbm": ach_d / peak, "ms": t_draft,
+                               "algorithmic_bytes": bytes_draft},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": 2 * args.steps, "clocks": clocks,
             "mean_accept_len": float(vout["accept_len"].float().mean().item()),
         }

@@ -214,6 +214,13 @@ pps_status pps_philox_words(pps_row_ids ids, int64_t n_rows, int64_t vocab, int3
  * difference to out_max_err[0] (device float, must hold 0 before the call). */
 pps_status pps_selftest_key_error(uint64_t w_begin, uint64_t w_end, float* out_max_err, pps_stream_t stream);
 
+/* Throughput self-test of the keyed source alone: generates n_blocks Philox
+ * blocks (4 words each) with the streaming kernels' row-specialised
+ * generator, in a grid of out_len / 256 CTAs of 256 threads, and writes one
+ * folded word per thread to out [out_len] (device, out_len >= 256).  Timing
+ * it gives the multiply-bound ceiling of the race kernels. */
+pps_status pps_selftest_philox_rate(uint64_t n_blocks, uint32_t* out, int32_t out_len, pps_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -261,4 +261,9 @@ pps_status pps_selftest_key_error(uint64_t w_begin, uint64_t w_end, float* out_m
     return launch_selftest(w_begin, w_end, out_max_err, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
 }
 
+pps_status pps_selftest_philox_rate(uint64_t n_blocks, uint32_t* out, int32_t out_len, pps_stream_t stream) {
+    if (!out || out_len < 256 || n_blocks == 0) return PPS_ERR_INVALID_ARG;
+    return launch_philox_rate(n_blocks, out, out_len, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
 }  // extern "C"

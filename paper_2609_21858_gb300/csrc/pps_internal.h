@@ -78,5 +78,6 @@ cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const ui
 cudaError_t launch_words(const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int64_t n_rows, int64_t V,
                          int32_t arrival, uint32_t* out, cudaStream_t stream);
 cudaError_t launch_selftest(uint64_t w_begin, uint64_t w_end, float* out, cudaStream_t stream);
+cudaError_t launch_philox_rate(uint64_t n_blocks, uint32_t* out, int out_len, cudaStream_t stream);
 
 }  // namespace pps

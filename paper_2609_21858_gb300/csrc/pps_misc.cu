@@ -126,6 +126,31 @@ __global__ void selftest_kernel(uint64_t w0, uint64_t w1, float* out) {
     if ((threadIdx.x & 31) == 0) atomicMax(reinterpret_cast<unsigned int*>(out), __float_as_uint(worst));
 }
 
+// Philox-only throughput: every thread generates blocks c0 = t, t + stride, ...
+// with the row-specialised generator of the streaming kernels and folds the
+// words into one value, so the kernel is bound by the Philox multiplies alone
+// (the ceiling of the race kernels on bf16 rows).
+__global__ void __launch_bounds__(256) philox_rate_kernel(uint64_t key, uint64_t ctx, uint32_t pos, uint64_t n_blocks,
+                                                          uint32_t* out) {
+    RowPhilox rp;
+    rp.init(key, ctx, pos);
+    uint32_t acc = 0;
+    const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+    for (uint64_t b = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; b < n_blocks; b += 2 * stride) {
+        const uint4 v0 = rp.block((uint32_t)b);
+        const uint4 v1 = rp.block((uint32_t)(b + stride));
+        acc ^= v0.x ^ v0.y ^ v0.z ^ v0.w ^ v1.x ^ v1.y ^ v1.z ^ v1.w;
+    }
+    out[(uint64_t)blockIdx.x * blockDim.x + threadIdx.x] = acc;
+}
+
+cudaError_t launch_philox_rate(uint64_t n_blocks, uint32_t* out, int out_len, cudaStream_t stream) {
+    int blocks = out_len / 256;
+    if (blocks < 1) return cudaErrorInvalidValue;
+    philox_rate_kernel<<<blocks, 256, 0, stream>>>(0x0123456789abcdefull, 0xfedcba9876543210ull, 7u, n_blocks, out);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
                             int64_t n, int32_t n_seg, const int64_t* seg_off, float* out_score, double* out_sum,
                             cudaStream_t stream) {

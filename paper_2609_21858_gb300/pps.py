@@ -66,6 +66,8 @@ def lib():
             L.pps_wm_score.restype = ctypes.c_int
             L.pps_philox_words.argtypes = [RowIds, i64, i64, i32, vp, vp]
             L.pps_philox_words.restype = ctypes.c_int
+            L.pps_selftest_philox_rate.argtypes = [u64, vp, i32, vp]
+            L.pps_selftest_philox_rate.restype = ctypes.c_int
             L.pps_selftest_key_error.argtypes = [u64, u64, vp, vp]
             L.pps_selftest_key_error.restype = ctypes.c_int
             _lib = L
@@ -238,3 +240,10 @@ def selftest_key_error(w_begin: int = 0, w_end: int = 1 << 32, stream=None) -> f
     out = torch.zeros(1, dtype=torch.float32, device="cuda")
     _check("pps_selftest_key_error", lib().pps_selftest_key_error(w_begin, w_end, _ptr(out), _stream(stream)))
     return float(out.item())
+
+
+def selftest_philox_rate(n_blocks: int, out_len: int, stream=None):
+    """Launch the Philox-only throughput kernel (returns the folded words)."""
+    out = torch.empty(out_len, dtype=torch.int32, device="cuda")
+    _check("pps_selftest_philox_rate", lib().pps_selftest_philox_rate(n_blocks, _ptr(out), out_len, _stream(stream)))
+    return out
