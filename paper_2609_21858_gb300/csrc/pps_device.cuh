@@ -136,6 +136,45 @@ struct RowPhilox {
         }
         return make_uint4(x0, x1, x2, x3);
     }
+
+    // NB blocks at counters c0[b], computed round-major so that the NB
+    // independent multiply chains are interleaved instruction by instruction
+    template <int NB>
+    __device__ __forceinline__ void blocks(const uint32_t (&c0)[NB], uint4 (&out)[NB]) const {
+        uint32_t x0[NB], x1[NB], x2[NB], x3[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            uint32_t hi0, lo0;
+            mulhilo(kPhiloxM0, c0[b], hi0, lo0);
+            x3[b] = lo0;
+            x2[b] = hi0 ^ r1_c3k;
+        }
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            uint32_t h1, l1;
+            mulhilo(kPhiloxM1, x2[b], h1, l1);
+            x0[b] = h1 ^ r2_f;
+            x1[b] = l1;
+            x2[b] = x3[b] ^ r2_gh;
+            x3[b] = r2_lo0;
+        }
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+                uint32_t a0, b0, a1, b1;
+                mulhilo(kPhiloxM0, x0[b], a0, b0);
+                mulhilo(kPhiloxM1, x2[b], a1, b1);
+                const uint32_t n0 = a1 ^ x1[b] ^ rk0[r], n2 = a0 ^ x3[b] ^ rk1[r];
+                x0[b] = n0;
+                x1[b] = b1;
+                x2[b] = n2;
+                x3[b] = b0;
+            }
+        }
+#pragma unroll
+        for (int b = 0; b < NB; ++b) out[b] = make_uint4(x0[b], x1[b], x2[b], x3[b]);
+    }
 };
 
 // ------------------------------------------------------------------ transforms
@@ -214,18 +253,36 @@ __device__ __forceinline__ float ex2_approx(float x) {
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
-__device__ __forceinline__ float filter_sum(uint32_t w, float l, float c, float tz) {
-    float T = ex2_approx(fmaf(l, c, tz));
+#ifndef PPS_FILTER
+#define PPS_FILTER 0
+#endif
+#if PPS_FILTER == 0
+// 2^23 + (w >> 9) as fp32 bits from one mad.hi; cut 2^24 - 2, T scaled by 2^23
+constexpr float kFilterScaleLog2 = 23.0f;
+constexpr float kFilterCut = 16777214.0f;  // 2^24 - 2
+__device__ __forceinline__ float filter_word(uint32_t w) {
     uint32_t bb;
     asm("mad.hi.u32 %0, %1, %2, %3;" : "=r"(bb) : "r"(w), "r"(1u << 23), "r"(0x4b000000u));
-    return T + __uint_as_float(bb);
+    return __uint_as_float(bb);
 }
-constexpr float kFilterCut = 16777214.0f;  // 2^24 - 2
+#else
+// 0x4b000000 | (w >> 8) as fp32 bits from one byte permute: 2^23 + (w >> 8) for
+// w < 2^31 and 2 (w >> 8) above; the token can be dropped when T + f <= 2^25 - 2
+// (T scaled by 2^25), and the fp32 sum errs by at most 2, so the cut is 2^25 - 4.
+// Below 2^31 the test drops only words with u < 3/4 - e_z, inside the safe
+// region u <= 1 - e_z.
+constexpr float kFilterScaleLog2 = 25.0f;
+constexpr float kFilterCut = 33554428.0f;  // 2^25 - 4
+__device__ __forceinline__ float filter_word(uint32_t w) { return __uint_as_float(__byte_perm(w, 0x4bu, 0x4321)); }
+#endif
+__device__ __forceinline__ float filter_sum(uint32_t w, float l, float c, float tz) {
+    return ex2_approx(fmaf(l, c, tz)) + filter_word(w);
+}
 __device__ __forceinline__ bool filter_pass(uint32_t w, float l, float c, float tz) {
     return filter_sum(w, l, c, tz) >= kFilterCut;
 }
 __device__ __forceinline__ float filter_tz(float theta) {
-    return theta + (kFilterMargin + kLog2Ln2 + 23.0f);
+    return theta + (kFilterMargin + kLog2Ln2 + kFilterScaleLog2);
 }
 
 // bf16 -> fp32 (exact)

@@ -34,6 +34,12 @@
 #ifndef PPS_PREFETCH
 #define PPS_PREFETCH 0  // 1: load the next iteration's vectors one iteration ahead (costs registers)
 #endif
+#ifndef PPS_INTERLEAVE
+#define PPS_INTERLEAVE 0  // 1: Philox blocks of an iteration computed round-major
+#endif
+#ifndef PPS_PACKED
+#define PPS_PACKED 0  // 1: pairs of filter sums with packed fp32x2 fma/add
+#endif
 #ifndef PPS_RACE_MIN_BLOCKS
 #define PPS_RACE_MIN_BLOCKS 12  // one-warp CTAs resident per SM (register budget 168, no spills)
 #endif
@@ -387,6 +393,32 @@ __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64
 
 // ---------------------------------------------------------------- the fast loop
 
+// filter sums of the four tokens of one block, max of the four
+__device__ __forceinline__ float block_filter_max(const uint4& w, const float (&l)[4], float c, float tz) {
+#if PPS_PACKED
+    float z0, z1, z2, z3;
+    asm("{\n\t.reg .b64 a, b, t, d;\n\t"
+        "mov.b64 a, {%4, %5};\n\tmov.b64 b, {%8, %8};\n\tmov.b64 t, {%9, %9};\n\t"
+        "fma.rn.f32x2 d, a, b, t;\n\tmov.b64 {%0, %1}, d;\n\t"
+        "mov.b64 a, {%6, %7};\n\tfma.rn.f32x2 d, a, b, t;\n\tmov.b64 {%2, %3}, d;\n\t}"
+        : "=f"(z0), "=f"(z1), "=f"(z2), "=f"(z3)
+        : "f"(l[0]), "f"(l[1]), "f"(l[2]), "f"(l[3]), "f"(c), "f"(tz));
+    const float t0 = ex2_approx(z0), t1 = ex2_approx(z1), t2 = ex2_approx(z2), t3 = ex2_approx(z3);
+    float s0, s1, s2, s3;
+    asm("{\n\t.reg .b64 a, b, d;\n\t"
+        "mov.b64 a, {%4, %5};\n\tmov.b64 b, {%8, %9};\n\tadd.rn.f32x2 d, a, b;\n\tmov.b64 {%0, %1}, d;\n\t"
+        "mov.b64 a, {%6, %7};\n\tmov.b64 b, {%10, %11};\n\tadd.rn.f32x2 d, a, b;\n\tmov.b64 {%2, %3}, d;\n\t}"
+        : "=f"(s0), "=f"(s1), "=f"(s2), "=f"(s3)
+        : "f"(t0), "f"(t1), "f"(t2), "f"(t3), "f"(filter_word(w.x)), "f"(filter_word(w.y)),
+          "f"(filter_word(w.z)), "f"(filter_word(w.w)));
+    return fmaxf(fmaxf(s0, s1), fmaxf(s2, s3));
+#else
+    const float m01 = fmaxf(filter_sum(w.x, l[0], c, tz), filter_sum(w.y, l[1], c, tz));
+    const float m23 = fmaxf(filter_sum(w.z, l[2], c, tz), filter_sum(w.w, l[3], c, tz));
+    return fmaxf(m01, m23);
+#endif
+}
+
 // Fast scan over iterations [it0, n_it) of the full vectors starting at
 // vector v0 of a row.  Each iteration covers PPS_UNITS x 32 (bf16) or x 64
 // (fp32) vectors; every lane takes PPS_UNITS units of 8 tokens = 2 x
@@ -427,15 +459,27 @@ __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* ro
         p += STEP;
 #endif
         unsigned bm = 0;
+#if PPS_INTERLEAVE
+        uint32_t cb[NB];
+        uint4 wb[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) cb[b] = cl + block_offset<DT>(b);
+        rp.blocks<NB>(cb, wb);
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            float l[4];
+            block_logits<DT>(d, b, l);
+            bm |= (unsigned)(block_filter_max(wb[b], l, c, tz) >= kFilterCut) << b;
+        }
+#else
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
             const uint4 w = rp.block(cl + block_offset<DT>(b));
             float l[4];
             block_logits<DT>(d, b, l);
-            const float m01 = fmaxf(filter_sum(w.x, l[0], c, tz), filter_sum(w.y, l[1], c, tz));
-            const float m23 = fmaxf(filter_sum(w.z, l[2], c, tz), filter_sum(w.w, l[3], c, tz));
-            bm |= (unsigned)(fmaxf(m01, m23) >= kFilterCut) << b;
+            bm |= (unsigned)(block_filter_max(w, l, c, tz) >= kFilterCut) << b;
         }
+#endif
         if (__any_sync(FULL, bm != 0)) {
             // append this lane's flagged blocks at its offset in the warp's batch
             const int n = __popc(bm);
