@@ -40,6 +40,12 @@ constexpr float kFilterMargin = 0.015625f;
 
 __device__ __forceinline__ float key_err_bound(float k) { return kErrAbs + kErrRel * (fabsf(k) + kErrSpan); }
 
+// Filter bound for a list whose k-th key is t: t plus four error bounds, so
+// that a row's k-th key tau <= t and a drop bound of filter_slack(t) always
+// pass the completeness test tau + err(tau) + err(bound) < bound (|tau| grows
+// by at most t - tau, and err by kErrRel times that).  +inf stays +inf.
+__device__ __forceinline__ float filter_slack(float t) { return t + 4.0f * key_err_bound(t); }
+
 // ------------------------------------------------------------------ Philox
 
 __device__ __forceinline__ void mulhilo(uint32_t a, uint32_t b, uint32_t& hi, uint32_t& lo) {

@@ -229,21 +229,31 @@ struct WarpList {
     int li;
     float th;  // key of entry kp-1 (+inf while not full)
     int thi;
-    float tz;  // filter threshold (pps_device.cuh)
+    float tf;  // filter bound: the filter drops only tokens with keys >= tf; never rises
+    float tz;  // filter threshold for tf (pps_device.cuh)
     int kp;
+    int k;     // entries the row needs (kp > k leaves room for near ties)
 
-    __device__ __forceinline__ void reset(int kp_) {
+    __device__ __forceinline__ void reset(int kp_, int k_) {
         lk = kInf;
         li = INT_MAX;
         th = kInf;
         thi = INT_MAX;
+        tf = kInf;
         tz = kInf;
         kp = kp_;
+        k = k_;
     }
+    // lower tf to b (no effect when b >= tf)
+    __device__ __forceinline__ void bound(float b) {
+        tf = fminf(tf, b);
+        tz = filter_tz(tf);
+    }
+    // after the list changed: tf <= min(th, (entry k-1) + filter_slack)
     __device__ __forceinline__ void refresh() {
         th = __shfl_sync(FULL, lk, kp - 1);
         thi = __shfl_sync(FULL, li, kp - 1);
-        tz = filter_tz(th);
+        bound(fminf(th, filter_slack(__shfl_sync(FULL, lk, k - 1))));
     }
 };
 
@@ -391,6 +401,47 @@ __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64
     return st;
 }
 
+// A filter bound for an empty list.  Lane j keys exactly (key32, the list's
+// own key) the 8 tokens of its first unit of the segment's first fast
+// iteration and keeps its smallest; the bound is filter_slack of the k-th
+// smallest of the 32 lane minima.  Those k tokens lie in the segment, so the
+// row's k-th key is at most their largest, and the slack keeps every token
+// that could tie with it (tf itself is recorded as a drop bound).  Without
+// it every block of the first iteration would pass the filter and be queued.
+template <int DT>
+__device__ __noinline__ float seed_theta(const char* row, int64_t v0, float c, uint64_t key, uint64_t ctx,
+                                         uint32_t pos, int k) {
+    const int lane = threadIdx.x & 31;
+    RowPhilox rp;
+    rp.init(key, ctx, pos);
+    const uint4* p = reinterpret_cast<const uint4*>(row) + v0 + lane;
+    uint4 d[2];
+    d[0] = __ldg(p);
+    d[1] = DT == 1 ? d[0] : __ldg(p + 32);
+    const uint32_t cl = DT == 1 ? (uint32_t)(2 * (v0 + lane)) : (uint32_t)(v0 + lane);
+    float bk = kInf;
+    int bi = INT_MAX;
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+        const uint32_t cb = cl + block_offset<DT>(b);
+        const uint4 q = rp.block(cb);
+        const uint32_t wq[4] = {q.x, q.y, q.z, q.w};
+        float l[4];
+        block_logits<DT>(d, b, l);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float k = key32(wq[e], l[e], c);
+            const int i = (int)(4 * cb + e);
+            if (lex_less(k, i, bk, bi)) {
+                bk = k;
+                bi = i;
+            }
+        }
+    }
+    warp_sort(bk, bi, lane);
+    return filter_slack(__shfl_sync(FULL, bk, k - 1));
+}
+
 // ---------------------------------------------------------------- the fast loop
 
 // filter sums of the four tokens of one block, max of the four
@@ -515,6 +566,7 @@ __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int
     SlowState st{L};
     int64_t base = v0;
     if (n_it > 0) {
+        st.L.bound(seed_theta<DT>(row, v0, c, key, ctx, pos, st.L.k));
         int64_t it = 0;
         int qn = 0;
         while (it < n_it) {
@@ -729,7 +781,7 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
     float lk = L.lk;
     int li = L.li;
     // every token of the segment left out of the list has a key >= theta_drop
-    float theta_drop = L.th;
+    float theta_drop = fminf(L.th, L.tf);
     bool final_here = v0 == 0 && v1 == nv;
     if (!final_here) {
         // publish this segment's list; the last warp of the row merges all segments
@@ -811,7 +863,7 @@ __global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(con
         const char* row = reinterpret_cast<const char*>(a.logits) + (size_t)r * (size_t)a.stride * esz;
 
         WarpList L;
-        L.reset(kp);
+        L.reset(kp, kr);
         stream_segment<DT, VEC>(L, row, a.V, v0, v1, c, key, ctx, pos, s_queue);
 
         finish_segment<DT, VERIFY>(a, r, gw, NW, v0, v1, L, kr, kp);
