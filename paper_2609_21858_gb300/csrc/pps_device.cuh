@@ -96,7 +96,15 @@ struct RowPhilox {
     uint32_t r2_lo0;          // lo(M0 * y0)                             (round 2, word 3)
     uint32_t rk0[8], rk1[8];  // keys of rounds 3..10
 
+    // Called by all 32 lanes of a warp with the same row.  The warp reductions
+    // (of equal values) mark the row constants as warp-uniform, so the
+    // compiler keeps them and the round keys in uniform registers.
     __device__ __forceinline__ void init(uint64_t key, uint64_t ctx, uint32_t pos) {
+        key = ((uint64_t)__reduce_or_sync(0xffffffffu, (uint32_t)(key >> 32)) << 32) |
+              __reduce_or_sync(0xffffffffu, (uint32_t)key);
+        ctx = ((uint64_t)__reduce_or_sync(0xffffffffu, (uint32_t)(ctx >> 32)) << 32) |
+              __reduce_or_sync(0xffffffffu, (uint32_t)ctx);
+        pos = __reduce_or_sync(0xffffffffu, pos);
         const uint32_t k0 = (uint32_t)key, k1 = (uint32_t)(key >> 32);
         const uint32_t c2 = (uint32_t)ctx, c3 = (uint32_t)(ctx >> 32);
         uint32_t hi1, lo1;
