@@ -243,14 +243,20 @@ def main():
                 score_sum=torch.empty(t.n_seq, dtype=torch.float64, device=dev))
     stream = torch.cuda.current_stream(dev)
 
+    def draft(q):
+        pps.draft_list(q, dk, dc, dp, t.K, row_k=row_k, ws=ws_d, status=status, out=dout, stream=stream)
+
+    def verify(p):
+        pps.verify_tree(p, nk, nc, np_, t.gamma, seq_off, ndr, dout["tok"], dout["ndist"], child, ws=ws_v,
+                        status=status, out=vout, stream=stream)
+
     def step(q, p, ev=None):
         if ev is not None:
             ev[0].record(stream)
-        pps.draft_list(q, dk, dc, dp, t.K, row_k=row_k, ws=ws_d, status=status, out=dout, stream=stream)
+        draft(q)
         if ev is not None:
             ev[1].record(stream)
-        pps.verify_tree(p, nk, nc, np_, t.gamma, seq_off, ndr, dout["tok"], dout["ndist"], child, ws=ws_v,
-                        status=status, out=vout, stream=stream)
+        verify(p)
         if ev is not None:
             ev[2].record(stream)
 
@@ -314,7 +320,10 @@ def main():
     philox_tok_s = philox_only_rate(dev) if rank == 0 else None
     emitted = float(vout["n_emitted"].sum().item())
 
-    # ---- end to end through host buffers
+    # ---- end to end through host buffers: every step copies its q and p logits from pinned host
+    # memory (copy stream, two device buffers used in turn) and reads its emitted tokens and score
+    # sums back.  The draft kernel waits only for q, the verify kernel for p, and the next step's
+    # copies overlap this step's kernels.
     e2e = None
     if args.e2e_steps > 0:
         hq = torch.empty(q.shape, dtype=q.dtype, pin_memory=True)
@@ -324,31 +333,47 @@ def main():
         h_em = torch.empty(vout["emitted"].shape, dtype=torch.int32, pin_memory=True)
         h_ne = torch.empty(t.n_seq, dtype=torch.int32, pin_memory=True)
         h_ss = torch.empty(t.n_seq, dtype=torch.float64, pin_memory=True)
-        dq, dp2 = torch.empty_like(q), torch.empty_like(p)
+        bufs = [(torch.empty_like(q), torch.empty_like(p)) for _ in range(2)]
+        copy_stream = torch.cuda.Stream(dev)
+        freed = [torch.cuda.Event() for _ in range(2)]
+        for f in freed:
+            f.record(stream)
 
-        def e2e_step():
-            dq.copy_(hq, non_blocking=True)
-            dp2.copy_(hp, non_blocking=True)
-            step(dq, dp2)
+        def e2e_step(k):
+            dq, dp2 = bufs[k & 1]
+            ev_q, ev_p = torch.cuda.Event(), torch.cuda.Event()
+            copy_stream.wait_event(freed[k & 1])  # the kernels of step k-2 are done with this buffer
+            with torch.cuda.stream(copy_stream):
+                dq.copy_(hq, non_blocking=True)
+                ev_q.record(copy_stream)
+                dp2.copy_(hp, non_blocking=True)
+                ev_p.record(copy_stream)
+            stream.wait_event(ev_q)
+            draft(dq)
+            stream.wait_event(ev_p)
+            verify(dp2)
+            freed[k & 1].record(stream)
             h_em.copy_(vout["emitted"], non_blocking=True)
             h_ne.copy_(vout["n_emitted"], non_blocking=True)
             h_ss.copy_(vout["score_sum"], non_blocking=True)
 
-        e2e_step()
+        e2e_step(0)
         torch.cuda.synchronize(dev)
         barrier(world)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for _ in range(args.e2e_steps):
-            e2e_step()
+        copy_stream.wait_event(e0)
+        for k in range(args.e2e_steps):
+            e2e_step(k)
         e1.record(stream)
         torch.cuda.synchronize(dev)
         e_ms = max_over_ranks(e0.elapsed_time(e1) / args.e2e_steps, world)
         e2e = {"value": rows_per_step * world / (e_ms / 1e3), "unit": "rows/s",
                "h2d_bytes_per_step": int(hq.numel() * esz + hp.numel() * esz),
                "d2h_bytes_per_step": int(h_em.numel() * 4 + h_ne.numel() * 4 + h_ss.numel() * 8),
-               "ms_per_step": e_ms}
-        del hq, hp, dq, dp2
+               "ms_per_step": e_ms,
+               "pipeline": "q and p copies on a copy stream, two device buffers; kernels wait per input"}
+        del hq, hp, bufs
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
