@@ -77,6 +77,8 @@ def lib():
             L.orc_wm_score.restype = None
             L.orc_words.argtypes = [i64, i64, u64p, u64p, u32p, i32, u32p]
             L.orc_words.restype = None
+            L.orc_truncate_rows.argtypes = [f32p, i64, i64, i64, f64, i32, f64, f32p, f64p]
+            L.orc_truncate_rows.restype = None
             L.orc_set_threads.argtypes = [ctypes.c_int]
             L.orc_set_threads.restype = ctypes.c_int
             _lib = L
@@ -202,3 +204,14 @@ def wm_score(tokens, key, ctx, pos, seg_off=None):
                        _ptr(pos, ctypes.c_uint32), _ptr(sc, ctypes.c_double), n_seg, _ptr(so, ctypes.c_int64),
                        _ptr(sums, ctypes.c_double))
     return sc, sums
+
+
+def truncate_rows(logits, top_k: int = 0, top_p: float = 1.0, T: float = 1.0):
+    """Top-k then top-p truncation as masking: (logits with removed tokens set to -inf, margin)."""
+    l = _c(logits, np.float32)
+    n, V = l.shape
+    out = np.zeros((n, V), np.float32)
+    mg = np.zeros(n, np.float64)
+    lib().orc_truncate_rows(_ptr(l, ctypes.c_float), n, V, V, float(T), int(top_k), float(top_p),
+                            _ptr(out, ctypes.c_float), _ptr(mg, ctypes.c_double))
+    return out, mg

@@ -40,6 +40,12 @@
  *   orc_wm_score       A_t = -ln(1 - r_t(w_t)) with pivot r_t = u of the
  *                      emitted token (Eq. 2; App. D.1 "Gumbel watermark";
  *                      detector algorithm, App. E).
+ *   orc_truncate_rows  the logit processing of the experiments (Sec. 6 setup:
+ *                      top-k = 50, top-p = 1; truncation leaves a support of at
+ *                      most k tokens, Sec. 4.2): tokens outside the top-k /
+ *                      top-p set get logit -inf, i.e. P = 0 and E/P = +inf, so
+ *                      the race over the masked row is the race of the
+ *                      truncated distribution.
  */
 #include <math.h>
 #include <stdint.h>
@@ -334,6 +340,82 @@ void orc_wm_score(int64_t n, const int32_t* tokens, const uint64_t* key, const u
         double S = 0.0;
         for (int64_t t = seg_off[g]; t < seg_off[g + 1]; ++t) S += score[t];
         sums[g] = S;
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* truncation before the race                                          */
+/* ------------------------------------------------------------------ */
+
+static int orc_double_desc(const void* a, const void* b)
+{
+    double x = *(const double*)a, y = *(const double*)b;
+    return x > y ? -1 : (x < y ? 1 : 0);
+}
+
+static int orc_double_asc(const void* a, const void* b)
+{
+    return -orc_double_desc(a, b);
+}
+
+/* out[r*V + i] = l[i] if token i survives the truncation, -inf otherwise.
+ *   top-k (top_k > 0): l_(k) is the k-th largest usable logit counting
+ *     duplicates (usable: neither NaN nor -inf); a token is kept iff its logit
+ *     is >= l_(k), so every token tied with l_(k) is kept.  With fewer than k
+ *     usable tokens all usable tokens are kept.  top_k <= 0: all usable tokens.
+ *   top-p (top_p < 1), on the top-k survivors with probabilities
+ *     softmax(l / T) over them: walk the survivors in ascending logit order,
+ *     adding each token's probability e_j / Z (e_j = exp((l_j - max l) / T),
+ *     Z = the sum of the e_j taken in the same ascending order) to a running
+ *     sum.  Tokens of equal logit form one group; a group is removed iff the
+ *     running sum at its last token is <= 1 - top_p.  The group of the largest
+ *     logit is always kept.  (For distinct logits this is the usual nucleus
+ *     rule; a group is never split.)
+ *   margin[r] (nullable): the smallest |running sum - (1 - top_p)| over the
+ *     group ends (+inf without top-p), for flip accounting. */
+void orc_truncate_rows(const float* logits, int64_t n_rows, int64_t V, int64_t stride, double T,
+                       int32_t top_k, double top_p, float* out, double* margin)
+{
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t r = 0; r < n_rows; ++r) {
+        const float* l = logits + r * stride;
+        float* o = out + r * V;
+        double* v = (double*)malloc(sizeof(double) * (size_t)(V > 0 ? V : 1));
+        int64_t n = 0;
+        for (int64_t i = 0; i < V; ++i)
+            if (!isnan(l[i]) && l[i] != -INFINITY) v[n++] = (double)l[i];
+        double cut = -INFINITY;
+        if (top_k > 0 && n >= top_k) {
+            qsort(v, (size_t)n, sizeof(double), orc_double_desc);
+            cut = v[top_k - 1];
+        }
+        double mg = INFINITY;
+        if (top_p < 1.0 && n > 0) {
+            /* survivors of top-k, ascending */
+            int64_t m = 0;
+            for (int64_t i = 0; i < V; ++i)
+                if (!isnan(l[i]) && l[i] != -INFINITY && (double)l[i] >= cut) v[m++] = (double)l[i];
+            qsort(v, (size_t)m, sizeof(double), orc_double_asc);
+            double top = v[m - 1], Z = 0.0;
+            for (int64_t j = 0; j < m; ++j) Z += exp((v[j] - top) / T);
+            double run = 0.0, keep_from = top;
+            for (int64_t j = 0; j < m; ++j) {
+                run += exp((v[j] - top) / T) / Z;
+                int group_end = j + 1 == m || v[j + 1] != v[j];
+                if (!group_end) continue;
+                double d = fabs(run - (1.0 - top_p));
+                if (d < mg) mg = d;
+                if (v[j] == top) break;
+                if (run <= 1.0 - top_p) keep_from = j + 1 < m ? v[j + 1] : top;
+                else { keep_from = v[j]; break; }
+            }
+            /* the kept survivors are those with logit >= keep_from */
+            if (keep_from > cut) cut = keep_from;
+        }
+        for (int64_t i = 0; i < V; ++i)
+            o[i] = (!isnan(l[i]) && l[i] != -INFINITY && (double)l[i] >= cut) ? l[i] : -INFINITY;
+        if (margin) margin[r] = mg;
+        free(v);
     }
 }
 
