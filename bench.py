@@ -39,7 +39,7 @@ def kernel_source_digest() -> str:
     import hashlib
     h = hashlib.sha1()
     csrc = os.path.join(ROOT, "paper_2609_21858_gb300", "csrc")
-    for name in ("pps_race.cu", "pps_device.cuh", "pps_internal.h"):
+    for name in ("pps_race.cu", "pps_device.cuh", "pps_internal.h", "pps_trunc.cuh"):
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(name.encode() + b"\0" + f.read())
     return h.hexdigest()
@@ -166,7 +166,7 @@ def max_over_ranks(x: float, world: int) -> float:
     return float(t.item())
 
 
-def oracle_sample(wl, n_draft_rows: int, n_target_rows: int, seed: int = 0):
+def oracle_sample(wl, n_draft_rows: int, n_target_rows: int, seed: int = 0, top_k: int = 0, top_p: float = 1.0):
     """Host copies of a bounded sample of the workload's rows and a timer over them."""
     import oracle
     from paper_2609_21858_gb300 import synth
@@ -185,8 +185,12 @@ def oracle_sample(wl, n_draft_rows: int, n_target_rows: int, seed: int = 0):
 
     def run():
         t0 = time.perf_counter()
-        oracle.draft_rows(q, *ids_d, t.K, row_k=rk)
-        oracle.target_rows(p, *ids_n)
+        qq, pp = q, p
+        if top_k > 0:
+            qq, _ = oracle.truncate_rows(q, top_k, top_p)
+            pp, _ = oracle.truncate_rows(p, top_k, top_p)
+        oracle.draft_rows(qq, *ids_d, t.K, row_k=rk)
+        oracle.target_rows(pp, *ids_n)
         return time.perf_counter() - t0
 
     return run, len(dr), len(nr), cores
@@ -202,6 +206,8 @@ def main():
     ap.add_argument("--n-seq", type=int, default=None, help="override the number of sequences (smaller profiling cases)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--n-tokens", type=int, default=10_000_000, help="detector workload size")
+    ap.add_argument("--top-k", type=int, default=0, help="truncate every row to its top-k set before the race")
+    ap.add_argument("--top-p", type=float, default=1.0, help="then to its top-p set (with --top-k)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
@@ -244,11 +250,12 @@ def main():
     stream = torch.cuda.current_stream(dev)
 
     def draft(q):
-        pps.draft_list(q, dk, dc, dp, t.K, row_k=row_k, ws=ws_d, status=status, out=dout, stream=stream)
+        pps.draft_list(q, dk, dc, dp, t.K, row_k=row_k, ws=ws_d, status=status, out=dout, stream=stream,
+                       top_k=args.top_k, top_p=args.top_p)
 
     def verify(p):
         pps.verify_tree(p, nk, nc, np_, t.gamma, seq_off, ndr, dout["tok"], dout["ndist"], child, ws=ws_v,
-                        status=status, out=vout, stream=stream)
+                        status=status, out=vout, stream=stream, top_k=args.top_k, top_p=args.top_p)
 
     def step(q, p, ev=None):
         if ev is not None:
@@ -316,7 +323,7 @@ def main():
     clk = (clocks.get("sm_mhz") or 2070.0) * 1e6
     mul_peak = sms * WIDE_MULS_PER_SM_CLK * clk / 1e12
     mul_ach = tok_verify * WIDE_MULS_PER_TOKEN / (t_verify / 1e3) / 1e12
-    traffic = _traffic("verify")
+    traffic = _traffic("verify") if args.top_k == 0 else None
     philox_tok_s = philox_only_rate(dev) if rank == 0 else None
     emitted = float(vout["n_emitted"].sum().item())
 
@@ -377,7 +384,7 @@ def main():
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        run, nd, nn, cores = oracle_sample(wl, 8, 8)
+        run, nd, nn, cores = oracle_sample(wl, 8, 8, top_k=args.top_k, top_p=args.top_p)
         dt = run()
         reps = max(1, int(args.cpu_seconds / max(dt, 1e-3)))
         tot = sum(run() for _ in range(reps))
@@ -385,6 +392,7 @@ def main():
                "sample": f"{nd} draft + {nn} target rows of the same workload, x{reps} repetitions, "
                          f"{tot:.1f} s on {cores} threads"}
 
+    trunc = f", top-k {args.top_k}, top-p {args.top_p}" if args.top_k > 0 else ""
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": args.steps,
@@ -392,7 +400,7 @@ def main():
             "vs_baseline": None, "dtype": "bf16" if wl.dtype == torch.bfloat16 else "f32",
             "data": "synthetic (seeded Zipf-rank logits; no model, no dataset)",
             "config": {"workload": f"{args.workload}: B={t.n_seq}, V={wl.vocab}, K={t.K}, gamma={t.gamma}, "
-                                   f"{t.n_nodes} target rows + {t.n_draft} draft rows per step",
+                                   f"{t.n_nodes} target rows + {t.n_draft} draft rows per step{trunc}",
                        "rows_per_step": rows_per_step, "l2": l2_note,
                        "parallelism": f"replicas x{world}"},
             "gb_per_s": ach_all, "emitted_tokens_per_s": emitted * world / (ms_step / 1e3),
@@ -411,6 +419,9 @@ def main():
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": 2 * args.steps, "clocks": clocks,
             "mean_accept_len": float(vout["accept_len"].float().mean().item()),
         }
+        if args.top_k > 0:
+            # truncated race: the scan keys no token outside the top-k set, so HBM bounds it
+            line["roofline"] = dict(line["roofline_hbm"], kernel="trunc_kernel (pps_verify_tree_trunc)", ms=t_verify)
         print(json.dumps(line))
 
 

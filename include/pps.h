@@ -157,6 +157,44 @@ pps_status pps_verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_node
                            double* out_score_sum, uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream);
 
 /*
+ * Truncated calls -- pps_draft_list / pps_verify_tree with the logit
+ * processing of the experiments (top-k = 50, top-p = 1 in Sec. 6) applied to
+ * each row before the race; a truncated distribution has a support of at
+ * most k tokens (Sec. 4.2).  Tokens outside the kept set S get P = 0
+ * (E/P = +inf), so the race, lists, walk and scores are those of the
+ * renormalised truncated distributions of P and Q.
+ *
+ * top_k        1 <= top_k <= PPS_MAX_TOP_K: S holds every token whose logit is
+ *              >= the top_k-th largest usable logit (ties of it included;
+ *              NaN and -inf logits never; all usable tokens if fewer than top_k)
+ * top_p        0 < top_p <= 1: then, with probabilities softmax(logit / T) over
+ *              the top-k set, whole groups of equal logits are removed from the
+ *              bottom while the running mass, summed token by token in
+ *              ascending logit order, is <= 1 - top_p; the largest group stays.
+ *              1 = no top-p.
+ * Every other argument, output and the workspace size are those of
+ * pps_draft_list / pps_verify_tree.  PPS_ERR_INVALID_ARG for top_k or top_p
+ * out of range.  A row whose top-k tie group does not fit the 64-entry list
+ * is still exact: it is finished with a second pass over its logits.
+ */
+#define PPS_MAX_TOP_K 64
+
+pps_status pps_draft_list_trunc(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab,
+                                int64_t row_stride, pps_row_ids ids, float temperature, int32_t top_k, float top_p,
+                                int32_t K, const int32_t* row_k, pps_draft_mode mode, int32_t* out_tok,
+                                float* out_key, int32_t* out_mult, int32_t* out_ndistinct, int32_t* out_samples,
+                                uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream);
+
+pps_status pps_verify_tree_trunc(const void* p_logits, pps_dtype dtype, int64_t n_nodes, int64_t vocab,
+                                 int64_t row_stride, pps_row_ids ids, float temperature, int32_t top_k, float top_p,
+                                 int32_t n_seq, int32_t gamma, const int32_t* seq_off, const int32_t* node_draft_row,
+                                 int64_t n_draft, const int32_t* draft_tok, const int32_t* draft_ndistinct, int32_t K,
+                                 const int32_t* child_node, int32_t* out_winner, uint32_t* out_word,
+                                 int32_t* out_accept_len, int32_t* out_n_emitted, int32_t* out_emitted,
+                                 float* out_score, double* out_score_sum, uint32_t* status, void* ws,
+                                 size_t ws_bytes, pps_stream_t stream);
+
+/*
  * pps_wm_score -- detector pass (detector algorithm of App. E; Eq. 2):
  * regenerate the first-arrival word of every observed token under its
  * context's identity and score it, A_t = -ln(1 - u_t).

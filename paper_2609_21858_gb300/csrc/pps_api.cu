@@ -14,7 +14,7 @@ namespace pps {
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 size_t workspace_bytes(int64_t n_rows, int32_t n_seq) {
-    return align256(sizeof(Partial) * (size_t)(n_rows + (int64_t)kGridMax)) + align256(sizeof(uint32_t) * (size_t)n_rows) +
+    return align256(kSlotBytes * (size_t)(n_rows + (int64_t)kGridMax)) + align256(sizeof(uint32_t) * (size_t)n_rows) +
            align256(sizeof(uint32_t) * (size_t)(n_seq > 0 ? n_seq : 0));
 }
 
@@ -22,7 +22,7 @@ void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials
                      uint32_t** seq_cnt) {
     char* p = static_cast<char*>(ws);
     *partials = reinterpret_cast<Partial*>(p);
-    p += align256(sizeof(Partial) * (size_t)(n_rows + (int64_t)kGridMax));
+    p += align256(kSlotBytes * (size_t)(n_rows + (int64_t)kGridMax));
     *row_cnt = reinterpret_cast<uint32_t*>(p);
     p += align256(sizeof(uint32_t) * (size_t)n_rows);
     *seq_cnt = reinterpret_cast<uint32_t*>(p);
@@ -128,10 +128,18 @@ pps_status pps_workspace_clear(void* ws, size_t ws_bytes, pps_stream_t stream) {
     return cudaMemsetAsync(ws, 0, ws_bytes, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
 }
 
-pps_status pps_draft_list(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t row_stride,
-                          pps_row_ids ids, float temperature, int32_t K, const int32_t* row_k, pps_draft_mode mode,
-                          int32_t* out_tok, float* out_key, int32_t* out_mult, int32_t* out_ndistinct,
-                          int32_t* out_samples, uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream) {
+// top_k = 0: no truncation (the full-vocabulary race)
+static pps_status check_trunc(int32_t top_k, float top_p) {
+    if (top_k < 1 || top_k > PPS_MAX_TOP_K) return PPS_ERR_INVALID_ARG;
+    if (!(top_p > 0.0f) || !(top_p <= 1.0f)) return PPS_ERR_INVALID_ARG;
+    return PPS_OK;
+}
+
+static pps_status draft_list(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t row_stride,
+                             pps_row_ids ids, float temperature, int32_t top_k, float top_p, int32_t K,
+                             const int32_t* row_k, pps_draft_mode mode, int32_t* out_tok, float* out_key,
+                             int32_t* out_mult, int32_t* out_ndistinct, int32_t* out_samples, uint32_t* status,
+                             void* ws, size_t ws_bytes, pps_stream_t stream) {
     pps_status st = check_rows(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature);
     if (st != PPS_OK) return st;
     if (mode != PPS_DRAFT_DISTINCT && mode != PPS_DRAFT_IID) return PPS_ERR_UNSUPPORTED;
@@ -150,18 +158,49 @@ pps_status pps_draft_list(const void* q_logits, pps_dtype dtype, int64_t n_rows,
     a.out_samples = out_samples;
     a.status = status;
     workspace_carve(ws, n_rows, 0, &a.partials, &a.row_cnt, &a.seq_cnt);
+    a.tpartials = reinterpret_cast<TruncPartial*>(a.partials);
+    a.top_k = top_k;
+    a.top_p = top_p;
     const int dt = dtype == PPS_BF16 ? 1 : 0;
     const bool vec = vec_ok(q_logits, dtype, row_stride);
-    a.G = race_grid(a.total, dt, false, vec);
-    return launch_race(a, dt, false, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+    cudaError_t e;
+    if (top_k > 0) {
+        a.G = trunc_grid(a.total, dt, false, vec);
+        e = launch_trunc(a, dt, false, vec, (cudaStream_t)stream);
+    } else {
+        a.G = race_grid(a.total, dt, false, vec);
+        e = launch_race(a, dt, false, vec, (cudaStream_t)stream);
+    }
+    return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
 }
 
-pps_status pps_verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_nodes, int64_t vocab, int64_t row_stride,
-                           pps_row_ids ids, float temperature, int32_t n_seq, int32_t gamma, const int32_t* seq_off,
-                           const int32_t* node_draft_row, int64_t n_draft, const int32_t* draft_tok,
-                           const int32_t* draft_ndistinct, int32_t K, const int32_t* child_node, int32_t* out_winner, uint32_t* out_word,
-                           int32_t* out_accept_len, int32_t* out_n_emitted, int32_t* out_emitted, float* out_score,
-                           double* out_score_sum, uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream) {
+pps_status pps_draft_list(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t row_stride,
+                          pps_row_ids ids, float temperature, int32_t K, const int32_t* row_k, pps_draft_mode mode,
+                          int32_t* out_tok, float* out_key, int32_t* out_mult, int32_t* out_ndistinct,
+                          int32_t* out_samples, uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream) {
+    return draft_list(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature, 0, 1.0f, K, row_k, mode, out_tok,
+                      out_key, out_mult, out_ndistinct, out_samples, status, ws, ws_bytes, stream);
+}
+
+pps_status pps_draft_list_trunc(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab,
+                                int64_t row_stride, pps_row_ids ids, float temperature, int32_t top_k, float top_p,
+                                int32_t K, const int32_t* row_k, pps_draft_mode mode, int32_t* out_tok,
+                                float* out_key, int32_t* out_mult, int32_t* out_ndistinct, int32_t* out_samples,
+                                uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream) {
+    pps_status st = check_trunc(top_k, top_p);
+    if (st != PPS_OK) return st;
+    return draft_list(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature, top_k, top_p, K, row_k, mode,
+                      out_tok, out_key, out_mult, out_ndistinct, out_samples, status, ws, ws_bytes, stream);
+}
+
+static pps_status verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_nodes, int64_t vocab,
+                              int64_t row_stride, pps_row_ids ids, float temperature, int32_t top_k, float top_p,
+                              int32_t n_seq, int32_t gamma, const int32_t* seq_off, const int32_t* node_draft_row,
+                              int64_t n_draft, const int32_t* draft_tok, const int32_t* draft_ndistinct, int32_t K,
+                              const int32_t* child_node, int32_t* out_winner, uint32_t* out_word,
+                              int32_t* out_accept_len, int32_t* out_n_emitted, int32_t* out_emitted, float* out_score,
+                              double* out_score_sum, uint32_t* status, void* ws, size_t ws_bytes,
+                              pps_stream_t stream) {
     pps_status st = check_rows(p_logits, dtype, n_nodes, vocab, row_stride, ids, temperature);
     if (st != PPS_OK) return st;
     if (n_seq < 0 || gamma < 1 || gamma > 64 || K < 1 || K > PPS_MAX_K || n_draft < 0) return PPS_ERR_INVALID_ARG;
@@ -191,10 +230,49 @@ pps_status pps_verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_node
     a.out_ss = out_score_sum;
     a.status = status;
     workspace_carve(ws, n_nodes, n_seq, &a.partials, &a.row_cnt, &a.seq_cnt);
+    a.tpartials = reinterpret_cast<TruncPartial*>(a.partials);
+    a.top_k = top_k;
+    a.top_p = top_p;
     const int dt = dtype == PPS_BF16 ? 1 : 0;
     const bool vec = vec_ok(p_logits, dtype, row_stride);
-    a.G = race_grid(a.total, dt, true, vec);
-    return launch_race(a, dt, true, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+    cudaError_t e;
+    if (top_k > 0) {
+        a.G = trunc_grid(a.total, dt, true, vec);
+        e = launch_trunc(a, dt, true, vec, (cudaStream_t)stream);
+    } else {
+        a.G = race_grid(a.total, dt, true, vec);
+        e = launch_race(a, dt, true, vec, (cudaStream_t)stream);
+    }
+    return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_nodes, int64_t vocab, int64_t row_stride,
+                           pps_row_ids ids, float temperature, int32_t n_seq, int32_t gamma, const int32_t* seq_off,
+                           const int32_t* node_draft_row, int64_t n_draft, const int32_t* draft_tok,
+                           const int32_t* draft_ndistinct, int32_t K, const int32_t* child_node, int32_t* out_winner,
+                           uint32_t* out_word, int32_t* out_accept_len, int32_t* out_n_emitted, int32_t* out_emitted,
+                           float* out_score, double* out_score_sum, uint32_t* status, void* ws, size_t ws_bytes,
+                           pps_stream_t stream) {
+    return verify_tree(p_logits, dtype, n_nodes, vocab, row_stride, ids, temperature, 0, 1.0f, n_seq, gamma, seq_off,
+                       node_draft_row, n_draft, draft_tok, draft_ndistinct, K, child_node, out_winner, out_word,
+                       out_accept_len, out_n_emitted, out_emitted, out_score, out_score_sum, status, ws, ws_bytes,
+                       stream);
+}
+
+pps_status pps_verify_tree_trunc(const void* p_logits, pps_dtype dtype, int64_t n_nodes, int64_t vocab,
+                                 int64_t row_stride, pps_row_ids ids, float temperature, int32_t top_k, float top_p,
+                                 int32_t n_seq, int32_t gamma, const int32_t* seq_off, const int32_t* node_draft_row,
+                                 int64_t n_draft, const int32_t* draft_tok, const int32_t* draft_ndistinct, int32_t K,
+                                 const int32_t* child_node, int32_t* out_winner, uint32_t* out_word,
+                                 int32_t* out_accept_len, int32_t* out_n_emitted, int32_t* out_emitted,
+                                 float* out_score, double* out_score_sum, uint32_t* status, void* ws,
+                                 size_t ws_bytes, pps_stream_t stream) {
+    pps_status st = check_trunc(top_k, top_p);
+    if (st != PPS_OK) return st;
+    return verify_tree(p_logits, dtype, n_nodes, vocab, row_stride, ids, temperature, top_k, top_p, n_seq, gamma,
+                       seq_off, node_draft_row, n_draft, draft_tok, draft_ndistinct, K, child_node, out_winner,
+                       out_word, out_accept_len, out_n_emitted, out_emitted, out_score, out_score_sum, status, ws,
+                       ws_bytes, stream);
 }
 
 pps_status pps_draft_list_noalloc(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab,

@@ -19,6 +19,18 @@ struct alignas(16) Partial {
     int32_t pad[2];
 };
 
+// one partial top-k list of a row segment for the truncated race (sorted by
+// logit descending, then token ascending; empty entries (-inf, INT_MAX))
+constexpr int kTopMax = 64;  // largest top-k of the truncated race
+struct alignas(16) TruncPartial {
+    float v[kTopMax];
+    int32_t idx[kTopMax];
+    float dropmax;  // largest logit evicted from the segment's list (-inf: none)
+    int32_t pad[3];
+};
+// workspace slot: room for either kind of partial list
+constexpr size_t kSlotBytes = sizeof(TruncPartial) > sizeof(Partial) ? sizeof(TruncPartial) : sizeof(Partial);
+
 struct RaceArgs {
     const void* logits;
     int64_t n_rows, V, stride;
@@ -57,8 +69,12 @@ struct RaceArgs {
     int64_t nv;     // 16-byte vectors per row (last one may be partial)
     int64_t total;  // n_rows * nv
     int G;
+    // truncation (truncated race only): top-k in [1, kTopMax], top-p in (0, 1]
+    int top_k;
+    float top_p;
     // workspace
     Partial* partials;   // [n_rows + kGridMax]: slot (warp + row)
+    TruncPartial* tpartials;  // the same slots, for the truncated race
     uint32_t* row_cnt;   // [n_rows]
     uint32_t* seq_cnt;   // [n_seq]
 };
@@ -70,6 +86,8 @@ void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials
 // launchers (pps_race.cu)
 cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
 int race_grid(int64_t total, int dtype, bool verify, bool vec);
+cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
+int trunc_grid(int64_t total, int dtype, bool verify, bool vec);
 
 // launchers (pps_misc.cu)
 cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,

@@ -363,9 +363,10 @@ __device__ __noinline__ SlowState flush_queue(SlowState st, const uint32_t* q, i
 
 // Scalar-load path, one vector per lane at a time: the last partial
 // iteration of a segment, the ragged vector of a row, and unaligned rows.
+// Tokens with a logit below `floor` take no part (-inf: none excluded).
 template <int DT>
 __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64_t V, int64_t base, int64_t v1,
-                                            float c, uint64_t key, uint64_t ctx, uint32_t pos) {
+                                            float c, uint64_t key, uint64_t ctx, uint32_t pos, float floor) {
     constexpr int VW = DT == 1 ? 8 : 4;
     const int lane = threadIdx.x & 31;
     RowPhilox rp;
@@ -383,9 +384,12 @@ __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64
         // the vector's blocks: bf16 2 (counters 2v, 2v+1), fp32 1 (counter v)
 #pragma unroll
         for (int h = 0; h < (DT == 1 ? 2 : 1); ++h) {
-            const unsigned vh = (valid >> (4 * h)) & 0xfu;
+            unsigned vh = (valid >> (4 * h)) & 0xfu;
             float l[4];
             block_logits<DT>(d, h, l);
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                if (l[e] < floor) vh &= ~(1u << e);
             const uint32_t cb = DT == 1 ? (uint32_t)(2 * v + h) : (uint32_t)v;
             // any token of the block over the cut?
             bool pass = false;
@@ -578,7 +582,7 @@ __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int
         }
         base = v0 + n_it * STEP;
     }
-    if (base < v1) st = tail_loop<DT>(st, row, V, base, v1, c, key, ctx, pos);
+    if (base < v1) st = tail_loop<DT>(st, row, V, base, v1, c, key, ctx, pos, -kInf);
     L = st.L;
 }
 
@@ -592,41 +596,13 @@ __device__ __forceinline__ float logit_at(const RaceArgs& a, int64_t r, int64_t 
 
 __device__ void walk_sequence(const RaceArgs& a, int s);
 
-// Warp 0 finishes row r from its complete list (lk, li) and the drop bound.
+// Outputs of row r from its sorted entries: lane m holds the m-th smallest
+// (key, token) of the row's list (dk fp64 when exact, sk fp32), nvalid of them
+// usable.  Verify rows: the winner and its word.  Draft rows: the list, its
+// multiplicities and labels (IID: the kr smallest multi-arrival scores).
 template <int DT, bool VERIFY>
-__device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk, int li, float theta_drop, int kr,
-                                          int kp, int lane) {
-    const int nvalid = __popc(__ballot_sync(FULL, lane < kp && lk < kInf));
-    const float tau = nvalid >= kr ? __shfl_sync(FULL, lk, kr - 1) : kInf;
-    bool complete;
-    if (nvalid < kr)
-        complete = theta_drop == kInf;
-    else if (tau == -kInf)
-        complete = true;
-    else
-        complete = theta_drop == kInf || theta_drop > tau + key_err_bound(tau) + key_err_bound(theta_drop);
-    if (lane == 0 && a.status) {
-        unsigned f = complete ? 0u : PPS_FLAG_GUARD;
-        if (nvalid >= kr && tau > -kInf && fabsf(tau) > 65536.0f) f |= PPS_FLAG_LOGIT_RANGE;
-        if (f) atomicOr(a.status, f);
-    }
-    // near ties among the first min(nvalid, kr+1) entries
-    float nk = __shfl_down_sync(FULL, lk, 1);
-    int lim = min(nvalid, kr + 1);
-    bool close = lane + 1 < lim && !(nk - lk > key_err_bound(lk) + key_err_bound(nk));
-    const bool need_exact = (__ballot_sync(FULL, close) != 0) || (!VERIFY && a.iid);
-    const uint64_t key = a.key[r], ctx = a.ctx[r];
-    const uint32_t pos = a.pos[r];
-    double dk = (double)INFINITY;
-    float sk = key_to_s(lk);
-    if (need_exact) {
-        if (lane < nvalid) {
-            uint32_t w = word_of(key, ctx, pos, li, 1);
-            dk = key64(w, logit_at<DT>(a, r, li), a.T);
-        }
-        warp_sort_d(dk, li, lane);
-        sk = (float)dk;
-    }
+__device__ __forceinline__ void emit_row(const RaceArgs& a, int64_t r, double dk, float sk, int li, int nvalid, int kr,
+                                         int lane, uint64_t key, uint64_t ctx, uint32_t pos) {
     if (VERIFY) {
         int win = __shfl_sync(FULL, li, 0);
         if (nvalid == 0) win = -1;
@@ -693,6 +669,44 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
         if (a.out_samples) a.out_samples[o] = lane < kr ? sample : -1;
     }
     if (lane == 0) a.out_nd[r] = nd;
+}
+
+// Warp 0 finishes row r from its complete list (lk, li) and the drop bound.
+template <int DT, bool VERIFY>
+__device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk, int li, float theta_drop, int kr,
+                                          int kp, int lane) {
+    const int nvalid = __popc(__ballot_sync(FULL, lane < kp && lk < kInf));
+    const float tau = nvalid >= kr ? __shfl_sync(FULL, lk, kr - 1) : kInf;
+    bool complete;
+    if (nvalid < kr)
+        complete = theta_drop == kInf;
+    else if (tau == -kInf)
+        complete = true;
+    else
+        complete = theta_drop == kInf || theta_drop > tau + key_err_bound(tau) + key_err_bound(theta_drop);
+    if (lane == 0 && a.status) {
+        unsigned f = complete ? 0u : PPS_FLAG_GUARD;
+        if (nvalid >= kr && tau > -kInf && fabsf(tau) > 65536.0f) f |= PPS_FLAG_LOGIT_RANGE;
+        if (f) atomicOr(a.status, f);
+    }
+    // near ties among the first min(nvalid, kr+1) entries
+    float nk = __shfl_down_sync(FULL, lk, 1);
+    int lim = min(nvalid, kr + 1);
+    bool close = lane + 1 < lim && !(nk - lk > key_err_bound(lk) + key_err_bound(nk));
+    const bool need_exact = (__ballot_sync(FULL, close) != 0) || (!VERIFY && a.iid);
+    const uint64_t key = a.key[r], ctx = a.ctx[r];
+    const uint32_t pos = a.pos[r];
+    double dk = (double)INFINITY;
+    float sk = key_to_s(lk);
+    if (need_exact) {
+        if (lane < nvalid) {
+            uint32_t w = word_of(key, ctx, pos, li, 1);
+            dk = key64(w, logit_at<DT>(a, r, li), a.T);
+        }
+        warp_sort_d(dk, li, lane);
+        sk = (float)dk;
+    }
+    emit_row<DT, VERIFY>(a, r, dk, sk, li, nvalid, kr, lane, key, ctx, pos);
 }
 
 __device__ __forceinline__ int64_t warp_of(int64_t g, int64_t total, int64_t NW) {
@@ -773,6 +787,23 @@ __device__ __noinline__ void walk_sequence(const RaceArgs& a, int s) {
 // End of a row segment: publish the warp's list, or merge the row's lists if
 // this warp is the last to finish the row, then finish the row (and the walk
 // of its sequence when it is the sequence's last node).  Out of line.
+// Sequence ticket after node row r is final: the warp that finishes a
+// sequence's last node walks it.
+__device__ __noinline__ void sequence_ticket(const RaceArgs& a, int64_t r, int lane) {
+    __threadfence();
+    if (lane == 0) {
+        int s = seq_of_node(a.seq_off, a.n_seq, r);
+        int nn = __ldg(a.seq_off + s + 1) - __ldg(a.seq_off + s);
+        unsigned t = atomicAdd(a.seq_cnt + s, 1u);
+        if (t == (unsigned)(nn - 1)) {
+            a.seq_cnt[s] = 0u;
+            __threadfence();
+            walk_sequence(a, s);
+        }
+    }
+    __syncwarp();
+}
+
 template <int DT, bool VERIFY>
 __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_t gw, int64_t NW, int64_t v0,
                                         int64_t v1, const WarpList L, int kr, int kp) {
@@ -814,21 +845,7 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
     }
     if (final_here) {
         finalize_row<DT, VERIFY>(a, r, lk, li, theta_drop, kr, kp, lane);
-        if constexpr (VERIFY) {
-            // sequence ticket: the warp that finishes a sequence's last node walks it
-            __threadfence();
-            if (lane == 0) {
-                int s = seq_of_node(a.seq_off, a.n_seq, r);
-                int nn = __ldg(a.seq_off + s + 1) - __ldg(a.seq_off + s);
-                unsigned t = atomicAdd(a.seq_cnt + s, 1u);
-                if (t == (unsigned)(nn - 1)) {
-                    a.seq_cnt[s] = 0u;
-                    __threadfence();
-                    walk_sequence(a, s);
-                }
-            }
-            __syncwarp();
-        }
+        if constexpr (VERIFY) sequence_ticket(a, r, lane);
     }
 }
 
@@ -870,6 +887,8 @@ __global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(con
     }
 }
 
+
+#include "pps_trunc.cuh"
 
 int race_grid(int64_t total, int dtype, bool verify, bool vec) {
     static int sms = 0, occ[2][2][2] = {};
@@ -916,6 +935,56 @@ cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cud
         } else {
             if (vec) race_kernel<0, false, true><<<grid, block, 0, stream>>>(a);
             else race_kernel<0, false, false><<<grid, block, 0, stream>>>(a);
+        }
+    }
+    return cudaGetLastError();
+}
+
+int trunc_grid(int64_t total, int dtype, bool verify, bool vec) {
+    static int sms = 0, occ[2][2][2] = {};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (sms == 0) {
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (sms <= 0) sms = 1;
+    }
+    int& o = occ[dtype][verify][vec];
+    if (o == 0) {
+        const void* fn = nullptr;
+        if (dtype == 1)
+            fn = verify ? (vec ? (const void*)trunc_kernel<1, true, true> : (const void*)trunc_kernel<1, true, false>)
+                        : (vec ? (const void*)trunc_kernel<1, false, true> : (const void*)trunc_kernel<1, false, false>);
+        else
+            fn = verify ? (vec ? (const void*)trunc_kernel<0, true, true> : (const void*)trunc_kernel<0, true, false>)
+                        : (vec ? (const void*)trunc_kernel<0, false, true> : (const void*)trunc_kernel<0, false, false>);
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, kThreads, 0);
+        if (o <= 0) o = 1;
+    }
+    int64_t g = (int64_t)sms * o;
+    int64_t by_size = (total + kMinVecsPerWarp - 1) / kMinVecsPerWarp;
+    if (by_size < g) g = by_size;
+    if (g > kGridMax) g = kGridMax;
+    if (g < 1) g = 1;
+    return (int)g;
+}
+
+cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream) {
+    dim3 grid(a.G), block(kThreads);
+    if (dtype == 1) {
+        if (verify) {
+            if (vec) trunc_kernel<1, true, true><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<1, true, false><<<grid, block, 0, stream>>>(a);
+        } else {
+            if (vec) trunc_kernel<1, false, true><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<1, false, false><<<grid, block, 0, stream>>>(a);
+        }
+    } else {
+        if (verify) {
+            if (vec) trunc_kernel<0, true, true><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<0, true, false><<<grid, block, 0, stream>>>(a);
+        } else {
+            if (vec) trunc_kernel<0, false, true><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<0, false, false><<<grid, block, 0, stream>>>(a);
         }
     }
     return cudaGetLastError();

@@ -20,6 +20,7 @@ F32, BF16 = 0, 1
 DISTINCT, IID = 0, 1
 FLAG_GUARD, FLAG_LOGIT_RANGE = 1, 2
 MAX_K = 32
+MAX_TOP_K = 64
 
 _lock = threading.Lock()
 _lib = None
@@ -59,6 +60,12 @@ def lib():
             L.pps_verify_tree.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, i32, i32, vp, vp, i64, vp,
                                           vp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
             L.pps_verify_tree.restype = ctypes.c_int
+            L.pps_draft_list_trunc.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, i32, f32, i32, vp,
+                                               ctypes.c_int, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+            L.pps_draft_list_trunc.restype = ctypes.c_int
+            L.pps_verify_tree_trunc.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, i32, f32, i32, i32, vp,
+                                                vp, i64, vp, vp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+            L.pps_verify_tree_trunc.restype = ctypes.c_int
             L.pps_draft_list_noalloc.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, i32, vp, ctypes.c_int,
                                                  vp, vp, vp, vp, vp, vp, vp]
             L.pps_draft_list_noalloc.restype = ctypes.c_int
@@ -132,8 +139,9 @@ def workspace_clear(ws: torch.Tensor, stream=None):
 
 
 def draft_list(q_logits, key, ctx, pos, K: int, row_k=None, mode: int = DISTINCT, temperature: float = 1.0,
-               ws=None, status=None, out=None, keys: bool = True, samples: bool = True, stream=None):
-    """pps_draft_list.  Returns dict(tok, key, mult, ndist, samples) of CUDA tensors."""
+               ws=None, status=None, out=None, keys: bool = True, samples: bool = True, stream=None,
+               top_k: int = 0, top_p: float = 1.0):
+    """pps_draft_list (pps_draft_list_trunc when top_k > 0).  Returns dict(tok, key, mult, ndist, samples)."""
     n, V, stride = _rows(q_logits)
     dev = q_logits.device
     if out is None:
@@ -146,6 +154,14 @@ def draft_list(q_logits, key, ctx, pos, K: int, row_k=None, mode: int = DISTINCT
         ws = workspace(n, 0, dev)
     if row_k is not None and (row_k.dtype != torch.int32 or not row_k.is_cuda):
         raise TypeError("row_k must be a CUDA int32 tensor")
+    if top_k > 0:
+        code = lib().pps_draft_list_trunc(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
+                                          float(temperature), int(top_k), float(top_p), int(K), _ptr(row_k),
+                                          int(mode), _ptr(out["tok"]), _ptr(out.get("key")), _ptr(out["mult"]),
+                                          _ptr(out["ndist"]), _ptr(out.get("samples")), _ptr(status), _ptr(ws),
+                                          ws.numel(), _stream(stream))
+        _check("pps_draft_list_trunc", code)
+        return out
     code = lib().pps_draft_list(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
                                 float(temperature), int(K), _ptr(row_k), int(mode), _ptr(out["tok"]),
                                 _ptr(out.get("key")), _ptr(out["mult"]), _ptr(out["ndist"]), _ptr(out.get("samples")),
@@ -178,8 +194,10 @@ def draft_list_noalloc(q_logits, key, ctx, pos, K: int, row_k=None, mode: int = 
 
 
 def verify_tree(p_logits, key, ctx, pos, gamma: int, seq_off, node_draft_row, draft_tok, draft_ndist, child_node,
-                temperature: float = 1.0, ws=None, status=None, out=None, stream=None):
-    """pps_verify_tree.  Returns dict(winner, word, accept_len, n_emitted, emitted, score, score_sum)."""
+                temperature: float = 1.0, ws=None, status=None, out=None, stream=None, top_k: int = 0,
+                top_p: float = 1.0):
+    """pps_verify_tree (pps_verify_tree_trunc when top_k > 0).
+    Returns dict(winner, word, accept_len, n_emitted, emitted, score, score_sum)."""
     n, V, stride = _rows(p_logits)
     dev = p_logits.device
     n_seq = seq_off.numel() - 1
@@ -199,6 +217,16 @@ def verify_tree(p_logits, key, ctx, pos, gamma: int, seq_off, node_draft_row, dr
                     ("draft_ndist", draft_ndist), ("child_node", child_node)):
         if not t.is_cuda or t.dtype != torch.int32 or not t.is_contiguous():
             raise TypeError(f"{name} must be a contiguous CUDA int32 tensor")
+    if top_k > 0:
+        code = lib().pps_verify_tree_trunc(_ptr(p_logits), _dtype_code(p_logits), n, V, stride, _ids(key, ctx, pos),
+                                           float(temperature), int(top_k), float(top_p), n_seq, int(gamma),
+                                           _ptr(seq_off), _ptr(node_draft_row), draft_tok.shape[0], _ptr(draft_tok),
+                                           _ptr(draft_ndist), int(K), _ptr(child_node), _ptr(out["winner"]),
+                                           _ptr(out["word"]), _ptr(out["accept_len"]), _ptr(out["n_emitted"]),
+                                           _ptr(out["emitted"]), _ptr(out["score"]), _ptr(out["score_sum"]),
+                                           _ptr(status), _ptr(ws), ws.numel(), _stream(stream))
+        _check("pps_verify_tree_trunc", code)
+        return out
     code = lib().pps_verify_tree(_ptr(p_logits), _dtype_code(p_logits), n, V, stride, _ids(key, ctx, pos),
                                  float(temperature), n_seq, int(gamma), _ptr(seq_off), _ptr(node_draft_row),
                                  draft_tok.shape[0], _ptr(draft_tok), _ptr(draft_ndist), int(K), _ptr(child_node), _ptr(out["winner"]),

@@ -88,3 +88,26 @@ def test_workspace_size_grows_with_rows_and_sequences():
     c = pps.workspace_size(200, 1000, 8, 50)
     assert 0 < a < b <= c
     assert pps.status_string(pps.ERR_WORKSPACE) == "workspace missing or too small"
+
+
+def test_truncated_calls_validate_top_k_and_top_p():
+    L = pps.lib()
+    fake = ctypes.c_void_p(256)
+    ids = pps.RowIds(256, 256, 256)
+
+    def draft(tk, tp, **kw):
+        a = dict(K=4, ws=fake)
+        a.update(kw)
+        return L.pps_draft_list_trunc(fake, pps.BF16, 4, 100, 100, ids, 1.0, tk, tp, a["K"], None, pps.DISTINCT,
+                                      fake, None, fake, fake, None, None, a["ws"], 1 << 30, None)
+
+    def verify(tk, tp):
+        return L.pps_verify_tree_trunc(fake, pps.F32, 10, 100, 100, ids, 1.0, tk, tp, 2, 2, fake, fake, 4, fake, fake,
+                                       2, fake, fake, fake, fake, fake, fake, fake, fake, None, fake, 1 << 30, None)
+
+    for tk, tp in ((0, 1.0), (-3, 1.0), (pps.MAX_TOP_K + 1, 1.0), (5, 0.0), (5, -0.5), (5, 1.01),
+                   (5, float("nan"))):
+        assert draft(tk, tp) == pps.ERR_INVALID_ARG, (tk, tp)
+        assert verify(tk, tp) == pps.ERR_INVALID_ARG, (tk, tp)
+    assert draft(5, 0.9, K=0) == pps.ERR_INVALID_ARG   # the untruncated checks still apply
+    assert draft(5, 0.9, ws=None) == pps.ERR_WORKSPACE
