@@ -264,21 +264,16 @@ __device__ __forceinline__ float from_order_key(uint32_t u) {
     return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
 }
 
-// Threshold for an empty list: the k-th largest of the 32 x NV per-vector
-// maxima of the first iteration (bitwise search on order keys).  They are
-// maxima of distinct vectors, so at least k tokens of the segment reach it
-// and l_(k) >= it.
+// Threshold for an empty buffer, from the first iteration's vectors: the
+// k-th largest of the 32 x NV per-vector maxima (bitwise search on order
+// keys).  They are maxima of distinct vectors of the segment, so at least k
+// of its tokens reach it and l_(k) >= it.
 template <int DT>
-__device__ __noinline__ float seed_top(const char* row, int64_t v0, int k) {
+__device__ __forceinline__ float seed_thr(const uint4 (&d)[PPS_TRUNC_UNITS], int k) {
     constexpr int NV = PPS_TRUNC_UNITS;
-    const int lane = threadIdx.x & 31;
-    const uint4* p = reinterpret_cast<const uint4*>(row) + v0 + lane;
     uint32_t key[NV];
 #pragma unroll
-    for (int j = 0; j < NV; ++j) {
-        const uint4 d[1] = {__ldg(p + 32 * j)};
-        key[j] = order_key(vecs_max<DT>(d, 0, 1));
-    }
+    for (int j = 0; j < NV; ++j) key[j] = order_key(vecs_max<DT>(d, j, 1));
     uint32_t res = 0;
     for (int b = 31; b >= 0; --b) {
         const uint32_t cand = res | (1u << b);
@@ -474,15 +469,32 @@ __device__ __noinline__ CandState cand_append(CandState C, float* sv, int* si, c
     }
 }
 
-// One iteration of the fast scan (NV vectors per lane, d[j] = vector vfirst +
-// 32 j): a packed max tree per lane and a vote; when a lane reaches the
-// threshold its flagged vectors are staged in shared memory and their wanted
-// tokens appended.
+// Flagged vectors wait in a per-warp queue in shared memory (their 16 bytes
+// and their index in the row); one iteration adds at most 32 x NV.
+constexpr int kTQueueCap = 32 + 32 * PPS_TRUNC_UNITS;
+
+// Work off the queue, one vector per lane, 32 at a time.
 template <int DT>
-__device__ __forceinline__ void topk_step(CandState& C, float* sv, int* si, uint4* st,
+__device__ __noinline__ CandState topk_flush(CandState C, float* sv, int* si, const uint4* qv, const uint32_t* qi,
+                                             int qn, int k) {
+    constexpr int VW = DT == 1 ? 8 : 4;
+    const int lane = threadIdx.x & 31;
+    __syncwarp();
+    for (int base = 0; base < qn; base += 32) {
+        const bool mine = base + lane < qn;
+        const int i0 = mine ? (int)(qi[base + lane] * VW) : 0;
+        C = cand_append<DT>(C, sv, si, qv + base, mine ? 1u : 0u, i0, k);
+    }
+    return C;
+}
+
+// One iteration of the fast scan (NV vectors per lane, d[j] = vector vfirst +
+// 32 j): a packed max tree per lane and a vote; vectors with a logit at or
+// over the threshold are queued, and the queue is worked off once it holds 32.
+template <int DT>
+__device__ __forceinline__ void topk_step(CandState& C, float* sv, int* si, uint4* qv, uint32_t* qi, int& qn,
                                           const uint4 (&d)[PPS_TRUNC_UNITS], int64_t vfirst, int k) {
     constexpr int NV = PPS_TRUNC_UNITS;
-    constexpr int VW = DT == 1 ? 8 : 4;
     const int lane = threadIdx.x & 31;
     unsigned vf = 0;
     if constexpr (DT == 1) {
@@ -514,26 +526,58 @@ __device__ __forceinline__ void topk_step(CandState& C, float* sv, int* si, uint
             for (int j = 0; j < NV; ++j) vf |= (unsigned)(mv[j] >= C.thr) << j;
         }
     }
+    const int n = __popc(vf);
+    int off = n;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(FULL, off, o);
+        if (lane >= o) off += t;
+    }
+    const int total = __shfl_sync(FULL, off, 31);
+    off += qn - n;
 #pragma unroll
     for (int j = 0; j < NV; ++j)
-        if ((vf >> j) & 1u) st[j * 32 + lane] = d[j];
-    C = cand_append<DT>(C, sv, si, st, vf, (int)(vfirst * VW), k);
+        if ((vf >> j) & 1u) {
+            qv[off] = d[j];
+            qi[off] = (uint32_t)(vfirst + 32 * j);
+            ++off;
+        }
+    qn += total;
+    if (qn >= 32) {
+        C = topk_flush<DT>(C, sv, si, qv, qi, qn, k);
+        qn = 0;
+    }
 }
 
+// The fast scan of the full vectors [v0, vend) of a row: iterations of NV
+// vectors 32 apart per lane; in the last, partial one the vectors past vend
+// read as -inf.  The first iteration also seeds the threshold.
 template <int DT>
-__device__ __forceinline__ void topk_scan(CandState& C, float* sv, int* si, uint4* st, const char* row, int64_t v0,
-                                          int64_t n_it, int k) {
+__device__ __forceinline__ void topk_scan(CandState& C, float* sv, int* si, uint4* qv, uint32_t* qi,
+                                          const char* row, int64_t v0, int64_t vend, int k) {
     constexpr int NV = PPS_TRUNC_UNITS;
     constexpr int STEP = 32 * NV;
     const int lane = threadIdx.x & 31;
+    const uint32_t ninf = DT == 1 ? 0xff80ff80u : 0xff800000u;
+    const uint4 fill = make_uint4(ninf, ninf, ninf, ninf);
+    const int64_t n_it = (vend - v0 + STEP - 1) / STEP;
     const uint4* p = reinterpret_cast<const uint4*>(row) + v0 + lane;
+    int qn = 0;
     for (int64_t it = 0; it < n_it; ++it) {
+        const int64_t vb = v0 + it * STEP + lane;
         uint4 d[NV];
+        if (v0 + (it + 1) * STEP <= vend) {
 #pragma unroll
-        for (int j = 0; j < NV; ++j) d[j] = ldg_stream(p + 32 * j);
+            for (int j = 0; j < NV; ++j) d[j] = ldg_stream(p + 32 * j);
+        } else {
+#pragma unroll
+            for (int j = 0; j < NV; ++j) d[j] = vb + 32 * j < vend ? ldg_stream(p + 32 * j) : fill;
+        }
         p += STEP;
-        topk_step<DT>(C, sv, si, st, d, v0 + it * STEP + lane, k);
+        if (it == 0) C.thr = seed_thr<DT>(d, k);
+        topk_step<DT>(C, sv, si, qv, qi, qn, d, vb, k);
     }
+    if (qn > 0) C = topk_flush<DT>(C, sv, si, qv, qi, qn, k);
 }
 
 // Scalar-load path: the last partial iteration of a segment, the ragged
@@ -565,21 +609,18 @@ __device__ __noinline__ TopList topk_tail(TopList L, const char* row, int64_t V,
 
 template <int DT, bool VEC>
 __device__ __forceinline__ void topk_segment(TopList& L, const char* row, int64_t V, int64_t v0, int64_t v1, int k,
-                                             float* sv, int* si, uint4* st) {
+                                             float* sv, int* si, uint4* qv, uint32_t* qi) {
     constexpr int VW = DT == 1 ? 8 : 4;
-    constexpr int STEP = 32 * PPS_TRUNC_UNITS;
     const int64_t nfull = V / VW;
     const int64_t vend = VEC ? min(v1, nfull) : v0;
-    const int64_t n_it = vend > v0 ? (vend - v0) / STEP : 0;
-    int64_t base = v0;
-    if (n_it > 0) {
-        CandState C{seed_top<DT>(row, v0, k), -kInf, 0};
-        topk_scan<DT>(C, sv, si, st, row, v0, n_it, k);
+    if (vend > v0) {
+        CandState C{-kInf, -kInf, 0};
+        topk_scan<DT>(C, sv, si, qv, qi, row, v0, vend, k);
         if (C.n > kTopMax) C = cand_compact(C, sv, si, k);
         L = cand_to_list(C, sv, si, k);
-        base = v0 + n_it * STEP;
     }
-    if (base < v1) L = topk_tail<DT>(L, row, V, base, v1, k);
+    // the row's ragged last vector, or a whole unaligned segment
+    if (vend < v1) L = topk_tail<DT>(L, row, V, vend > v0 ? vend : v0, v1, k);
 }
 
 // ---------------------------------------------------------------- finishing a truncated row
@@ -634,26 +675,25 @@ __device__ __noinline__ float top_p_keep(const TopList& L, float lk, int64_t ext
 }
 
 // lower 32 of two lists sorted ascending by (key, token): into x
-__device__ __forceinline__ void merge_low_d(double& xk, int& xi, double yk, int yi, int lane) {
-    const double rk = __shfl_sync(FULL, yk, 31 - lane);
+__device__ __forceinline__ void merge_low_f(float& xk, int& xi, float yk, int yi, int lane) {
+    const float rk = __shfl_sync(FULL, yk, 31 - lane);
     const int ri = __shfl_sync(FULL, yi, 31 - lane);
-    if (lex_less_d(rk, ri, xk, xi)) {
+    if (lex_less(rk, ri, xk, xi)) {
         xk = rk;
         xi = ri;
     }
 #pragma unroll
     for (int stride = 16; stride > 0; stride >>= 1) {
-        const double ok = __shfl_xor_sync(FULL, xk, stride);
+        const float ok = __shfl_xor_sync(FULL, xk, stride);
         const int oi = __shfl_xor_sync(FULL, xi, stride);
         const bool lower = (lane & stride) == 0;
-        const bool o_less = lex_less_d(ok, oi, xk, xi);
+        const bool o_less = lex_less(ok, oi, xk, xi);
         if (lower ? o_less : (!o_less && !(ok == xk && oi == xi))) {
             xk = ok;
             xi = oi;
         }
     }
 }
-
 template <int DT, bool VERIFY>
 __device__ __noinline__ void finalize_trunc(const RaceArgs& a, int64_t r, const TopList& L, int kr, int kp,
                                             float* s_val) {
@@ -683,18 +723,19 @@ __device__ __noinline__ void finalize_trunc(const RaceArgs& a, int64_t r, const 
         finalize_row<DT, VERIFY>(a, r, st.L.lk, st.L.li, fminf(st.L.th, st.L.tf), kr, kp, lane);
         return;
     }
-    // S = the list's entries with logit >= keep: exact fp64 keys, sorted
-    double ka = (double)INFINITY, kb = (double)INFINITY;
+    // S = the list's entries with logit >= keep: the race's fp32 keys, the 32
+    // smallest in lane order; finalize_row re-keys near ties in fp64 (S is
+    // complete, so nothing was dropped: drop bound +inf)
+    float ka = kInf, kb = kInf;
     int ia = L.ai, ib = L.bi;
-    if (L.av > -kInf && L.av >= keep) ka = key64(word_of(key, ctx, pos, ia, 1), L.av, a.T);
-    if (L.bv > -kInf && L.bv >= keep) kb = key64(word_of(key, ctx, pos, ib, 1), L.bv, a.T);
-    if (ka == (double)INFINITY) ia = INT_MAX;
-    if (kb == (double)INFINITY) ib = INT_MAX;
-    warp_sort_d(ka, ia, lane);
-    warp_sort_d(kb, ib, lane);
-    merge_low_d(ka, ia, kb, ib, lane);
-    const int nvalid = __popc(__ballot_sync(FULL, ka < (double)INFINITY));
-    emit_row<DT, VERIFY>(a, r, ka, (float)ka, ia, nvalid, kr, lane, key, ctx, pos);
+    if (L.av > -kInf && L.av >= keep) ka = key32(word_of(key, ctx, pos, ia, 1), L.av, a.c);
+    if (L.bv > -kInf && L.bv >= keep) kb = key32(word_of(key, ctx, pos, ib, 1), L.bv, a.c);
+    if (ka == kInf) ia = INT_MAX;
+    if (kb == kInf) ib = INT_MAX;
+    warp_sort(ka, ia, lane);
+    warp_sort(kb, ib, lane);
+    merge_low_f(ka, ia, kb, ib, lane);
+    finalize_row<DT, VERIFY>(a, r, ka, ia, kInf, kr, kp, lane);
 }
 
 template <int DT, bool VERIFY>
@@ -746,7 +787,8 @@ __global__ void __launch_bounds__(kThreads, PPS_TRUNC_MIN_BLOCKS) trunc_kernel(c
     __shared__ float s_val[kTopMax];
     __shared__ float s_cv[kCandCap];
     __shared__ int s_ci[kCandCap];
-    __shared__ uint4 s_stage[32 * PPS_TRUNC_UNITS];
+    __shared__ uint4 s_qv[kTQueueCap];
+    __shared__ uint32_t s_qi[kTQueueCap];
     const int64_t NW = a.G;
     const int64_t gw = blockIdx.x;
     const int64_t g0 = gw * a.total / NW, g1 = (gw + 1) * a.total / NW;
@@ -764,7 +806,7 @@ __global__ void __launch_bounds__(kThreads, PPS_TRUNC_MIN_BLOCKS) trunc_kernel(c
         const char* row = reinterpret_cast<const char*>(a.logits) + (size_t)r * (size_t)a.stride * esz;
         TopList L;
         L.reset();
-        topk_segment<DT, VEC>(L, row, a.V, v0, v1, a.top_k, s_cv, s_ci, s_stage);
+        topk_segment<DT, VEC>(L, row, a.V, v0, v1, a.top_k, s_cv, s_ci, s_qv, s_qi);
         finish_trunc_segment<DT, VERIFY>(a, r, gw, NW, v0, v1, L, kr, kp, s_val);
     }
 }
