@@ -165,7 +165,7 @@ static pps_status draft_list(const void* q_logits, pps_dtype dtype, int64_t n_ro
     const bool vec = vec_ok(q_logits, dtype, row_stride);
     cudaError_t e;
     if (top_k > 0) {
-        a.G = trunc_grid(a.total, dt, false, vec);
+        a.G = trunc_grid(a.total, a.n_rows, dt, false, vec);
         e = launch_trunc(a, dt, false, vec, (cudaStream_t)stream);
     } else {
         a.G = race_grid(a.total, dt, false, vec);
@@ -237,7 +237,7 @@ static pps_status verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_n
     const bool vec = vec_ok(p_logits, dtype, row_stride);
     cudaError_t e;
     if (top_k > 0) {
-        a.G = trunc_grid(a.total, dt, true, vec);
+        a.G = trunc_grid(a.total, a.n_rows, dt, true, vec);
         e = launch_trunc(a, dt, true, vec, (cudaStream_t)stream);
     } else {
         a.G = race_grid(a.total, dt, true, vec);

@@ -87,7 +87,7 @@ void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials
 cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
 int race_grid(int64_t total, int dtype, bool verify, bool vec);
 cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
-int trunc_grid(int64_t total, int dtype, bool verify, bool vec);
+int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec);
 
 // launchers (pps_misc.cu)
 cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,

@@ -940,7 +940,11 @@ cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cud
     return cudaGetLastError();
 }
 
-int trunc_grid(int64_t total, int dtype, bool verify, bool vec) {
+// Rows stay whole where the grid allows (a segment's candidate count grows
+// like k ln(segment / k), and a row finished by one warp needs no merge):
+// with at most as many rows as resident warps, each row gets the same number
+// of warps s; with more rows, the grid is the resident one.
+int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec) {
     static int sms = 0, occ[2][2][2] = {};
     int dev = 0;
     cudaGetDevice(&dev);
@@ -963,6 +967,7 @@ int trunc_grid(int64_t total, int dtype, bool verify, bool vec) {
     int64_t g = (int64_t)sms * o;
     int64_t by_size = (total + kMinVecsPerWarp - 1) / kMinVecsPerWarp;
     if (by_size < g) g = by_size;
+    if (n_rows > 0 && n_rows <= g) g = n_rows * (g / n_rows);
     if (g > kGridMax) g = kGridMax;
     if (g < 1) g = 1;
     return (int)g;

@@ -30,8 +30,11 @@
 #ifndef PPS_TRUNC_UNITS
 #define PPS_TRUNC_UNITS 8  // 16-byte vectors per lane per iteration of the top-k scan (even)
 #endif
+#ifndef PPS_TRUNC_EAGER
+#define PPS_TRUNC_EAGER 96  // buffered candidates at which a queue flush also compacts
+#endif
 #ifndef PPS_TRUNC_MIN_BLOCKS
-#define PPS_TRUNC_MIN_BLOCKS 16
+#define PPS_TRUNC_MIN_BLOCKS 20
 #endif
 
 // ---------------------------------------------------------------- top lists
@@ -303,6 +306,7 @@ struct CandState {
     }
 };
 
+template <int DT>
 __device__ __noinline__ CandState cand_compact(CandState C, float* sv, int* si, int k) {
     constexpr int PER = kCandCap / 32;
     const int lane = threadIdx.x & 31;
@@ -316,15 +320,17 @@ __device__ __noinline__ CandState cand_compact(CandState C, float* sv, int* si, 
         ix[j] = q < C.n ? si[q] : INT_MAX;
     }
     __syncwarp();
-    // t = the k-th largest buffered logit, bit by bit on order keys
+    // t = the k-th largest buffered logit, bit by bit on order keys (bf16
+    // values: the high 16 bits decide, the low ones are all 0 or all 1)
     uint32_t res = 0;
-    for (int b = 31; b >= 0; --b) {
+    for (int b = 31; b >= (DT == 1 ? 16 : 0); --b) {
         const uint32_t cand = res | (1u << b);
         int n = 0;
 #pragma unroll
         for (int j = 0; j < PER; ++j) n += v[j] > -kInf && order_key(v[j]) >= cand;
         if (__reduce_add_sync(FULL, (unsigned)n) >= (unsigned)k) res = cand;
     }
+    if (DT == 1 && !(res & 0x80000000u)) res |= 0xffffu;  // a negative value: its key ends in ones
     const float t = from_order_key(res);
     int ng = 0;
 #pragma unroll
@@ -465,7 +471,7 @@ __device__ __noinline__ CandState cand_append(CandState C, float* sv, int* si, c
         C.n += done ? __shfl_sync(FULL, off + cnt, last) : 0;
         if (fits) vf = 0;
         __syncwarp();
-        C = cand_compact(C, sv, si, k);
+        C = cand_compact<DT>(C, sv, si, k);
     }
 }
 
@@ -485,6 +491,8 @@ __device__ __noinline__ CandState topk_flush(CandState C, float* sv, int* si, co
         const int i0 = mine ? (int)(qi[base + lane] * VW) : 0;
         C = cand_append<DT>(C, sv, si, qv + base, mine ? 1u : 0u, i0, k);
     }
+    // raise the threshold early: a stale one lets through many more tokens
+    if (C.n >= PPS_TRUNC_EAGER) C = cand_compact<DT>(C, sv, si, k);
     return C;
 }
 
@@ -616,7 +624,7 @@ __device__ __forceinline__ void topk_segment(TopList& L, const char* row, int64_
     if (vend > v0) {
         CandState C{-kInf, -kInf, 0};
         topk_scan<DT>(C, sv, si, qv, qi, row, v0, vend, k);
-        if (C.n > kTopMax) C = cand_compact(C, sv, si, k);
+        if (C.n > kTopMax) C = cand_compact<DT>(C, sv, si, k);
         L = cand_to_list(C, sv, si, k);
     }
     // the row's ragged last vector, or a whole unaligned segment
