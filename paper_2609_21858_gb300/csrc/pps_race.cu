@@ -594,7 +594,7 @@ __device__ __forceinline__ float logit_at(const RaceArgs& a, int64_t r, int64_t 
     return load_logit<DT>(base, i);
 }
 
-__device__ void walk_sequence(const RaceArgs& a, int s);
+__device__ void walk_sequence(const RaceArgs& a, int s, int lane);
 
 // Outputs of row r from its sorted entries: lane m holds the m-th smallest
 // (key, token) of the row's list (dk fp64 when exact, sk fp32), nvalid of them
@@ -726,39 +726,51 @@ __device__ __forceinline__ int seq_of_node(const int32_t* seq_off, int n_seq, in
     return lo;
 }
 
-__device__ __noinline__ void walk_sequence(const RaceArgs& a, int s) {
+// The walk of sequence s by the whole warp: per step one round of loads for
+// the node (winner, word, draft row) and one for its draft list and children
+// (lane m takes list slot m); emitted token t is kept by lane t % 32, and the
+// scores of all emitted tokens are computed at once at the end.
+__device__ __noinline__ void walk_sequence(const RaceArgs& a, int s, int lane) {
     const int W = a.gamma + 1;
     int c = __ldg(a.seq_off + s);
     if (c < 0 || c >= a.n_rows) return;
     int acc = 0, ne = 0;
-    double S = 0.0;
+    int y_[3] = {-1, -1, -1};
+    uint32_t w_[3] = {0u, 0u, 0u};
+    auto keep = [&](int y, uint32_t w) {
+        if ((ne & 31) == lane) {
+            const int q = ne >> 5;
+            if (q == 0) { y_[0] = y; w_[0] = w; }
+            else if (q == 1) { y_[1] = y; w_[1] = w; }
+            else { y_[2] = y; w_[2] = w; }
+        }
+        ++ne;
+    };
     bool stopped = false;
     for (int step = 0; step < a.gamma; ++step) {
-        int y = __ldcg(a.out_winner + c);
+        const int y = __ldcg(a.out_winner + c);
+        const uint32_t w = __ldcg(a.out_word + c);
+        const int dr = __ldg(a.node_draft_row + c);
         if (y < 0) {
             stopped = true;
             break;
         }
-        double A = score64(__ldcg(a.out_word + c));
-        a.out_em[(size_t)s * W + ne] = y;
-        a.out_sc[(size_t)s * W + ne] = (float)A;
-        S += A;
-        ++ne;
-        int dr = __ldg(a.node_draft_row + c), found = -1;
+        keep(y, w);
+        int found = -1, nxt = -1;
         if (dr >= 0 && dr < a.n_draft) {
-            int nd = min(__ldg(a.draft_nd + dr), a.Kd);
-            for (int m = 0; m < nd; ++m)
-                if (__ldg(a.draft_tok + (size_t)dr * a.Kd + m) == y) {
-                    found = m;
-                    break;
-                }
+            const int nd = min(__ldg(a.draft_nd + dr), a.Kd);
+            int t = -1, ch = -1;
+            if (lane < nd) {
+                t = __ldg(a.draft_tok + (size_t)dr * a.Kd + lane);
+                ch = __ldg(a.child_node + (size_t)dr * a.Kd + lane);
+            }
+            const unsigned hit = __ballot_sync(FULL, lane < nd && t == y);
+            if (hit) {
+                found = __ffs(hit) - 1;
+                nxt = __shfl_sync(FULL, ch, found);
+            }
         }
-        if (found < 0) {
-            stopped = true;
-            break;
-        }
-        int nxt = __ldg(a.child_node + (size_t)dr * a.Kd + found);
-        if (nxt < 0 || nxt >= a.n_rows) {
+        if (found < 0 || nxt < 0 || nxt >= a.n_rows) {
             stopped = true;
             break;
         }
@@ -766,22 +778,31 @@ __device__ __noinline__ void walk_sequence(const RaceArgs& a, int s) {
         ++acc;
     }
     if (!stopped) {
-        int y = __ldcg(a.out_winner + c);
-        if (y >= 0) {
-            double A = score64(__ldcg(a.out_word + c));
-            a.out_em[(size_t)s * W + ne] = y;
-            a.out_sc[(size_t)s * W + ne] = (float)A;
-            S += A;
-            ++ne;
+        const int y = __ldcg(a.out_winner + c);
+        const uint32_t w = __ldcg(a.out_word + c);
+        if (y >= 0) keep(y, w);
+    }
+    // scores of the emitted tokens, their sum in emission order
+    double A[3];
+    double S = 0.0;
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+        const int t = q * 32 + lane;
+        A[q] = t < ne ? score64(w_[q]) : 0.0;
+        if (t < W) {
+            a.out_em[(size_t)s * W + t] = t < ne ? y_[q] : -1;
+            a.out_sc[(size_t)s * W + t] = (float)A[q];
         }
     }
-    for (int t = ne; t < W; ++t) {
-        a.out_em[(size_t)s * W + t] = -1;
-        a.out_sc[(size_t)s * W + t] = 0.0f;
+    for (int t = 0; t < ne; ++t) {
+        const int q = t >> 5;
+        S += __shfl_sync(FULL, q == 0 ? A[0] : (q == 1 ? A[1] : A[2]), t & 31);
     }
-    a.out_acc[s] = acc;
-    a.out_ne[s] = ne;
-    a.out_ss[s] = S;
+    if (lane == 0) {
+        a.out_acc[s] = acc;
+        a.out_ne[s] = ne;
+        a.out_ss[s] = S;
+    }
 }
 
 // End of a row segment: publish the warp's list, or merge the row's lists if
@@ -791,15 +812,18 @@ __device__ __noinline__ void walk_sequence(const RaceArgs& a, int s) {
 // sequence's last node walks it.
 __device__ __noinline__ void sequence_ticket(const RaceArgs& a, int64_t r, int lane) {
     __threadfence();
+    int s = 0;
+    unsigned last = 0;
     if (lane == 0) {
-        int s = seq_of_node(a.seq_off, a.n_seq, r);
+        s = seq_of_node(a.seq_off, a.n_seq, r);
         int nn = __ldg(a.seq_off + s + 1) - __ldg(a.seq_off + s);
         unsigned t = atomicAdd(a.seq_cnt + s, 1u);
-        if (t == (unsigned)(nn - 1)) {
-            a.seq_cnt[s] = 0u;
-            __threadfence();
-            walk_sequence(a, s);
-        }
+        last = t == (unsigned)(nn - 1);
+        if (last) a.seq_cnt[s] = 0u;
+    }
+    if (__shfl_sync(FULL, last, 0)) {
+        __threadfence();
+        walk_sequence(a, __shfl_sync(FULL, s, 0), lane);
     }
     __syncwarp();
 }
