@@ -32,6 +32,7 @@ METRIC = "verified rows/s and GB/s vs HBM peak at V=128256, K=8, B=64 (1xGB300)"
 WIDE_MULS_PER_TOKEN = 4.5
 WIDE_MULS_PER_SM_CLK = 32
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "race_kernel_zipf_k8_traffic.txt")
+TRUNC_TRAFFIC_FILE = os.path.join(ROOT, "profiles", "trunc_kernel_zipf_k8_top50_traffic.txt")
 
 
 def kernel_source_digest() -> str:
@@ -62,11 +63,11 @@ def philox_only_rate(dev) -> float:
     return 5 * 4 * n_blocks / (e0.elapsed_time(e1) / 1e3)
 
 
-def _traffic(which: str):
+def _traffic(which: str, path: str = TRAFFIC_FILE):
     """DRAM bytes per launch from the committed ncu summary, if it was taken on the current kernel."""
     try:
         kv = {}
-        with open(TRAFFIC_FILE) as f:
+        with open(path) as f:
             for line in f:
                 if "=" in line and not line.startswith("#"):
                     k, v = line.strip().split("=", 1)
@@ -323,7 +324,12 @@ def main():
     clk = (clocks.get("sm_mhz") or 2070.0) * 1e6
     mul_peak = sms * WIDE_MULS_PER_SM_CLK * clk / 1e12
     mul_ach = tok_verify * WIDE_MULS_PER_TOKEN / (t_verify / 1e3) / 1e12
-    traffic = _traffic("verify") if args.top_k == 0 else None
+    traffic = None
+    if args.workload == "zipf_k8" and args.n_seq is None:
+        if args.top_k == 0:
+            traffic = _traffic("verify")
+        elif args.top_k == 50 and args.top_p == 1.0:
+            traffic = _traffic("verify", TRUNC_TRAFFIC_FILE)
     philox_tok_s = philox_only_rate(dev) if rank == 0 else None
     emitted = float(vout["n_emitted"].sum().item())
 
