@@ -77,6 +77,14 @@ def lib():
             L.orc_wm_score.restype = None
             L.orc_words.argtypes = [i64, i64, u64p, u64p, u32p, i32, u32p]
             L.orc_words.restype = None
+            L.orc_score_kind.argtypes = [ctypes.c_uint32, i32, f64]
+            L.orc_score_kind.restype = f64
+            L.orc_gamma_tail_logp.argtypes = [i64, f64]
+            L.orc_gamma_tail_logp.restype = f64
+            L.orc_chernoff_u_logp.argtypes = [i64, f64]
+            L.orc_chernoff_u_logp.restype = f64
+            L.orc_wm_detect.argtypes = [i64, i32p, u64p, u64p, u32p, i32, f64, i32, i64p, f64p, f64p, f64p]
+            L.orc_wm_detect.restype = None
             L.orc_truncate_rows.argtypes = [f32p, i64, i64, i64, f64, i32, f64, f32p, f64p]
             L.orc_truncate_rows.restype = None
             L.orc_set_threads.argtypes = [ctypes.c_int]
@@ -215,3 +223,36 @@ def truncate_rows(logits, top_k: int = 0, top_p: float = 1.0, T: float = 1.0):
     lib().orc_truncate_rows(_ptr(l, ctypes.c_float), n, V, V, float(T), int(top_k), float(top_p),
                             _ptr(out, ctypes.c_float), _ptr(mg, ctypes.c_double))
     return out, mg
+
+
+AARONSON, U_SCORE, LI, PL = 0, 1, 2, 3
+
+
+def score_kind(w: int, kind: int, param: float = 0.0) -> float:
+    return float(lib().orc_score_kind(w, int(kind), float(param)))
+
+
+def gamma_tail_logp(M: int, S: float) -> float:
+    """ln P(Gamma(M,1) >= S)"""
+    return float(lib().orc_gamma_tail_logp(int(M), float(S)))
+
+
+def chernoff_u_logp(M: int, S: float) -> float:
+    """Chernoff bound on ln P(sum of M iid U(0,1) >= S)"""
+    return float(lib().orc_chernoff_u_logp(int(M), float(S)))
+
+
+def wm_detect(tokens, key, ctx, pos, seg_off, kind: int = AARONSON, param: float = 0.0):
+    """Per token scores, per segment sums and log p-values of the detector pass."""
+    t = _c(tokens, np.int32)
+    n = t.shape[0]
+    key, ctx, pos = _c(key, np.uint64), _c(ctx, np.uint64), _c(pos, np.uint32)
+    so = _c(seg_off, np.int64)
+    n_seg = so.shape[0] - 1
+    sc = np.zeros(n, np.float64)
+    sums = np.zeros(n_seg, np.float64)
+    logp = np.zeros(n_seg, np.float64)
+    lib().orc_wm_detect(n, _ptr(t, ctypes.c_int32), _ptr(key, ctypes.c_uint64), _ptr(ctx, ctypes.c_uint64),
+                        _ptr(pos, ctypes.c_uint32), int(kind), float(param), n_seg, _ptr(so, ctypes.c_int64),
+                        _ptr(sc, ctypes.c_double), _ptr(sums, ctypes.c_double), _ptr(logp, ctypes.c_double))
+    return sc, sums, logp

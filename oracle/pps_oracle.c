@@ -40,6 +40,18 @@
  *   orc_wm_score       A_t = -ln(1 - r_t(w_t)) with pivot r_t = u of the
  *                      emitted token (Eq. 2; App. D.1 "Gumbel watermark";
  *                      detector algorithm, App. E).
+ *   orc_score_kind     per-token detection scores of the same pivot r = u
+ *                      (App. D): Aaronson A = -ln(1 - r); the U-score r;
+ *                      Li et al.'s optimal Gumbel score h*_{gum,Delta}(r) =
+ *                      ln(k r^(Delta/(1-Delta)) + [q > 0] r^((1-q)/q)),
+ *                      k = floor(1/(1-Delta)), q = 1 - k(1-Delta); Lattimore's
+ *                      truncated power law min(eps^-1/2, (1-r)^-1/2) - (2 - sqrt eps).
+ *   orc_gamma_tail_logp  ln P(Gamma(M,1) >= S), the exact null p-value of S_A
+ *                      (App. D.2; detector algorithm, App. E), for integer M as
+ *                      the Poisson sum P(Poisson(S) <= M - 1).
+ *   orc_chernoff_u_logp  the Chernoff bound on the U-score tail,
+ *                      inf over lambda >= 0 of M ln((e^lambda - 1)/lambda) - lambda S
+ *                      (App. D.2), by golden-section search on the convex exponent.
  *   orc_truncate_rows  the logit processing of the experiments (Sec. 6 setup:
  *                      top-k = 50, top-p = 1; truncation leaves a support of at
  *                      most k tokens, Sec. 4.2): tokens outside the top-k /
@@ -416,6 +428,97 @@ void orc_truncate_rows(const float* logits, int64_t n_rows, int64_t V, int64_t s
             o[i] = (!isnan(l[i]) && l[i] != -INFINITY && (double)l[i] >= cut) ? l[i] : -INFINITY;
         if (margin) margin[r] = mg;
         free(v);
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* detection scores and p-values                                       */
+/* ------------------------------------------------------------------ */
+
+/* kind 0 Aaronson, 1 U-score, 2 Li (param Delta), 3 Lattimore PL (param eps) */
+double orc_score_kind(uint32_t w, int32_t kind, double param)
+{
+    double r = orc_uniform(w), one_minus_r = orc_one_minus_uniform(w);
+    if (kind == 0) return orc_score_word(w);
+    if (kind == 1) return r;
+    if (kind == 2) {
+        double k = floor(1.0 / (1.0 - param));
+        double q = 1.0 - k * (1.0 - param);
+        double ln_r = w < 0x80000000u ? log(r) : log1p(-one_minus_r);
+        double sum = k * exp(ln_r * param / (1.0 - param));
+        if (q > 0.0) sum += exp(ln_r * (1.0 - q) / q);
+        return log(sum);
+    }
+    if (kind == 3) {
+        double cap = 1.0 / sqrt(param), x = 1.0 / sqrt(one_minus_r);
+        return (x < cap ? x : cap) - (2.0 - sqrt(param));
+    }
+    return NAN;
+}
+
+/* ln P(Gamma(M,1) >= S) = ln sum_{j=0}^{M-1} e^{-S} S^j / j!  (M >= 1), the terms
+ * added in log space from j = 0 up */
+double orc_gamma_tail_logp(int64_t M, double S)
+{
+    if (S <= 0.0) return 0.0;
+    double lt = -S, ls = log(S), m = lt, acc = 1.0;  /* running log-sum-exp: m + ln acc */
+    for (int64_t j = 1; j < M; ++j) {
+        lt += ls - log((double)j);
+        if (lt > m) { acc = acc * exp(m - lt) + 1.0; m = lt; }
+        else acc += exp(lt - m);
+    }
+    return m + log(acc);
+}
+
+static double orc_chernoff_exponent(double lambda, double M, double S)
+{
+    if (lambda == 0.0) return 0.0;
+    return M * log(expm1(lambda) / lambda) - lambda * S;
+}
+
+/* min over lambda >= 0 of the Chernoff exponent (0 at lambda = 0); the
+ * exponent is convex in lambda, so golden-section search on [0, L] with L
+ * grown until the exponent rises */
+double orc_chernoff_u_logp(int64_t M, double S)
+{
+    double Md = (double)M;
+    if (S <= 0.5 * Md) return 0.0;
+    if (S >= Md) return -INFINITY;
+    double hi = 1.0;
+    while (orc_chernoff_exponent(2.0 * hi, Md, S) < orc_chernoff_exponent(hi, Md, S) && hi < 1e6) hi *= 2.0;
+    double lo = 0.0, up = 2.0 * hi;
+    const double g = 0.6180339887498949;
+    double a = up - g * (up - lo), b = lo + g * (up - lo);
+    double fa = orc_chernoff_exponent(a, Md, S), fb = orc_chernoff_exponent(b, Md, S);
+    for (int it = 0; it < 200; ++it) {
+        if (fa < fb) { up = b; b = a; fb = fa; a = up - g * (up - lo); fa = orc_chernoff_exponent(a, Md, S); }
+        else { lo = a; a = b; fa = fb; b = lo + g * (up - lo); fb = orc_chernoff_exponent(b, Md, S); }
+    }
+    double best = fa < fb ? fa : fb;
+    return best < 0.0 ? best : 0.0;
+}
+
+/* Detector pass with a score kind: per token score (kind, param) of the
+ * regenerated first-arrival word; per segment sums and log p-values
+ * (kind 0: Gamma tail, kind 1: Chernoff bound on the U-score; NaN otherwise). */
+void orc_wm_detect(int64_t n, const int32_t* tokens, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
+                   int32_t kind, double param, int32_t n_seg, const int64_t* seg_off, double* score, double* sums,
+                   double* logp)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t t = 0; t < n; ++t)
+        score[t] = orc_score_kind(orc_word(key[t], ctx[t], pos[t], tokens[t], 1), kind, param);
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int32_t g = 0; g < n_seg; ++g) {
+        double S = 0.0;
+        for (int64_t t = seg_off[g]; t < seg_off[g + 1]; ++t) S += score[t];
+        sums[g] = S;
+        int64_t M = seg_off[g + 1] - seg_off[g];
+        if (!logp) continue;
+        if (M == 0) logp[g] = 0.0;
+        else if (kind == 0) logp[g] = orc_gamma_tail_logp(M, S);
+        else if (kind == 1) logp[g] = orc_chernoff_u_logp(M, S);
+        else logp[g] = NAN;
     }
 }
 
