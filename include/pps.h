@@ -211,6 +211,39 @@ pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32
                         float* out_score, double* out_sum, pps_stream_t stream);
 
 /*
+ * pps_wm_detect -- the detector pass with a choice of per-token score of the
+ * same pivot r = u (App. D) and per-segment log p-values (App. D.2; detector
+ * algorithm, App. E).  Arguments as pps_wm_score, plus:
+ *
+ * kind         PPS_SCORE_AARONSON  -ln(1 - r)                    (param unused)
+ *              PPS_SCORE_U         r, the U-score                (param unused)
+ *              PPS_SCORE_LI        Li et al.'s optimal Gumbel score
+ *                                  ln(k r^(D/(1-D)) + [q > 0] r^((1-q)/q)),
+ *                                  k = floor(1/(1-D)), q = 1 - k(1-D); param D in (0, 1)
+ *              PPS_SCORE_POWER_LAW Lattimore's truncated power law
+ *                                  min(e^(-1/2), (1-r)^(-1/2)) - (2 - e^(1/2)); param e in (0, 1]
+ * out_score    nullable [n] per-token scores (fp32)
+ * out_sum      [n_seg] (or [1]) per-segment sums (fp64); zeroed by the call;
+ *              nullable only when out_logp is NULL
+ * out_logp     nullable [n_seg] (or [1]) natural log of the segment's null
+ *              p-value, M = its token count: AARONSON ln P(Gamma(M,1) >= S)
+ *              (exact); U the Chernoff bound
+ *              inf_l M ln((e^l - 1)/l) - l S (0 for S <= M/2); NaN for the
+ *              other kinds (the paper gives them no null law); 0 for M = 0.
+ * PPS_ERR_INVALID_ARG for param out of range, PPS_ERR_UNSUPPORTED for kind.
+ */
+typedef enum {
+    PPS_SCORE_AARONSON = 0,
+    PPS_SCORE_U = 1,
+    PPS_SCORE_LI = 2,
+    PPS_SCORE_POWER_LAW = 3
+} pps_score_kind;
+
+pps_status pps_wm_detect(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,
+                         pps_score_kind kind, double param, float* out_score, double* out_sum, double* out_logp,
+                         pps_stream_t stream);
+
+/*
  * pps_draft_list_noalloc -- pps_draft_list for callers that must not
  * allocate device memory per call and cannot hand the library a workspace:
  * code running under an allocator that forbids new allocations once serving

@@ -315,15 +315,46 @@ pps_status pps_draft_list_noalloc(const void* q_logits, pps_dtype dtype, int64_t
     return launch_race(a, dt, false, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
 }
 
-pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,
-                        float* out_score, double* out_sum, pps_stream_t stream) {
+pps_status pps_wm_detect(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,
+                         pps_score_kind kind, double param, float* out_score, double* out_sum, double* out_logp,
+                         pps_stream_t stream) {
     if (n < 0) return PPS_ERR_INVALID_ARG;
     if (seg_off && n_seg < 1) return PPS_ERR_INVALID_ARG;
     if (n > 0 && (!tokens || !ids.key || !ids.ctx_hash || !ids.pos)) return PPS_ERR_INVALID_ARG;
     if (!out_score && !out_sum) return PPS_ERR_INVALID_ARG;
-    cudaError_t e = launch_wm_score(tokens, ids.key, ids.ctx_hash, ids.pos, n, seg_off ? n_seg : 1, seg_off, out_score,
-                                    out_sum, (cudaStream_t)stream);
+    if (out_logp && !out_sum) return PPS_ERR_INVALID_ARG;
+    ScoreParams P;
+    std::memset(&P, 0, sizeof(P));
+    P.kind = (int)kind;
+    switch (kind) {
+        case PPS_SCORE_AARONSON:
+        case PPS_SCORE_U:
+            break;
+        case PPS_SCORE_LI: {
+            if (!(param > 0.0 && param < 1.0)) return PPS_ERR_INVALID_ARG;
+            const double k = std::floor(1.0 / (1.0 - param)), q = 1.0 - k * (1.0 - param);
+            P.k = (float)k;
+            P.a = (float)(param / (1.0 - param));
+            P.has_q = q > 0.0 ? 1.0f : 0.0f;
+            P.b = q > 0.0 ? (float)((1.0 - q) / q) : 0.0f;
+            break;
+        }
+        case PPS_SCORE_POWER_LAW:
+            if (!(param > 0.0 && param <= 1.0)) return PPS_ERR_INVALID_ARG;
+            P.cap = (float)(1.0 / std::sqrt(param));
+            P.centre = (float)(2.0 - std::sqrt(param));
+            break;
+        default:
+            return PPS_ERR_UNSUPPORTED;
+    }
+    cudaError_t e = launch_wm_score(tokens, ids.key, ids.ctx_hash, ids.pos, n, seg_off ? n_seg : 1, seg_off, P,
+                                    out_score, out_sum, out_logp, (cudaStream_t)stream);
     return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,
+                        float* out_score, double* out_sum, pps_stream_t stream) {
+    return pps_wm_detect(tokens, ids, n, n_seg, seg_off, PPS_SCORE_AARONSON, 0.0, out_score, out_sum, nullptr, stream);
 }
 
 pps_status pps_philox_words(pps_row_ids ids, int64_t n_rows, int64_t vocab, int32_t arrival, uint32_t* out,

@@ -16,6 +16,7 @@
 #pragma once
 #include <cstdint>
 #include <cuda_runtime.h>
+#include "pps_internal.h"
 
 namespace pps {
 
@@ -245,6 +246,23 @@ __device__ __forceinline__ double score64(uint32_t w) {
 __device__ __forceinline__ float score32(uint32_t w) {
     if (w < 0x80000000u) return -log1pf(-fmaf((float)w, 0x1p-32f, 0x1p-33f));
     return -logf(fmaf((float)(~w), 0x1p-32f, 0x1p-33f));
+}
+
+// Detection score kinds of the pivot r = u (App. D): Aaronson -ln(1 - r), the
+// U-score r, Li et al.'s h*_{gum,Delta}(r) = ln(k r^a + [q > 0] r^b) with
+// a = Delta/(1-Delta), b = (1-q)/q, and the truncated power law
+// min(cap, (1-r)^(-1/2)) - centre.  Constants come from the host.
+__device__ __forceinline__ float score_kind32(uint32_t w, const ScoreParams& P) {
+    if (P.kind == 0) return score32(w);
+    const float u = fmaf((float)w, 0x1p-32f, 0x1p-33f);     // r
+    const float v = fmaf((float)(~w), 0x1p-32f, 0x1p-33f);  // 1 - r
+    if (P.kind == 1) return w < 0x80000000u ? u : 1.0f - v;
+    if (P.kind == 2) {
+        const float lr = w < 0x80000000u ? logf(u) : log1pf(-v);
+        const float x = P.k * expf(P.a * lr) + (P.has_q != 0.0f ? expf(P.b * lr) : 0.0f);
+        return logf(x);
+    }
+    return fminf(P.cap, 1.0f / sqrtf(v)) - P.centre;
 }
 
 // fp32 key k = log2(E) + log2(log2 e) - l log2(e)/T  ->  s = ln E - l/T = (k - log2(log2 e)) ln 2

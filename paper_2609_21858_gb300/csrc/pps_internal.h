@@ -90,9 +90,14 @@ cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cu
 int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec);
 
 // launchers (pps_misc.cu)
+// detection score kind and its constants (pps_device.cuh score_kind32)
+struct ScoreParams {
+    int kind;  // 0 Aaronson, 1 U, 2 Li, 3 power law
+    float a, b, k, has_q, cap, centre;
+};
 cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
-                            int64_t n, int32_t n_seg, const int64_t* seg_off, float* out_score, double* out_sum,
-                            cudaStream_t stream);
+                            int64_t n, int32_t n_seg, const int64_t* seg_off, const ScoreParams& P, float* out_score,
+                            double* out_sum, double* out_logp, cudaStream_t stream);
 cudaError_t launch_words(const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int64_t n_rows, int64_t V,
                          int32_t arrival, uint32_t* out, cudaStream_t stream);
 cudaError_t launch_selftest(uint64_t w_begin, uint64_t w_end, float* out, cudaStream_t stream);

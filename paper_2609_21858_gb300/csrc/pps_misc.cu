@@ -20,8 +20,8 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
                                                        const uint64_t* __restrict__ key,
                                                        const uint64_t* __restrict__ ctx,
                                                        const uint32_t* __restrict__ pos, int64_t n, int32_t n_seg,
-                                                       const int64_t* __restrict__ seg_off, float* out_score,
-                                                       double* out_sum) {
+                                                       const int64_t* __restrict__ seg_off, ScoreParams P,
+                                                       float* out_score, double* out_sum) {
     const int lane = threadIdx.x & 31;
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t c0 = gw * kScoreChunk;
@@ -49,7 +49,7 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
         float A = 0.0f;
         if (t < c1) {
             int64_t tok = tokens[t];
-            A = score32(word_of(key[t], ctx[t], pos[t], tok, 1));
+            A = score_kind32(word_of(key[t], ctx[t], pos[t], tok, 1), P);
             if (out_score) out_score[t] = A;
         }
         if (!out_sum) continue;
@@ -97,6 +97,89 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
         }
     }
     if (out_sum && !seg_off && lane == 0) atomicAdd(out_sum, carry);
+}
+
+// ln P(Gamma(M,1) >= S) for integer M >= 1, as the Poisson probability
+// P(N <= M-1), N ~ Poisson(S): for S >= M the terms e^-S S^j / j! are summed
+// downward from j = M-1 (ratios j/S < 1); below, 1 - P(N >= M) with the upper
+// terms summed upward from j = M (ratios S/j < 1).  Stops when a term no
+// longer changes the sum.
+__device__ double gamma_tail_logp(int64_t M, double S) {
+    if (!(S > 0.0)) return 0.0;
+    const double ls = log(S);
+    if (S >= (double)M) {
+        const double inv = 1.0 / S;
+        double r = 1.0, sum = 1.0;
+        for (int64_t j = M - 1; j > 0; --j) {
+            r *= (double)j * inv;
+            const double ns = sum + r;
+            if (ns == sum) break;
+            sum = ns;
+        }
+        return -S + (double)(M - 1) * ls - lgamma((double)M) + log(sum);
+    }
+    double r = 1.0, sum = 1.0;
+    for (int64_t j = M + 1;; ++j) {
+        r *= S / (double)j;
+        const double ns = sum + r;
+        if (ns == sum) break;
+        sum = ns;
+    }
+    const double up = exp(-S + (double)M * ls - lgamma((double)M + 1.0)) * sum;
+    return log1p(-up);
+}
+
+// Chernoff bound on ln P(U_1 + ... + U_M >= S): the exponent
+// M ln((e^l - 1)/l) - l S at the l where the mean of the exponentially tilted
+// uniform, 1/(1 - e^-l) - 1/l, equals S/M (Newton steps kept inside a
+// bisection bracket).  0 for S <= M/2, -inf for S >= M.
+__device__ double chernoff_u_logp(int64_t M, double S) {
+    const double x = S / (double)M;
+    if (!(x > 0.5)) return 0.0;
+    if (x >= 1.0) return -INFINITY;
+    auto mean = [](double l) {
+        if (l < 1e-3) return 0.5 + l / 12.0 - l * l * l / 720.0;
+        return 1.0 / (-expm1(-l)) - 1.0 / l;
+    };
+    auto slope = [](double l) {  // variance of the tilted uniform
+        if (l < 1e-3) return 1.0 / 12.0 - l * l / 240.0;
+        const double e = exp(-l), d = -expm1(-l);
+        return 1.0 / (l * l) - e / (d * d);
+    };
+    double lo = 0.0, hi = 2.0 / (1.0 - x) + 10.0;
+    double l = x < 0.75 ? 12.0 * (x - 0.5) : 1.0 / (1.0 - x);
+    for (int it = 0; it < 100; ++it) {
+        const double f = mean(l) - x;
+        if (f > 0.0) hi = l;
+        else lo = l;
+        double nl = l - f / slope(l);
+        if (!(nl > lo && nl < hi)) nl = 0.5 * (lo + hi);
+        if (fabs(nl - l) <= 1e-15 * l) {
+            l = nl;
+            break;
+        }
+        l = nl;
+    }
+    const double e = (double)M * log(expm1(l) / l) - l * S;
+    return e < 0.0 ? e : 0.0;
+}
+
+// per-segment ln p-values from the segment sums (kind 0 Gamma tail, 1 Chernoff on U)
+__global__ void seg_logp_kernel(int64_t n, int32_t n_seg, const int64_t* __restrict__ seg_off,
+                                const double* __restrict__ sums, int kind, double* out_logp) {
+    const int g = blockIdx.x * blockDim.x + threadIdx.x;
+    if (g >= n_seg) return;
+    const int64_t M = seg_off ? seg_off[g + 1] - seg_off[g] : n;
+    double lp;
+    if (M <= 0)
+        lp = 0.0;
+    else if (kind == 0)
+        lp = gamma_tail_logp(M, sums[g]);
+    else if (kind == 1)
+        lp = chernoff_u_logp(M, sums[g]);
+    else
+        lp = __longlong_as_double(0x7ff8000000000000ll);  // NaN: no null law for this score
+    out_logp[g] = lp;
 }
 
 __global__ void words_kernel(const uint64_t* __restrict__ key, const uint64_t* __restrict__ ctx,
@@ -152,17 +235,26 @@ cudaError_t launch_philox_rate(uint64_t n_blocks, uint32_t* out, int out_len, cu
 }
 
 cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
-                            int64_t n, int32_t n_seg, const int64_t* seg_off, float* out_score, double* out_sum,
-                            cudaStream_t stream) {
+                            int64_t n, int32_t n_seg, const int64_t* seg_off, const ScoreParams& P, float* out_score,
+                            double* out_sum, double* out_logp, cudaStream_t stream) {
+    const int32_t ns = seg_off ? n_seg : 1;
     if (out_sum) {
-        cudaError_t e = cudaMemsetAsync(out_sum, 0, sizeof(double) * (size_t)(seg_off ? n_seg : 1), stream);
+        cudaError_t e = cudaMemsetAsync(out_sum, 0, sizeof(double) * (size_t)ns, stream);
         if (e != cudaSuccess) return e;
     }
-    if (n == 0) return cudaSuccess;
-    int64_t warps = (n + kScoreChunk - 1) / kScoreChunk;
-    int64_t blocks = (warps * 32 + 255) / 256;
-    wm_score_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, key, ctx, pos, n, n_seg, seg_off, out_score, out_sum);
-    return cudaGetLastError();
+    if (n > 0) {
+        int64_t warps = (n + kScoreChunk - 1) / kScoreChunk;
+        int64_t blocks = (warps * 32 + 255) / 256;
+        wm_score_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, key, ctx, pos, n, n_seg, seg_off, P, out_score,
+                                                              out_sum);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    if (out_logp && ns > 0) {
+        seg_logp_kernel<<<(ns + 127) / 128, 128, 0, stream>>>(n, ns, seg_off, out_sum, P.kind, out_logp);
+        return cudaGetLastError();
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_words(const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int64_t n_rows, int64_t V,

@@ -70,6 +70,8 @@ def lib():
                                                  vp, vp, vp, vp, vp, vp, vp]
             L.pps_draft_list_noalloc.restype = ctypes.c_int
             L.pps_wm_score.argtypes = [vp, RowIds, i64, i32, vp, vp, vp, vp]
+            L.pps_wm_detect.argtypes = [vp, RowIds, i64, i32, vp, ctypes.c_int, ctypes.c_double, vp, vp, vp, vp]
+            L.pps_wm_detect.restype = ctypes.c_int
             L.pps_wm_score.restype = ctypes.c_int
             L.pps_philox_words.argtypes = [RowIds, i64, i64, i32, vp, vp]
             L.pps_philox_words.restype = ctypes.c_int
@@ -254,6 +256,28 @@ def wm_score(tokens, key, ctx, pos, seg_off=None, out_score=None, out_sum=None, 
                               _ptr(out_sum), _stream(stream))
     _check("pps_wm_score", code)
     return out_score, out_sum
+
+
+SCORE_AARONSON, SCORE_U, SCORE_LI, SCORE_POWER_LAW = 0, 1, 2, 3
+
+
+def wm_detect(tokens, key, ctx, pos, seg_off=None, kind: int = SCORE_AARONSON, param: float = 0.0,
+              want_scores: bool = True, want_logp: bool = True, stream=None):
+    """pps_wm_detect.  Returns (scores or None, sums, log p-values or None)."""
+    n = tokens.numel()
+    dev = tokens.device
+    n_seg = seg_off.numel() - 1 if seg_off is not None else 1
+    out_score = torch.empty(n, dtype=torch.float32, device=dev) if want_scores else None
+    out_sum = torch.empty(n_seg, dtype=torch.float64, device=dev)
+    out_logp = torch.empty(n_seg, dtype=torch.float64, device=dev) if want_logp else None
+    if tokens.dtype != torch.int32 or not tokens.is_cuda:
+        raise TypeError("tokens must be a CUDA int32 tensor")
+    if seg_off is not None and (seg_off.dtype != torch.int64 or not seg_off.is_cuda):
+        raise TypeError("seg_off must be a CUDA int64 tensor")
+    code = lib().pps_wm_detect(_ptr(tokens), _ids(key, ctx, pos), n, n_seg, _ptr(seg_off), int(kind), float(param),
+                               _ptr(out_score), _ptr(out_sum), _ptr(out_logp), _stream(stream))
+    _check("pps_wm_detect", code)
+    return out_score, out_sum, out_logp
 
 
 def philox_words(key, ctx, pos, vocab: int, arrival: int = 1, stream=None):

@@ -111,3 +111,19 @@ def test_truncated_calls_validate_top_k_and_top_p():
         assert verify(tk, tp) == pps.ERR_INVALID_ARG, (tk, tp)
     assert draft(5, 0.9, K=0) == pps.ERR_INVALID_ARG   # the untruncated checks still apply
     assert draft(5, 0.9, ws=None) == pps.ERR_WORKSPACE
+
+
+def test_detect_validates_kind_and_parameter():
+    L = pps.lib()
+    fake = ctypes.c_void_p(256)
+    ids = pps.RowIds(256, 256, 256)
+
+    def detect(kind, param, out_sum=fake, out_logp=fake):
+        return L.pps_wm_detect(fake, ids, 10, 1, None, kind, param, None, out_sum, out_logp, None)
+
+    assert detect(7, 0.0) == pps.ERR_UNSUPPORTED
+    for bad in (0.0, 1.0, -0.5, float("nan")):
+        assert detect(pps.SCORE_LI, bad) == pps.ERR_INVALID_ARG
+    for bad in (0.0, 1.5, float("nan")):
+        assert detect(pps.SCORE_POWER_LAW, bad) == pps.ERR_INVALID_ARG
+    assert detect(pps.SCORE_AARONSON, 0.0, out_sum=None) == pps.ERR_INVALID_ARG  # p-values need the sums

@@ -1,0 +1,99 @@
+"""GPU parity of the detector suite (pps_wm_detect) against the oracle: the
+per-token scores of every kind, the per-segment sums, and the log p-values
+(evaluated by the oracle at the GPU's own sums, so that the two questions
+stay separate)."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_21858_gb300 import pps, synth
+from parity import dev_ids
+
+pytestmark = pytest.mark.gpu
+
+KINDS = [(pps.SCORE_AARONSON, 0.0), (pps.SCORE_U, 0.0), (pps.SCORE_LI, 0.3), (pps.SCORE_LI, 0.5),
+         (pps.SCORE_LI, 0.85), (pps.SCORE_POWER_LAW, 0.01), (pps.SCORE_POWER_LAW, 1.0)]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.set_device(0)
+    pps.lib()
+
+
+def _tuples(n, seed):
+    rng = np.random.default_rng(seed)
+    tok = rng.integers(0, 152064, n, dtype=np.int32)
+    key = rng.integers(0, 2 ** 64, n, dtype=np.uint64)
+    ctx = rng.integers(0, 2 ** 64, n, dtype=np.uint64)
+    pos = rng.integers(0, 2 ** 32, n, dtype=np.uint32)
+    return tok, key, ctx, pos
+
+
+def _segments(n, seed):
+    rng = np.random.default_rng(seed)
+    cuts = np.sort(rng.choice(np.arange(1, n), 60, replace=False))
+    seg = np.concatenate([[0], cuts[:20], cuts[20:21], cuts[20:], [n]]).astype(np.int64)  # includes an empty one
+    return seg
+
+
+@pytest.mark.parametrize("kind,param", KINDS)
+def test_scores_sums_and_p_values_match_the_oracle(kind, param):
+    n = 50000
+    tok, key, ctx, pos = _tuples(n, 11 + kind)
+    seg = _segments(n, 5)
+    k, c, p = dev_ids(key, ctx, pos)
+    sc, sums, logp = pps.wm_detect(torch.as_tensor(tok).cuda(), k, c, p, torch.as_tensor(seg).cuda(), kind, param)
+    torch.cuda.synchronize()
+    sc, sums, logp = sc.cpu().numpy(), sums.cpu().numpy(), logp.cpu().numpy()
+    osc, osums, _ = oracle.wm_detect(tok, key, ctx, pos, seg, kind, param)
+    # per-token fp32 scores against fp64: relative where large, absolute near zero
+    np.testing.assert_allclose(sc, osc, rtol=2e-5, atol=2e-6 * max(1.0, np.abs(osc).max()))
+    np.testing.assert_allclose(sums, osums, rtol=2e-5, atol=1e-4)
+    for g in range(len(seg) - 1):
+        M = int(seg[g + 1] - seg[g])
+        if M == 0:
+            assert logp[g] == 0.0
+        elif kind == pps.SCORE_AARONSON:
+            assert logp[g] == pytest.approx(oracle.gamma_tail_logp(M, float(sums[g])), rel=1e-10, abs=1e-12)
+        elif kind == pps.SCORE_U:
+            assert logp[g] == pytest.approx(oracle.chernoff_u_logp(M, float(sums[g])), rel=1e-9, abs=1e-12)
+        else:
+            assert math.isnan(logp[g])
+
+
+def test_p_values_in_watermarked_tails_and_single_segment():
+    # tokens chosen by the race (watermarked): large S_A, ln p far below zero; no seg_off = one segment
+    wl = synth.make_workload("chain4x4", n_seq=8, vocab=2000, dtype=torch.float32, seed=3)
+    t = wl.tree
+    v = pps.verify_tree(wl.p_logits.cuda(), wl.node_key.cuda(), wl.node_ctx.cuda(), wl.node_pos.cuda(), t.gamma,
+                        torch.as_tensor(t.seq_off).cuda(), torch.as_tensor(t.node_draft_row).cuda(),
+                        torch.zeros(t.n_draft, t.K, dtype=torch.int32, device="cuda") - 1,
+                        torch.zeros(t.n_draft, dtype=torch.int32, device="cuda"),
+                        torch.as_tensor(t.child_node).cuda())
+    win = v["winner"]
+    _, sums, logp = pps.wm_detect(win, wl.node_key.cuda(), wl.node_ctx.cuda(), wl.node_pos.cuda())
+    torch.cuda.synchronize()
+    M = t.n_nodes
+    S = float(sums.item())
+    assert S > M  # watermarked: E[A] > 1
+    assert logp.item() == pytest.approx(oracle.gamma_tail_logp(M, S), rel=1e-10)
+    assert logp.item() < math.log(1e-3)
+
+
+@pytest.mark.parametrize("M", [1, 2, 7, 128, 1000, 4096, 20000])
+def test_gamma_and_chernoff_for_one_segment_of_m_tokens(M):
+    # seg_off = NULL: one segment of all M tokens; null tokens, so S is near M (Aaronson) or M/2 (U)
+    tok, key, ctx, pos = _tuples(M, M)
+    k, c, p = dev_ids(key, ctx, pos)
+    t = torch.as_tensor(tok).cuda()
+    _, sa, la = pps.wm_detect(t, k, c, p, None, pps.SCORE_AARONSON)
+    _, su, lu = pps.wm_detect(t, k, c, p, None, pps.SCORE_U)
+    torch.cuda.synchronize()
+    assert la.item() == pytest.approx(oracle.gamma_tail_logp(M, float(sa.item())), rel=1e-10, abs=1e-12)
+    assert lu.item() == pytest.approx(oracle.chernoff_u_logp(M, float(su.item())), rel=1e-9, abs=1e-12)
