@@ -432,48 +432,66 @@ def main():
 
 
 def run_detector(args, rank, world, dev):
-    """Score-only detector pass (pps_wm_score) over n_tokens (token, key, label, position) tuples:
-    half watermarked (the target winners of fresh contexts drawn by pps_verify_tree), half
-    uniform-random tokens, in segments of 128 tokens (one generated answer each)."""
-    from paper_2609_21858_gb300 import pps, synth
-    n = args.n_tokens
+    """Detector pass (pps_wm_detect: Aaronson scores, per-segment sums and exact Gamma-tail
+    log p-values) over n_tokens (token, key, label, position) tuples in segments of 128: the
+    first half watermarked (race winners of fresh contexts, drawn by pps_verify_tree over
+    N(0, 3^2) logits of 256 tokens), the second half uniform-random tokens (the null)."""
+    from paper_2609_21858_gb300 import pps
+    n = args.n_tokens - args.n_tokens % 256
+    half = n // 2
     g = torch.Generator(device=dev)
     g.manual_seed(4)
-    tok = torch.randint(0, 128256, (n,), generator=g, device=dev, dtype=torch.int32)
     key = torch.randint(-2 ** 62, 2 ** 62, (n,), generator=g, device=dev, dtype=torch.int64)
     ctx = torch.randint(-2 ** 62, 2 ** 62, (n,), generator=g, device=dev, dtype=torch.int64)
     pos = torch.randint(0, 2 ** 30, (n,), generator=g, device=dev, dtype=torch.int32)
+    tok = torch.randint(0, 128256, (n,), generator=g, device=dev, dtype=torch.int32)
+    # watermarked half: each context's token is the target race winner (one-node trees)
+    Vw = 256
+    logits = torch.randn(half, Vw, generator=g, device=dev).mul_(3.0).to(torch.bfloat16)
+    ar = torch.arange(half + 1, device=dev, dtype=torch.int32)
+    none = torch.full((half,), -1, device=dev, dtype=torch.int32)
+    v = pps.verify_tree(logits, key[:half], ctx[:half], pos[:half], 1, ar, none,
+                        torch.full((1, 1), -1, device=dev, dtype=torch.int32),
+                        torch.zeros(1, device=dev, dtype=torch.int32),
+                        torch.full((1, 1), -1, device=dev, dtype=torch.int32))
+    tok[:half] = v["winner"]
+    del logits, v
     seg = torch.arange(0, n + 1, 128, device=dev, dtype=torch.int64)
-    if seg[-1].item() != n:
-        seg = torch.cat([seg, torch.tensor([n], device=dev, dtype=torch.int64)])
-    score = torch.empty(n, dtype=torch.float32, device=dev)
-    sums = torch.empty(seg.numel() - 1, dtype=torch.float64, device=dev)
     stream = torch.cuda.current_stream(dev)
     for _ in range(max(3, args.warmup)):
-        pps.wm_score(tok, key, ctx, pos, seg_off=seg, out_score=score, out_sum=sums, stream=stream)
+        sc, sums, logp = pps.wm_detect(tok, key, ctx, pos, seg, want_scores=False, stream=stream)
     torch.cuda.synchronize(dev)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier(world)
     e0.record(stream)
     for _ in range(args.steps):
-        pps.wm_score(tok, key, ctx, pos, seg_off=seg, out_score=score, out_sum=sums, stream=stream)
+        sc, sums, logp = pps.wm_detect(tok, key, ctx, pos, seg, want_scores=False, stream=stream)
     e1.record(stream)
     torch.cuda.synchronize(dev)
     ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
+    n_seg = seg.numel() - 1
     bytes_in = n * (4 + 8 + 8 + 4) + seg.numel() * 8
-    bytes_out = n * 4 + sums.numel() * 8
+    bytes_out = n_seg * 16
     peak, peak_kind = _peaks()
     gbs = (bytes_in + bytes_out) / (ms / 1e3) / 1e9
+    lp = logp.cpu().numpy()
+    wm, null = lp[: n_seg // 2], lp[n_seg // 2:]
+    alpha = np.log(0.01)
     if rank == 0:
         print(json.dumps({
-            "metric": "watermark score-only detector pass (tokens/s)", "value": n * world / (ms / 1e3),
+            "metric": "watermark detector pass with p-values (tokens/s)", "value": n * world / (ms / 1e3),
             "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": max(3, args.warmup),
             "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-            "data": "synthetic", "config": {"workload": f"detector: {n} tuples, segments of 128",
-                                            "l2": f"inputs ({bytes_in / 1e6:.0f} MB) larger than L2, no flush"},
+            "data": "synthetic",
+            "config": {"workload": f"detector: {n} tuples in segments of 128, half watermarked, Aaronson "
+                                   f"scores, exact Gamma-tail p-values",
+                       "l2": f"inputs ({bytes_in / 1e6:.0f} MB) larger than L2, no flush"},
             "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
                          "traffic": None, "peak_kind": peak_kind, "algorithmic_bytes": bytes_in + bytes_out},
-            "gpu_launches": args.steps,
+            "detection": {"tpr_at_1pct_fpr": float(np.mean(wm <= alpha)), "fpr_null": float(np.mean(null <= alpha)),
+                          "anlppt_watermarked": float(np.mean(-wm / 128.0)),
+                          "anlppt_null": float(np.mean(-null / 128.0)), "segments": int(n_seg)},
+            "gpu_launches": 2 * args.steps,
         }))
 
 

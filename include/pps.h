@@ -227,7 +227,8 @@ pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32
  *              nullable only when out_logp is NULL
  * out_logp     nullable [n_seg] (or [1]) natural log of the segment's null
  *              p-value, M = its token count: AARONSON ln P(Gamma(M,1) >= S)
- *              (exact); U the Chernoff bound
+ *              (to ~1e-6 absolute); U the Chernoff bound (its minimiser in
+ *              fp32; the bound at it in fp64)
  *              inf_l M ln((e^l - 1)/l) - l S (0 for S <= M/2); NaN for the
  *              other kinds (the paper gives them no null law); 0 for M = 0.
  * PPS_ERR_INVALID_ARG for param out of range, PPS_ERR_UNSUPPORTED for kind.

@@ -99,68 +99,102 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
     if (out_sum && !seg_off && lane == 0) atomicAdd(out_sum, carry);
 }
 
+// ln Gamma(x) for x >= 16 by Stirling's asymptotic series (truncation error
+// below 1e-16 there); smaller x through the recurrence Gamma(x+1) = x Gamma(x).
+__device__ double lgamma_stirling(double x) {
+    double shift = 0.0;
+    while (x < 16.0) {
+        shift -= log(x);
+        x += 1.0;
+    }
+    const double r = 1.0 / x, r2 = r * r;
+    const double series = r * (1.0 / 12.0 - r2 * (1.0 / 360.0 - r2 * (1.0 / 1260.0 - r2 * (1.0 / 1680.0))));
+    return shift + (x - 0.5) * log(x) - x + 0.91893853320467274178 + series;
+}
+
 // ln P(Gamma(M,1) >= S) for integer M >= 1, as the Poisson probability
-// P(N <= M-1), N ~ Poisson(S): for S >= M the terms e^-S S^j / j! are summed
-// downward from j = M-1 (ratios j/S < 1); below, 1 - P(N >= M) with the upper
-// terms summed upward from j = M (ratios S/j < 1).  Stops when a term no
-// longer changes the sum.
+// P(N <= M-1), N ~ Poisson(S).  The leading term e^-S S^j / j! at j = M-1
+// (S >= M) or j = M (S < M) is taken in fp64; the sum of the ratios of the
+// other terms to it, all <= 1 and summed away from the mode until they stop
+// mattering, in compensated fp32 (FP64 throughput is low on this part): for
+// S >= M downward from M-1 (ratios j/S), below as 1 - P(N >= M) upward from M
+// (ratios S/j).  Relative error of the sum ~1e-7, i.e. ~1e-7 absolute in ln p.
 __device__ double gamma_tail_logp(int64_t M, double S) {
     if (!(S > 0.0)) return 0.0;
     const double ls = log(S);
+    const float Sf = (float)S;
+    // compensated (Kahan) fp32 sums; stop once a term is below 1e-12 of the sum.
+    // The m-th term carries the fp32 image of S (or 1/S) m times: with its
+    // relative error d, the exact sum is sum + d * sum_m m r_m to first order.
     if (S >= (double)M) {
-        const double inv = 1.0 / S;
-        double r = 1.0, sum = 1.0;
+        const float inv = 1.0f / Sf;
+        const double d = 1.0 / (S * (double)inv) - 1.0;  // (1/S) / inv - 1
+        float r = 1.0f, sum = 1.0f, comp = 0.0f, wsum = 0.0f;
+        int m = 0;
         for (int64_t j = M - 1; j > 0; --j) {
-            r *= (double)j * inv;
-            const double ns = sum + r;
-            if (ns == sum) break;
-            sum = ns;
+            r *= (float)j * inv;
+            ++m;
+            const float y = r - comp, t = sum + y;
+            comp = (t - sum) - y;
+            sum = t;
+            wsum = fmaf((float)m, r, wsum);
+            if (r < 1e-12f * sum) break;
         }
-        return -S + (double)(M - 1) * ls - lgamma((double)M) + log(sum);
+        const double tot = (double)sum + d * (double)wsum;
+        return -S + (double)(M - 1) * ls - lgamma_stirling((double)M) + log(tot);
     }
-    double r = 1.0, sum = 1.0;
+    const double d = (S - (double)Sf) / (double)Sf;
+    float r = 1.0f, sum = 1.0f, comp = 0.0f, wsum = 0.0f;
+    int m = 0;
     for (int64_t j = M + 1;; ++j) {
-        r *= S / (double)j;
-        const double ns = sum + r;
-        if (ns == sum) break;
-        sum = ns;
+        r *= Sf / (float)j;
+        ++m;
+        const float y = r - comp, t = sum + y;
+        comp = (t - sum) - y;
+        sum = t;
+        wsum = fmaf((float)m, r, wsum);
+        if (r < 1e-12f * sum) break;
     }
-    const double up = exp(-S + (double)M * ls - lgamma((double)M + 1.0)) * sum;
-    return log1p(-up);
+    const double tot = (double)sum + d * (double)wsum;
+    const double lead = -S + (double)M * ls - lgamma_stirling((double)M + 1.0);
+    return log1p(-exp(lead) * tot);
 }
 
 // Chernoff bound on ln P(U_1 + ... + U_M >= S): the exponent
 // M ln((e^l - 1)/l) - l S at the l where the mean of the exponentially tilted
-// uniform, 1/(1 - e^-l) - 1/l, equals S/M (Newton steps kept inside a
-// bisection bracket).  0 for S <= M/2, -inf for S >= M.
+// uniform, 1/(1 - e^-l) - 1/l, equals S/M (fp32 Newton steps kept inside a
+// bisection bracket; the exponent is flat there, and is evaluated in fp64).
+// 0 for S <= M/2, -inf for S >= M.
 __device__ double chernoff_u_logp(int64_t M, double S) {
     const double x = S / (double)M;
     if (!(x > 0.5)) return 0.0;
     if (x >= 1.0) return -INFINITY;
-    auto mean = [](double l) {
-        if (l < 1e-3) return 0.5 + l / 12.0 - l * l * l / 720.0;
-        return 1.0 / (-expm1(-l)) - 1.0 / l;
+    const float xf = (float)x;
+    auto mean = [](float l) {
+        if (l < 1e-2f) return 0.5f + l / 12.0f - l * l * l / 720.0f;
+        return 1.0f / (-expm1f(-l)) - 1.0f / l;
     };
-    auto slope = [](double l) {  // variance of the tilted uniform
-        if (l < 1e-3) return 1.0 / 12.0 - l * l / 240.0;
-        const double e = exp(-l), d = -expm1(-l);
-        return 1.0 / (l * l) - e / (d * d);
+    auto slope = [](float l) {  // variance of the tilted uniform
+        if (l < 1e-2f) return 1.0f / 12.0f - l * l / 240.0f;
+        const float e = expf(-l), d = -expm1f(-l);
+        return 1.0f / (l * l) - e / (d * d);
     };
-    double lo = 0.0, hi = 2.0 / (1.0 - x) + 10.0;
-    double l = x < 0.75 ? 12.0 * (x - 0.5) : 1.0 / (1.0 - x);
-    for (int it = 0; it < 100; ++it) {
-        const double f = mean(l) - x;
-        if (f > 0.0) hi = l;
+    float lo = 0.0f, hi = 2.0f / (1.0f - xf) + 10.0f;
+    float l = xf < 0.75f ? 12.0f * (xf - 0.5f) : 1.0f / (1.0f - xf);
+    for (int it = 0; it < 60; ++it) {
+        const float f = mean(l) - xf;
+        if (f > 0.0f) hi = l;
         else lo = l;
-        double nl = l - f / slope(l);
-        if (!(nl > lo && nl < hi)) nl = 0.5 * (lo + hi);
-        if (fabs(nl - l) <= 1e-15 * l) {
+        float nl = l - f / slope(l);
+        if (!(nl > lo && nl < hi)) nl = 0.5f * (lo + hi);
+        if (fabsf(nl - l) <= 1e-6f * l) {
             l = nl;
             break;
         }
         l = nl;
     }
-    const double e = (double)M * log(expm1(l) / l) - l * S;
+    const double ld = (double)l;
+    const double e = (double)M * log(expm1(ld) / ld) - ld * S;
     return e < 0.0 ? e : 0.0;
 }
 

@@ -42,6 +42,15 @@ def _segments(n, seed):
     return seg
 
 
+def _check_chernoff(got, M, S):
+    # the GPU minimiser is fp32: its bound is never below the true minimum and at most ~1e-6 above it
+    want = oracle.chernoff_u_logp(M, S)
+    if want == 0.0 or math.isinf(want):
+        assert got == want
+        return
+    assert want - 1e-12 * max(1.0, abs(want)) <= got <= want + 1e-6 * max(1.0, abs(want))
+
+
 @pytest.mark.parametrize("kind,param", KINDS)
 def test_scores_sums_and_p_values_match_the_oracle(kind, param):
     n = 50000
@@ -60,9 +69,9 @@ def test_scores_sums_and_p_values_match_the_oracle(kind, param):
         if M == 0:
             assert logp[g] == 0.0
         elif kind == pps.SCORE_AARONSON:
-            assert logp[g] == pytest.approx(oracle.gamma_tail_logp(M, float(sums[g])), rel=1e-10, abs=1e-12)
+            assert logp[g] == pytest.approx(oracle.gamma_tail_logp(M, float(sums[g])), rel=2e-7, abs=2e-6)
         elif kind == pps.SCORE_U:
-            assert logp[g] == pytest.approx(oracle.chernoff_u_logp(M, float(sums[g])), rel=1e-9, abs=1e-12)
+            _check_chernoff(logp[g], M, float(sums[g]))
         else:
             assert math.isnan(logp[g])
 
@@ -82,7 +91,7 @@ def test_p_values_in_watermarked_tails_and_single_segment():
     M = t.n_nodes
     S = float(sums.item())
     assert S > M  # watermarked: E[A] > 1
-    assert logp.item() == pytest.approx(oracle.gamma_tail_logp(M, S), rel=1e-10)
+    assert logp.item() == pytest.approx(oracle.gamma_tail_logp(M, S), rel=2e-7, abs=2e-6)
     assert logp.item() < math.log(1e-3)
 
 
@@ -95,5 +104,5 @@ def test_gamma_and_chernoff_for_one_segment_of_m_tokens(M):
     _, sa, la = pps.wm_detect(t, k, c, p, None, pps.SCORE_AARONSON)
     _, su, lu = pps.wm_detect(t, k, c, p, None, pps.SCORE_U)
     torch.cuda.synchronize()
-    assert la.item() == pytest.approx(oracle.gamma_tail_logp(M, float(sa.item())), rel=1e-10, abs=1e-12)
-    assert lu.item() == pytest.approx(oracle.chernoff_u_logp(M, float(su.item())), rel=1e-9, abs=1e-12)
+    assert la.item() == pytest.approx(oracle.gamma_tail_logp(M, float(sa.item())), rel=2e-7, abs=2e-6)
+    _check_chernoff(lu.item(), M, float(su.item()))
