@@ -85,6 +85,13 @@ def lib():
             L.orc_chernoff_u_logp.restype = f64
             L.orc_wm_detect.argtypes = [i64, i32p, u64p, u64p, u32p, i32, f64, i32, i64p, f64p, f64p, f64p]
             L.orc_wm_detect.restype = None
+            L.orc_mix64.argtypes = [ctypes.c_uint64]
+            L.orc_mix64.restype = ctypes.c_uint64
+            L.orc_child_label.argtypes = [ctypes.c_uint64, i32]
+            L.orc_child_label.restype = ctypes.c_uint64
+            L.orc_tree_expand.argtypes = [i32, i32, i32, i32, i32p, i32p, i32p, u64p, u64p, u32p, i32p,
+                                          u64p, u64p, u32p, i32p, i32p, u64p, u64p, u32p]
+            L.orc_tree_expand.restype = None
             L.orc_truncate_rows.argtypes = [f32p, i64, i64, i64, f64, i32, f64, f32p, f64p]
             L.orc_truncate_rows.restype = None
             L.orc_set_threads.argtypes = [ctypes.c_int]
@@ -256,3 +263,29 @@ def wm_detect(tokens, key, ctx, pos, seg_off, kind: int = AARONSON, param: float
                         _ptr(pos, ctypes.c_uint32), int(kind), float(param), n_seg, _ptr(so, ctypes.c_int64),
                         _ptr(sc, ctypes.c_double), _ptr(sums, ctypes.c_double), _ptr(logp, ctypes.c_double))
     return sc, sums, logp
+
+
+def mix64(z: int) -> int:
+    return int(lib().orc_mix64(z))
+
+
+def child_label(parent: int, token: int) -> int:
+    return int(lib().orc_child_label(parent, int(token)))
+
+
+def tree_expand(n_seq, K, gamma, depth, d, key, ctx, pos, row_k, tree):
+    """One depth of the dynamic IID tree; `d` = draft_rows(IID) output of this depth's rows,
+    `tree` = dict(child_node [n_seq*R1, K], node_key/ctx/pos [n_seq*N1]) updated in place.
+    Returns (next_key, next_ctx, next_pos, next_k) of depth+1's rows."""
+    n = n_seq * K
+    nk, nc = np.zeros(n, np.uint64), np.zeros(n, np.uint64)
+    npos, nkk = np.zeros(n, np.uint32), np.zeros(n, np.int32)
+    tok, mult, nd = _c(d["tok"], np.int32), _c(d["mult"], np.int32), _c(d["ndist"], np.int32)
+    key, ctx, pos, rk = _c(key, np.uint64), _c(ctx, np.uint64), _c(pos, np.uint32), _c(row_k, np.int32)
+    lib().orc_tree_expand(n_seq, K, gamma, depth, _ptr(tok, ctypes.c_int32), _ptr(mult, ctypes.c_int32),
+                          _ptr(nd, ctypes.c_int32), _ptr(key, ctypes.c_uint64), _ptr(ctx, ctypes.c_uint64),
+                          _ptr(pos, ctypes.c_uint32), _ptr(rk, ctypes.c_int32), _ptr(nk, ctypes.c_uint64),
+                          _ptr(nc, ctypes.c_uint64), _ptr(npos, ctypes.c_uint32), _ptr(nkk, ctypes.c_int32),
+                          _ptr(tree["child_node"], ctypes.c_int32), _ptr(tree["node_key"], ctypes.c_uint64),
+                          _ptr(tree["node_ctx"], ctypes.c_uint64), _ptr(tree["node_pos"], ctypes.c_uint32))
+    return nk, nc, npos, nkk

@@ -52,6 +52,15 @@
  *   orc_chernoff_u_logp  the Chernoff bound on the U-score tail,
  *                      inf over lambda >= 0 of M ln((e^lambda - 1)/lambda) - lambda S
  *                      (App. D.2), by golden-section search on the convex exponent.
+ *   orc_tree_expand    one depth of the dynamic IID draft tree (Alg. 4 with
+ *                      MPFR lists, Eq. 4): every distinct label u of a
+ *                      context's k_r i.i.d. draft samples becomes a child
+ *                      c||u that draws nu(c||u) = its multiplicity samples at
+ *                      the next depth, so the draft paths of a sequence stay
+ *                      K at every depth.  Child context label: SplitMix64's
+ *                      output function of label(c) ^ ((u + 1) * 0x9E3779B97F4A7C15)
+ *                      (a reading: the paper leaves the labeler open),
+ *                      position + 1, same key.
  *   orc_truncate_rows  the logit processing of the experiments (Sec. 6 setup:
  *                      top-k = 50, top-p = 1; truncation leaves a support of at
  *                      most k tokens, Sec. 4.2): tokens outside the top-k /
@@ -519,6 +528,74 @@ void orc_wm_detect(int64_t n, const int32_t* tokens, const uint64_t* key, const 
         else if (kind == 0) logp[g] = orc_gamma_tail_logp(M, S);
         else if (kind == 1) logp[g] = orc_chernoff_u_logp(M, S);
         else logp[g] = NAN;
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* dynamic IID draft tree                                              */
+/* ------------------------------------------------------------------ */
+
+/* SplitMix64's output function (Steele, Lea, Flood, "Fast splittable
+ * pseudorandom number generators", OOPSLA'14) */
+uint64_t orc_mix64(uint64_t z)
+{
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+uint64_t orc_child_label(uint64_t parent, int32_t token)
+{
+    return orc_mix64(parent ^ ((uint64_t)(uint32_t)(token + 1) * 0x9E3779B97F4A7C15ull));
+}
+
+/* Fixed-capacity layout, per sequence b: node (d, i) = b*N1 + (d == 0 ? 0 :
+ * 1 + (d-1)*K + i), N1 = 1 + K*gamma; draft row (d, i) (d < gamma) = b*R1 +
+ * the same offset, R1 = 1 + K*(gamma-1).  Rows of depth d: w_d = (d == 0 ? 1 : K)
+ * per sequence, row (b, i) of the depth = b*w_d + i.  A row with k = 0 is an
+ * absent node.  For every present row (b, i) of depth d, its distinct draft
+ * labels m < ndist (in list order) get child slots j = 0, 1, ... in row order
+ * then list order; child j: ids (key, label(child), pos + 1), k = mult, its
+ * node index written to child_node[draft row (d, i)][m] and its ids to the
+ * node arrays; slots j >= the number of children get k = 0. */
+void orc_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t depth, const int32_t* tok,
+                     const int32_t* mult, const int32_t* ndist, const uint64_t* key, const uint64_t* ctx,
+                     const uint32_t* pos, const int32_t* row_k, uint64_t* next_key, uint64_t* next_ctx,
+                     uint32_t* next_pos, int32_t* next_k, int32_t* child_node, uint64_t* node_key,
+                     uint64_t* node_ctx, uint32_t* node_pos)
+{
+    int64_t N1 = 1 + (int64_t)K * gamma, R1 = 1 + (int64_t)K * (gamma - 1);
+    int32_t w = depth == 0 ? 1 : K;
+    int64_t off_d = depth == 0 ? 0 : 1 + (int64_t)(depth - 1) * K;   /* offset of depth d in a sequence */
+    int64_t off_n = 1 + (int64_t)depth * K;                          /* offset of depth d+1 */
+    for (int32_t b = 0; b < n_seq; ++b) {
+        int32_t j = 0;
+        for (int32_t i = 0; i < w; ++i) {
+            int64_t r = (int64_t)b * w + i;
+            int64_t dr = (int64_t)b * R1 + off_d + i;
+            for (int32_t m = 0; m < K; ++m) child_node[dr * K + m] = -1;
+            if (row_k[r] <= 0) continue;
+            for (int32_t m = 0; m < ndist[r]; ++m) {
+                int64_t q = (int64_t)b * K + j;
+                next_key[q] = key[r];
+                next_ctx[q] = orc_child_label(ctx[r], tok[r * K + m]);
+                next_pos[q] = pos[r] + 1u;
+                next_k[q] = mult[r * K + m];
+                int64_t node = (int64_t)b * N1 + off_n + j;
+                child_node[dr * K + m] = (int32_t)node;
+                node_key[node] = next_key[q];
+                node_ctx[node] = next_ctx[q];
+                node_pos[node] = next_pos[q];
+                ++j;
+            }
+        }
+        for (; j < K; ++j) {
+            int64_t q = (int64_t)b * K + j;
+            next_key[q] = key[(int64_t)b * w];
+            next_ctx[q] = 0;
+            next_pos[q] = 0;
+            next_k[q] = 0;
+        }
     }
 }
 

@@ -267,3 +267,32 @@ def u64(t: torch.Tensor) -> np.ndarray:
 
 def u32(t: torch.Tensor) -> np.ndarray:
     return t.detach().cpu().numpy().view(np.uint32)
+
+
+def _mix64_np(z: np.ndarray) -> np.ndarray:
+    z = z.astype(np.uint64)
+    with np.errstate(over="ignore"):
+        z = (z ^ (z >> np.uint64(30))) * np.uint64(0xBF58476D1CE4E5B9)
+        z = (z ^ (z >> np.uint64(27))) * np.uint64(0x94D049BB133111EB)
+    return z ^ (z >> np.uint64(31))
+
+
+def label_logits(labels, V: int, seed: int = 0, zipf: float = 1.0, noise: float = 1.5) -> np.ndarray:
+    """A synthetic "model": logits of a context as a fixed function of its 64-bit label,
+    -zipf * ln(rank) + noise * N(0,1), the ranks and the noise drawn from SplitMix64 of
+    (label, token, seed).  Deterministic, so both sides of a test see the same logits for
+    the same context, wherever it sits in a tree."""
+    lab = np.asarray(labels, dtype=np.uint64).reshape(-1, 1)
+    col = np.arange(V, dtype=np.uint64).reshape(1, -1)
+    with np.errstate(over="ignore"):
+        base = lab ^ (col * np.uint64(0x9E3779B97F4A7C15)) ^ np.uint64(seed & _MASK64)
+    h1 = _mix64_np(base)
+    h2 = _mix64_np(h1 ^ np.uint64(0xD1B54A32D192ED03))
+    u1 = ((h1 >> np.uint64(11)).astype(np.float64) + 0.5) / 2.0 ** 53
+    u2 = ((h2 >> np.uint64(11)).astype(np.float64) + 0.5) / 2.0 ** 53
+    g = np.sqrt(-2.0 * np.log(u1)) * np.cos(2.0 * np.pi * u2)
+    # a per-context permutation of ranks: order of an independent hash
+    perm = np.argsort(_mix64_np(h2 ^ np.uint64(0x5851F42D4C957F2D)), axis=1, kind="stable")
+    rank = np.empty_like(perm)
+    np.put_along_axis(rank, perm, np.arange(1, V + 1).reshape(1, -1).repeat(lab.shape[0], 0), axis=1)
+    return (-zipf * np.log(rank) + noise * g).astype(np.float32)
