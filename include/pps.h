@@ -195,6 +195,37 @@ pps_status pps_verify_tree_trunc(const void* p_logits, pps_dtype dtype, int64_t 
                                  size_t ws_bytes, pps_stream_t stream);
 
 /*
+ * pps_tree_expand -- one depth of the dynamic IID draft tree (Alg. 4 with
+ * MPFR lists, Eq. 4): each present context c of depth d drew nu(c) i.i.d.
+ * samples (pps_draft_list in PPS_DRAFT_IID mode with row_k = nu); every
+ * distinct label u becomes a child c||u of depth d+1 that draws
+ * nu(c||u) = mult(u) samples, so each sequence keeps K draft paths at every
+ * depth and has at most K nodes per depth.  Child identity: the same key,
+ * position + 1, label SplitMix64-output(label(c) ^ (u + 1) * 0x9E3779B97F4A7C15).
+ *
+ * Fixed-capacity layout (static; nothing else is reallocated per depth):
+ *   nodes      N1 = 1 + K*gamma per sequence; node (b, d, i) =
+ *              b*N1 + (d == 0 ? 0 : 1 + (d-1)*K + i); seq_off[b] = b*N1
+ *   draft rows R1 = 1 + K*(gamma-1) per sequence; the draft row of node
+ *              (b, d, i), d < gamma, is b*R1 + the same offset (node_draft_row)
+ *   depth rows the rows of depth d, w_d = (d == 0 ? 1 : K) per sequence, row
+ *              (b, i) = b*w_d + i: the rows one pps_draft_list call takes
+ * Inputs (depth d's rows, [n_seq*w_d]): draft_tok, draft_mult, draft_ndistinct
+ * (pps_draft_list outputs, stride K), rows (their identities), row_k (nu; 0 =
+ * an absent node, whose list is ignored).
+ * Outputs: next_key, next_ctx, next_pos, next_k [n_seq*K]: identities and nu
+ * of depth d+1's rows in child order (nu = 0 past the last child);
+ * child_node [n_seq*R1, K]: the rows of depth d get their children's node
+ * indices (-1 past ndistinct); node_key, node_ctx, node_pos [n_seq*N1]:
+ * identities of depth d+1's nodes.  All device pointers.
+ */
+pps_status pps_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t depth, const int32_t* draft_tok,
+                           const int32_t* draft_mult, const int32_t* draft_ndistinct, pps_row_ids rows,
+                           const int32_t* row_k, uint64_t* next_key, uint64_t* next_ctx, uint32_t* next_pos,
+                           int32_t* next_k, int32_t* child_node, uint64_t* node_key, uint64_t* node_ctx,
+                           uint32_t* node_pos, pps_stream_t stream);
+
+/*
  * pps_wm_score -- detector pass (detector algorithm of App. E; Eq. 2):
  * regenerate the first-arrival word of every observed token under its
  * context's identity and score it, A_t = -ln(1 - u_t).

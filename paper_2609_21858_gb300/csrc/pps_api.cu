@@ -357,6 +357,23 @@ pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32
     return pps_wm_detect(tokens, ids, n, n_seg, seg_off, PPS_SCORE_AARONSON, 0.0, out_score, out_sum, nullptr, stream);
 }
 
+pps_status pps_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t depth, const int32_t* draft_tok,
+                           const int32_t* draft_mult, const int32_t* draft_ndistinct, pps_row_ids rows,
+                           const int32_t* row_k, uint64_t* next_key, uint64_t* next_ctx, uint32_t* next_pos,
+                           int32_t* next_k, int32_t* child_node, uint64_t* node_key, uint64_t* node_ctx,
+                           uint32_t* node_pos, pps_stream_t stream) {
+    if (n_seq < 0 || K < 1 || K > PPS_MAX_K || gamma < 1 || gamma > 64 || depth < 0 || depth >= gamma)
+        return PPS_ERR_INVALID_ARG;
+    if (n_seq == 0) return PPS_OK;
+    if (!draft_tok || !draft_mult || !draft_ndistinct || !rows.key || !rows.ctx_hash || !rows.pos || !row_k ||
+        !next_key || !next_ctx || !next_pos || !next_k || !child_node || !node_key || !node_ctx || !node_pos)
+        return PPS_ERR_INVALID_ARG;
+    cudaError_t e = launch_tree_expand(n_seq, K, gamma, depth, draft_tok, draft_mult, draft_ndistinct, rows.key,
+                                       rows.ctx_hash, rows.pos, row_k, next_key, next_ctx, next_pos, next_k,
+                                       child_node, node_key, node_ctx, node_pos, (cudaStream_t)stream);
+    return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
 pps_status pps_philox_words(pps_row_ids ids, int64_t n_rows, int64_t vocab, int32_t arrival, uint32_t* out,
                             pps_stream_t stream) {
     if (n_rows < 0 || vocab < 1 || arrival < 1) return PPS_ERR_INVALID_ARG;

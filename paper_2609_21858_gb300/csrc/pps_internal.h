@@ -98,6 +98,11 @@ struct ScoreParams {
 cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
                             int64_t n, int32_t n_seg, const int64_t* seg_off, const ScoreParams& P, float* out_score,
                             double* out_sum, double* out_logp, cudaStream_t stream);
+cudaError_t launch_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t depth, const int32_t* tok,
+                               const int32_t* mult, const int32_t* ndist, const uint64_t* key, const uint64_t* ctx,
+                               const uint32_t* pos, const int32_t* row_k, uint64_t* next_key, uint64_t* next_ctx,
+                               uint32_t* next_pos, int32_t* next_k, int32_t* child_node, uint64_t* node_key,
+                               uint64_t* node_ctx, uint32_t* node_pos, cudaStream_t stream);
 cudaError_t launch_words(const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int64_t n_rows, int64_t V,
                          int32_t arrival, uint32_t* out, cudaStream_t stream);
 cudaError_t launch_selftest(uint64_t w_begin, uint64_t w_end, float* out, cudaStream_t stream);

@@ -216,6 +216,72 @@ __global__ void seg_logp_kernel(int64_t n, int32_t n_seg, const int64_t* __restr
     out_logp[g] = lp;
 }
 
+// SplitMix64's output function (Steele, Lea, Flood, OOPSLA'14): the labeler of
+// a child context, label(c || u) = mix(label(c) ^ (u + 1) * 0x9E3779B97F4A7C15)
+__device__ __forceinline__ uint64_t mix64(uint64_t z) {
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+// One depth of the dynamic IID draft tree (layout in pps.h): warp b takes
+// sequence b, lane i the depth's row i; the distinct labels of the present
+// rows get consecutive child slots (exclusive scan over the rows).
+__global__ void tree_expand_kernel(int32_t n_seq, int32_t K, int32_t gamma, int32_t depth,
+                                   const int32_t* __restrict__ tok, const int32_t* __restrict__ mult,
+                                   const int32_t* __restrict__ ndist, const uint64_t* __restrict__ key,
+                                   const uint64_t* __restrict__ ctx, const uint32_t* __restrict__ pos,
+                                   const int32_t* __restrict__ row_k, uint64_t* next_key, uint64_t* next_ctx,
+                                   uint32_t* next_pos, int32_t* next_k, int32_t* child_node, uint64_t* node_key,
+                                   uint64_t* node_ctx, uint32_t* node_pos) {
+    const int lane = threadIdx.x & 31;
+    const int64_t b = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (b >= n_seq) return;
+    const int64_t N1 = 1 + (int64_t)K * gamma, R1 = 1 + (int64_t)K * (gamma - 1);
+    const int w = depth == 0 ? 1 : K;
+    const int64_t off_d = depth == 0 ? 0 : 1 + (int64_t)(depth - 1) * K, off_n = 1 + (int64_t)depth * K;
+    const int64_t r = b * w + lane;
+    const bool row = lane < w;
+    int nd = 0;
+    if (row && row_k[r] > 0) nd = max(0, min(ndist[r], K));
+    int j0 = nd;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(FULL, j0, o);
+        if (lane >= o) j0 += t;
+    }
+    const int total = min(__shfl_sync(FULL, j0, 31), K);
+    j0 -= nd;
+    if (row) {
+        const int64_t dr = b * R1 + off_d + lane;
+        for (int m = 0; m < K; ++m) {
+            int node = -1;
+            const int j = j0 + m;
+            if (m < nd && j < K) {
+                const int64_t q = b * K + j;
+                const uint64_t lab = mix64(ctx[r] ^ ((uint64_t)(uint32_t)(tok[r * K + m] + 1) * 0x9E3779B97F4A7C15ull));
+                next_key[q] = key[r];
+                next_ctx[q] = lab;
+                next_pos[q] = pos[r] + 1u;
+                next_k[q] = mult[r * K + m];
+                node = (int)(b * N1 + off_n + j);
+                node_key[node] = key[r];
+                node_ctx[node] = lab;
+                node_pos[node] = pos[r] + 1u;
+            }
+            child_node[dr * K + m] = node;
+        }
+    }
+    for (int j = lane; j < K; j += 32)
+        if (j >= total) {
+            const int64_t q = b * K + j;
+            next_key[q] = key[b * w];
+            next_ctx[q] = 0;
+            next_pos[q] = 0;
+            next_k[q] = 0;
+        }
+}
+
 __global__ void words_kernel(const uint64_t* __restrict__ key, const uint64_t* __restrict__ ctx,
                              const uint32_t* __restrict__ pos, int64_t n_rows, int64_t V, int32_t arrival,
                              uint32_t* __restrict__ out) {
@@ -289,6 +355,19 @@ cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const ui
         return cudaGetLastError();
     }
     return cudaSuccess;
+}
+
+cudaError_t launch_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t depth, const int32_t* tok,
+                               const int32_t* mult, const int32_t* ndist, const uint64_t* key, const uint64_t* ctx,
+                               const uint32_t* pos, const int32_t* row_k, uint64_t* next_key, uint64_t* next_ctx,
+                               uint32_t* next_pos, int32_t* next_k, int32_t* child_node, uint64_t* node_key,
+                               uint64_t* node_ctx, uint32_t* node_pos, cudaStream_t stream) {
+    if (n_seq == 0) return cudaSuccess;
+    const int64_t blocks = ((int64_t)n_seq * 32 + 255) / 256;
+    tree_expand_kernel<<<(unsigned)blocks, 256, 0, stream>>>(n_seq, K, gamma, depth, tok, mult, ndist, key, ctx, pos,
+                                                              row_k, next_key, next_ctx, next_pos, next_k, child_node,
+                                                              node_key, node_ctx, node_pos);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_words(const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int64_t n_rows, int64_t V,

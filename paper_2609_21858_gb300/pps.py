@@ -70,6 +70,9 @@ def lib():
                                                  vp, vp, vp, vp, vp, vp, vp]
             L.pps_draft_list_noalloc.restype = ctypes.c_int
             L.pps_wm_score.argtypes = [vp, RowIds, i64, i32, vp, vp, vp, vp]
+            L.pps_tree_expand.argtypes = [i32, i32, i32, i32, vp, vp, vp, RowIds, vp, vp, vp, vp, vp, vp, vp, vp,
+                                          vp, vp]
+            L.pps_tree_expand.restype = ctypes.c_int
             L.pps_wm_detect.argtypes = [vp, RowIds, i64, i32, vp, ctypes.c_int, ctypes.c_double, vp, vp, vp, vp]
             L.pps_wm_detect.restype = ctypes.c_int
             L.pps_wm_score.restype = ctypes.c_int
@@ -256,6 +259,20 @@ def wm_score(tokens, key, ctx, pos, seg_off=None, out_score=None, out_sum=None, 
                               _ptr(out_sum), _stream(stream))
     _check("pps_wm_score", code)
     return out_score, out_sum
+
+
+def tree_expand(K: int, gamma: int, depth: int, draft, rows_key, rows_ctx, rows_pos, row_k, nxt: dict, child_node,
+                nodes: dict, stream=None):
+    """pps_tree_expand: children of depth `depth`'s rows (dynamic IID tree).  `draft` = the
+    pps_draft_list (IID) outputs of those rows; writes nxt = dict(key, ctx, pos, k) of the next
+    depth's rows, child_node and nodes = dict(key, ctx, pos) in place."""
+    n_seq = nxt["k"].numel() // K
+    code = lib().pps_tree_expand(n_seq, int(K), int(gamma), int(depth), _ptr(draft["tok"]), _ptr(draft["mult"]),
+                                 _ptr(draft["ndist"]), _ids(rows_key, rows_ctx, rows_pos), _ptr(row_k),
+                                 _ptr(nxt["key"]), _ptr(nxt["ctx"]), _ptr(nxt["pos"]), _ptr(nxt["k"]),
+                                 _ptr(child_node), _ptr(nodes["key"]), _ptr(nodes["ctx"]), _ptr(nodes["pos"]),
+                                 _stream(stream))
+    _check("pps_tree_expand", code)
 
 
 SCORE_AARONSON, SCORE_U, SCORE_LI, SCORE_POWER_LAW = 0, 1, 2, 3
