@@ -127,3 +127,18 @@ def test_detect_validates_kind_and_parameter():
     for bad in (0.0, 1.5, float("nan")):
         assert detect(pps.SCORE_POWER_LAW, bad) == pps.ERR_INVALID_ARG
     assert detect(pps.SCORE_AARONSON, 0.0, out_sum=None) == pps.ERR_INVALID_ARG  # p-values need the sums
+
+
+def test_tree_expand_validates_shape_arguments():
+    L = pps.lib()
+    fake = ctypes.c_void_p(256)
+    ids = pps.RowIds(256, 256, 256)
+
+    def expand(n_seq=4, K=4, gamma=3, depth=0, tok=fake):
+        return L.pps_tree_expand(n_seq, K, gamma, depth, tok, fake, fake, ids, fake, fake, fake, fake, fake, fake,
+                                 fake, fake, fake, None)
+
+    for kw in (dict(K=0), dict(K=33), dict(gamma=0), dict(gamma=65), dict(depth=-1), dict(depth=3), dict(n_seq=-1),
+               dict(tok=None)):
+        assert expand(**kw) == pps.ERR_INVALID_ARG, kw
+    assert expand(n_seq=0) == pps.OK
