@@ -228,6 +228,9 @@ def main():
     if args.workload == "detector":
         run_detector(args, rank, world, dev)
         return
+    if args.workload == "dynamic":
+        run_dynamic(args, rank, world, dev)
+        return
     wl = synth.make_workload(args.workload, device=dev, n_seq=args.n_seq)
     t = wl.tree
     g = lambda x: torch.as_tensor(np.asarray(x)).to(dev).contiguous()
@@ -492,6 +495,84 @@ def run_detector(args, rank, world, dev):
                           "anlppt_watermarked": float(np.mean(-wm / 128.0)),
                           "anlppt_null": float(np.mean(-null / 128.0)), "segments": int(n_seg)},
             "gpu_launches": 2 * args.steps,
+        }))
+
+
+def run_dynamic(args, rank, world, dev):
+    """The dynamic IID draft tree (the paper's multi-draft tree: every context draws its
+    multiplicity nu(c) of i.i.d. samples, K paths per depth): per step gamma pps_draft_list (IID)
+    + pps_tree_expand calls, then pps_verify_tree over every node slot.  B=64, V=128256, K=8,
+    gamma=5 (fixed capacity 41 node slots and 33 draft rows per sequence), bf16 logits: target
+    rows as zipf_k8, drafts = the node's target row + N(0,1) (the drafter's outputs are inputs)."""
+    from paper_2609_21858_gb300 import pps, synth, tree
+    n_seq, V, K, gamma = args.n_seq or 64, 128256, 8, 5
+    g = torch.Generator(device=dev)
+    g.manual_seed(2)
+    b = tree.TreeBuilder(n_seq, K, gamma, dev)
+    p = synth._zipf(g, b.n_nodes, V, 1.0, True, dev).to(torch.bfloat16)
+    N1 = 1 + K * gamma
+    q = []
+    for d in range(gamma):
+        off = 0 if d == 0 else 1 + (d - 1) * K
+        w = 1 if d == 0 else K
+        slots = (torch.arange(n_seq, device=dev)[:, None] * N1 + off + torch.arange(w, device=dev)[None, :]).ravel()
+        q.append((p[slots].float() + torch.randn(slots.numel(), V, generator=g, device=dev)).to(torch.bfloat16))
+    rk = torch.as_tensor(synth.splitmix64_stream(20, 2 * n_seq).view(np.int64), device=dev)
+    root_key, root_ctx = rk[:n_seq], rk[n_seq:]
+    root_pos = torch.arange(n_seq, dtype=torch.int32, device=dev) * 0 + 100
+    ws_v = pps.workspace(b.n_nodes, n_seq, dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    W = gamma + 1
+    vout = dict(winner=torch.empty(b.n_nodes, dtype=torch.int32, device=dev),
+                word=torch.empty(b.n_nodes, dtype=torch.int32, device=dev),
+                accept_len=torch.empty(n_seq, dtype=torch.int32, device=dev),
+                n_emitted=torch.empty(n_seq, dtype=torch.int32, device=dev),
+                emitted=torch.empty(n_seq, W, dtype=torch.int32, device=dev),
+                score=torch.empty(n_seq, W, dtype=torch.float32, device=dev),
+                score_sum=torch.empty(n_seq, dtype=torch.float64, device=dev))
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        b.run(root_key, root_ctx, root_pos, lambda d, *_: q[d], stream=stream)
+        b.verify(p, ws=ws_v, out=vout, status=status, stream=stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    assert int(status.item()) == 0, f"status flags {int(status.item())}"
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk = Clocks(dev.index or 0)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    clk.start()
+    time.sleep(0.3)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = clk.stop()
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
+    rows = b.n_draft + b.n_nodes
+    nbytes = rows * V * 2
+    peak, peak_kind = _peaks()
+    gbs = nbytes / (ms / 1e3) / 1e9
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": rows * world / (ms / 1e3), "unit": "rows/s", "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded Zipf-rank logits; no model, no dataset)",
+            "config": {"workload": f"dynamic IID tree: B={n_seq}, V={V}, K={K}, gamma={gamma}, "
+                                   f"{b.n_nodes} node slots + {b.n_draft} draft rows per step",
+                       "rows_per_step": rows, "l2": f"inputs ({nbytes / 1e9:.2f} GB) larger than L2, no flush",
+                       "parallelism": f"replicas x{world}"},
+            "gb_per_s": gbs,
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
+                         "traffic": None, "peak_kind": peak_kind, "algorithmic_bytes": nbytes},
+            "gpu_launches": args.steps * (2 * gamma + 1), "clocks": clocks,
+            "mean_accept_len": float(vout["accept_len"].float().mean().item()),
+            "mean_draft_nodes_per_seq": float((b.row_k[:b.n_draft] > 0).sum().item()) / n_seq,
         }))
 
 

@@ -206,16 +206,17 @@ pps_status pps_verify_tree_trunc(const void* p_logits, pps_dtype dtype, int64_t 
  * Fixed-capacity layout (static; nothing else is reallocated per depth):
  *   nodes      N1 = 1 + K*gamma per sequence; node (b, d, i) =
  *              b*N1 + (d == 0 ? 0 : 1 + (d-1)*K + i); seq_off[b] = b*N1
- *   draft rows R1 = 1 + K*(gamma-1) per sequence; the draft row of node
- *              (b, d, i), d < gamma, is b*R1 + the same offset (node_draft_row)
- *   depth rows the rows of depth d, w_d = (d == 0 ? 1 : K) per sequence, row
- *              (b, i) = b*w_d + i: the rows one pps_draft_list call takes
- * Inputs (depth d's rows, [n_seq*w_d]): draft_tok, draft_mult, draft_ndistinct
+ *   draft rows depth-major, n_seq*(1 + K*(gamma-1)) in all: depth d's rows
+ *              start at D_d = n_seq*(d == 0 ? 0 : 1 + (d-1)*K), w_d = (d == 0 ?
+ *              1 : K) per sequence, and node (b, d, i), d < gamma, owns draft
+ *              row D_d + b*w_d + i (node_draft_row).  A depth's rows are the
+ *              contiguous rows one pps_draft_list call takes.
+ * Inputs (depth d's rows (b, i) = b*w_d + i, [n_seq*w_d]): draft_tok, draft_mult, draft_ndistinct
  * (pps_draft_list outputs, stride K), rows (their identities), row_k (nu; 0 =
  * an absent node, whose list is ignored).
  * Outputs: next_key, next_ctx, next_pos, next_k [n_seq*K]: identities and nu
  * of depth d+1's rows in child order (nu = 0 past the last child);
- * child_node [n_seq*R1, K]: the rows of depth d get their children's node
+ * child_node [all draft rows, K]: the rows of depth d get their children's node
  * indices (-1 past ndistinct); node_key, node_ctx, node_pos [n_seq*N1]:
  * identities of depth d+1's nodes.  All device pointers.
  */

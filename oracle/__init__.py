@@ -275,7 +275,8 @@ def child_label(parent: int, token: int) -> int:
 
 def tree_expand(n_seq, K, gamma, depth, d, key, ctx, pos, row_k, tree):
     """One depth of the dynamic IID tree; `d` = draft_rows(IID) output of this depth's rows,
-    `tree` = dict(child_node [n_seq*R1, K], node_key/ctx/pos [n_seq*N1]) updated in place.
+    `tree` = dict(child_node [draft rows, K] (depth-major rows), node_key/ctx/pos [n_seq*N1]),
+    updated in place.
     Returns (next_key, next_ctx, next_pos, next_k) of depth+1's rows."""
     n = n_seq * K
     nk, nc = np.zeros(n, np.uint64), np.zeros(n, np.uint64)

@@ -550,9 +550,10 @@ uint64_t orc_child_label(uint64_t parent, int32_t token)
 }
 
 /* Fixed-capacity layout, per sequence b: node (d, i) = b*N1 + (d == 0 ? 0 :
- * 1 + (d-1)*K + i), N1 = 1 + K*gamma; draft row (d, i) (d < gamma) = b*R1 +
- * the same offset, R1 = 1 + K*(gamma-1).  Rows of depth d: w_d = (d == 0 ? 1 : K)
- * per sequence, row (b, i) of the depth = b*w_d + i.  A row with k = 0 is an
+ * 1 + (d-1)*K + i), N1 = 1 + K*gamma.  Draft rows depth-major: depth d's rows
+ * start at D_d = n_seq*(d == 0 ? 0 : 1 + (d-1)*K); w_d = (d == 0 ? 1 : K) per
+ * sequence; row (b, i) of the depth = b*w_d + i is draft row D_d + b*w_d + i,
+ * owned by node (b, d, i).  A row with k = 0 is an
  * absent node.  For every present row (b, i) of depth d, its distinct draft
  * labels m < ndist (in list order) get child slots j = 0, 1, ... in row order
  * then list order; child j: ids (key, label(child), pos + 1), k = mult, its
@@ -564,15 +565,15 @@ void orc_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t depth, con
                      uint32_t* next_pos, int32_t* next_k, int32_t* child_node, uint64_t* node_key,
                      uint64_t* node_ctx, uint32_t* node_pos)
 {
-    int64_t N1 = 1 + (int64_t)K * gamma, R1 = 1 + (int64_t)K * (gamma - 1);
+    int64_t N1 = 1 + (int64_t)K * gamma;
     int32_t w = depth == 0 ? 1 : K;
-    int64_t off_d = depth == 0 ? 0 : 1 + (int64_t)(depth - 1) * K;   /* offset of depth d in a sequence */
-    int64_t off_n = 1 + (int64_t)depth * K;                          /* offset of depth d+1 */
+    int64_t D_d = depth == 0 ? 0 : (int64_t)n_seq * (1 + (int64_t)(depth - 1) * K);  /* first draft row of depth d */
+    int64_t off_n = 1 + (int64_t)depth * K;                                          /* node offset of depth d+1 */
     for (int32_t b = 0; b < n_seq; ++b) {
         int32_t j = 0;
         for (int32_t i = 0; i < w; ++i) {
             int64_t r = (int64_t)b * w + i;
-            int64_t dr = (int64_t)b * R1 + off_d + i;
+            int64_t dr = D_d + r;
             for (int32_t m = 0; m < K; ++m) child_node[dr * K + m] = -1;
             if (row_k[r] <= 0) continue;
             for (int32_t m = 0; m < ndist[r]; ++m) {

@@ -237,9 +237,10 @@ __global__ void tree_expand_kernel(int32_t n_seq, int32_t K, int32_t gamma, int3
     const int lane = threadIdx.x & 31;
     const int64_t b = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (b >= n_seq) return;
-    const int64_t N1 = 1 + (int64_t)K * gamma, R1 = 1 + (int64_t)K * (gamma - 1);
+    const int64_t N1 = 1 + (int64_t)K * gamma;
     const int w = depth == 0 ? 1 : K;
-    const int64_t off_d = depth == 0 ? 0 : 1 + (int64_t)(depth - 1) * K, off_n = 1 + (int64_t)depth * K;
+    // draft rows are numbered depth-major: depth d's rows start at D_d = n_seq (1 + (d-1) K)
+    const int64_t D_d = depth == 0 ? 0 : (int64_t)n_seq * (1 + (int64_t)(depth - 1) * K), off_n = 1 + (int64_t)depth * K;
     const int64_t r = b * w + lane;
     const bool row = lane < w;
     int nd = 0;
@@ -253,7 +254,7 @@ __global__ void tree_expand_kernel(int32_t n_seq, int32_t K, int32_t gamma, int3
     const int total = min(__shfl_sync(FULL, j0, 31), K);
     j0 -= nd;
     if (row) {
-        const int64_t dr = b * R1 + off_d + lane;
+        const int64_t dr = D_d + b * w + lane;
         for (int m = 0; m < K; ++m) {
             int node = -1;
             const int j = j0 + m;

@@ -5,16 +5,15 @@ mode); every distinct label u becomes a child c||u that draws nu(c||u) = its
 multiplicity, so a sequence keeps K draft paths at every depth.  The drafter
 is the caller's: `draft_logits(depth, key, ctx, pos)` returns the logits of a
 depth's rows (a model forward on those contexts).  The tree lives in the
-fixed-capacity layout of pps_tree_expand (include/pps.h), so its node and
-draft-row numbering, seq_off and node_draft_row never change; the target
-model then scores every node slot and pps_verify_tree walks the tree.
+fixed-capacity layout of pps_tree_expand (include/pps.h): nodes
+sequence-major (so seq_off and node_draft_row never change), draft rows
+depth-major (so each depth's lists are written in place by one call).  The
+target model then scores every node slot and pps_verify_tree walks the tree.
 
 This module only allocates and sequences library calls; all arithmetic runs
 in libpps.
 """
 from __future__ import annotations
-
-from dataclasses import dataclass
 
 import numpy as np
 import torch
@@ -22,79 +21,73 @@ import torch
 from . import pps
 
 
-@dataclass
-class IIDTree:
-    n_seq: int
-    K: int
-    gamma: int
-    node_key: torch.Tensor        # [n_seq*N1] identities of every node slot
-    node_ctx: torch.Tensor
-    node_pos: torch.Tensor
-    seq_off: torch.Tensor         # [n_seq+1]
-    node_draft_row: torch.Tensor  # [n_seq*N1]
-    draft_tok: torch.Tensor       # [n_seq*R1, K] per draft row, in the layout's row order
-    draft_mult: torch.Tensor
-    draft_ndist: torch.Tensor     # [n_seq*R1]
-    child_node: torch.Tensor      # [n_seq*R1, K]
-    draft_k: torch.Tensor         # [n_seq*R1] nu of every draft row (0 = absent node)
+class TreeBuilder:
+    """Buffers for the dynamic IID trees of n_seq sequences (reused by every `run`)."""
 
-    @property
-    def nodes_per_seq(self) -> int:
-        return 1 + self.K * self.gamma
+    def __init__(self, n_seq: int, K: int, gamma: int, device="cuda"):
+        self.n_seq, self.K, self.gamma = n_seq, K, gamma
+        dev = torch.device(device)
+        N1 = 1 + K * gamma
+        self.n_nodes = n_seq * N1
+        self.n_draft = n_seq * (1 + K * (gamma - 1))
+        self.depth_start = [0] + [n_seq * (1 + (d - 1) * K) for d in range(1, gamma + 1)]
+        self.width = [1] + [K] * gamma
+        i32, i64 = dict(dtype=torch.int32, device=dev), dict(dtype=torch.int64, device=dev)
+        self.seq_off = torch.arange(n_seq + 1, **i32) * N1
+        ndr = np.full((n_seq, N1), -1, np.int64)
+        for d in range(gamma):
+            off = 0 if d == 0 else 1 + (d - 1) * K
+            w = self.width[d]
+            ndr[:, off:off + w] = self.depth_start[d] + np.arange(n_seq)[:, None] * w + np.arange(w)[None, :]
+        self.node_draft_row = torch.as_tensor(ndr.ravel().astype(np.int32), device=dev)
+        self.node_key = torch.zeros(self.n_nodes, **i64)
+        self.node_ctx = torch.zeros(self.n_nodes, **i64)
+        self.node_pos = torch.zeros(self.n_nodes, **i32)
+        self.draft_tok = torch.full((self.n_draft, K), -1, **i32)
+        self.draft_mult = torch.zeros((self.n_draft, K), **i32)
+        self.draft_ndist = torch.zeros(self.n_draft, **i32)
+        self.child_node = torch.full((self.n_draft, K), -1, **i32)
+        # identities and nu of every depth's rows, depth-major like the draft rows
+        self.row_key = torch.zeros(self.depth_start[gamma] + n_seq * K, **i64)
+        self.row_ctx = torch.zeros_like(self.row_key)
+        self.row_pos = torch.zeros(self.row_key.numel(), **i32)
+        self.row_k = torch.zeros(self.row_key.numel(), **i32)
+        self.roots = self.seq_off[:-1].long()
+        self.ws = pps.workspace(n_seq * K, 0, dev)
 
-    @property
-    def rows_per_seq(self) -> int:
-        return 1 + self.K * (self.gamma - 1)
+    def rows(self, d: int) -> slice:
+        return slice(self.depth_start[d], self.depth_start[d] + self.n_seq * self.width[d])
+
+    def run(self, root_key, root_ctx, root_pos, draft_logits, temperature: float = 1.0, top_k: int = 0,
+            top_p: float = 1.0, stream=None):
+        """Draft the trees: per depth one pps_draft_list (IID) and one pps_tree_expand."""
+        K = self.K
+        s0 = self.rows(0)
+        self.row_key[s0], self.row_ctx[s0], self.row_pos[s0] = root_key, root_ctx, root_pos
+        self.row_k[s0] = K
+        self.node_key[self.roots], self.node_ctx[self.roots], self.node_pos[self.roots] = root_key, root_ctx, root_pos
+        for d in range(self.gamma):
+            s, sn = self.rows(d), self.rows(d + 1)
+            key, ctx, pos, k = self.row_key[s], self.row_ctx[s], self.row_pos[s], self.row_k[s]
+            out = dict(tok=self.draft_tok[s], key=None, mult=self.draft_mult[s], ndist=self.draft_ndist[s],
+                       samples=None)
+            pps.draft_list(draft_logits(d, key, ctx, pos), key, ctx, pos, K, row_k=k, mode=pps.IID,
+                           temperature=temperature, ws=self.ws, out=out, top_k=top_k, top_p=top_p, stream=stream)
+            nxt = dict(key=self.row_key[sn], ctx=self.row_ctx[sn], pos=self.row_pos[sn], k=self.row_k[sn])
+            pps.tree_expand(K, self.gamma, d, out, key, ctx, pos, k, nxt, self.child_node,
+                            dict(key=self.node_key, ctx=self.node_ctx, pos=self.node_pos), stream=stream)
+        return self
+
+    def verify(self, p_logits, temperature: float = 1.0, top_k: int = 0, top_p: float = 1.0, ws=None, out=None,
+               status=None, stream=None):
+        """The target race over every node slot and the walk (pps_verify_tree)."""
+        return pps.verify_tree(p_logits, self.node_key, self.node_ctx, self.node_pos, self.gamma, self.seq_off,
+                               self.node_draft_row, self.draft_tok, self.draft_ndist, self.child_node,
+                               temperature=temperature, ws=ws, out=out, status=status, stream=stream, top_k=top_k,
+                               top_p=top_p)
 
 
-def layout(n_seq: int, K: int, gamma: int, device):
-    """seq_off and node_draft_row of the fixed-capacity layout, and the draft-row slots of each depth."""
-    N1, R1 = 1 + K * gamma, 1 + K * (gamma - 1)
-    seq_off = torch.arange(n_seq + 1, dtype=torch.int32, device=device) * N1
-    ndr = np.full(N1, -1, np.int64)
-    ndr[:R1] = np.arange(R1)  # node offset o < R1 (depth < gamma) owns draft row offset o
-    ndr = np.concatenate([np.where(ndr >= 0, ndr + b * R1, -1) for b in range(n_seq)])
-    depth_rows = []
-    for d in range(gamma):
-        off, w = (0, 1) if d == 0 else (1 + (d - 1) * K, K)
-        depth_rows.append(torch.as_tensor((np.arange(n_seq)[:, None] * R1 + off + np.arange(w)[None, :]).ravel(),
-                                          device=device))
-    return seq_off, torch.as_tensor(ndr.astype(np.int32), device=device), depth_rows
-
-
-def build(root_key, root_ctx, root_pos, K: int, gamma: int, draft_logits, temperature: float = 1.0,
-          top_k: int = 0, top_p: float = 1.0, stream=None) -> IIDTree:
-    """Draft a dynamic IID tree of depth gamma for every root context (tensors of n_seq)."""
-    dev = root_key.device
-    n_seq = root_key.numel()
-    N1, R1 = 1 + K * gamma, 1 + K * (gamma - 1)
-    seq_off, ndr, depth_rows = layout(n_seq, K, gamma, dev)
-    i64 = dict(dtype=torch.int64, device=dev)
-    t = IIDTree(n_seq, K, gamma,
-                node_key=torch.zeros(n_seq * N1, **i64), node_ctx=torch.zeros(n_seq * N1, **i64),
-                node_pos=torch.zeros(n_seq * N1, dtype=torch.int32, device=dev), seq_off=seq_off,
-                node_draft_row=ndr,
-                draft_tok=torch.full((n_seq * R1, K), -1, dtype=torch.int32, device=dev),
-                draft_mult=torch.zeros((n_seq * R1, K), dtype=torch.int32, device=dev),
-                draft_ndist=torch.zeros(n_seq * R1, dtype=torch.int32, device=dev),
-                child_node=torch.full((n_seq * R1, K), -1, dtype=torch.int32, device=dev),
-                draft_k=torch.zeros(n_seq * R1, dtype=torch.int32, device=dev))
-    roots = seq_off[:-1].long()
-    t.node_key[roots], t.node_ctx[roots], t.node_pos[roots] = root_key, root_ctx, root_pos
-    key, ctx, pos = root_key.contiguous(), root_ctx.contiguous(), root_pos.contiguous()
-    k = torch.full((n_seq,), K, dtype=torch.int32, device=dev)
-    for d in range(gamma):
-        logits = draft_logits(d, key, ctx, pos)
-        out = pps.draft_list(logits, key, ctx, pos, K, row_k=k, mode=pps.IID, temperature=temperature,
-                             top_k=top_k, top_p=top_p, stream=stream)
-        rows = depth_rows[d]
-        t.draft_tok[rows], t.draft_mult[rows], t.draft_ndist[rows], t.draft_k[rows] = (
-            out["tok"], out["mult"], out["ndist"], k)
-        # children of this depth (the leaves too: the target model scores them)
-        nxt = dict(key=torch.empty(n_seq * K, **i64), ctx=torch.empty(n_seq * K, **i64),
-                   pos=torch.empty(n_seq * K, dtype=torch.int32, device=dev),
-                   k=torch.empty(n_seq * K, dtype=torch.int32, device=dev))
-        pps.tree_expand(K, gamma, d, out, key, ctx, pos, k, nxt, t.child_node,
-                        dict(key=t.node_key, ctx=t.node_ctx, pos=t.node_pos), stream=stream)
-        key, ctx, pos, k = nxt["key"], nxt["ctx"], nxt["pos"], nxt["k"]
-    return t
+def build(root_key, root_ctx, root_pos, K: int, gamma: int, draft_logits, **kw) -> TreeBuilder:
+    """Draft dynamic IID trees for the root contexts (n_seq tensors) with fresh buffers."""
+    return TreeBuilder(root_key.numel(), K, gamma, root_key.device).run(root_key, root_ctx, root_pos, draft_logits,
+                                                                        **kw)

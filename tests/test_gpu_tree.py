@@ -42,10 +42,9 @@ def test_dynamic_tree_matches_the_oracle(K, gamma, V, dtype):
 
     t = tree.build(key, ctx, pos, K, gamma, draft_logits)
     torch.cuda.synchronize()
-    N1, R1 = t.nodes_per_seq, t.rows_per_seq
-    _, _, depth_rows = tree.layout(n_seq, K, gamma, "cpu")
+    N1 = 1 + K * gamma
     # oracle, depth by depth, expanding the GPU's own lists
-    otree = dict(child_node=np.full((n_seq * R1, K), -1, np.int32), node_key=np.zeros(n_seq * N1, np.uint64),
+    otree = dict(child_node=np.full((t.n_draft, K), -1, np.int32), node_key=np.zeros(n_seq * N1, np.uint64),
                  node_ctx=np.zeros(n_seq * N1, np.uint64), node_pos=np.zeros(n_seq * N1, np.uint32))
     roots = np.arange(n_seq) * N1
     otree["node_key"][roots], otree["node_ctx"][roots], otree["node_pos"][roots] = (
@@ -57,10 +56,10 @@ def test_dynamic_tree_matches_the_oracle(K, gamma, V, dtype):
         assert np.array_equal(gk, okey) and np.array_equal(gc, octx) and np.array_equal(gp, opos)
         lgo = torch.as_tensor(lg).to(dtype).float().numpy()
         od = oracle.draft_rows(lgo, okey, octx, opos, K, row_k=np.maximum(k, 1), mode=oracle.IID)
-        rows = depth_rows[d].numpy()
+        rows = t.rows(d)
         gd = dict(tok=t.draft_tok[rows].cpu().numpy(), mult=t.draft_mult[rows].cpu().numpy(),
                   ndist=t.draft_ndist[rows].cpu().numpy(), samples=None, key=None)
-        assert np.array_equal(t.draft_k[rows].cpu().numpy(), k)
+        assert np.array_equal(t.row_k[rows].cpu().numpy(), k)
         present = k > 0
         sub = lambda x: x[present]
         compare_draft({kk: (sub(v) if v is not None else None) for kk, v in gd.items()},
@@ -73,8 +72,7 @@ def test_dynamic_tree_matches_the_oracle(K, gamma, V, dtype):
     # target race over every node slot, then the walk
     plg = synth.label_logits(u64(t.node_ctx), V, seed=11)
     p = torch.as_tensor(plg).to(dtype).cuda()
-    v = pps.verify_tree(p, t.node_key, t.node_ctx, t.node_pos, gamma, t.seq_off, t.node_draft_row, t.draft_tok,
-                        t.draft_ndist, t.child_node)
+    v = t.verify(p)
     torch.cuda.synchronize()
     win, wd, _, mg = oracle.target_rows(torch.as_tensor(plg).to(dtype).float().numpy(), u64(t.node_key),
                                         u64(t.node_ctx), t.node_pos.cpu().numpy().view(np.uint32))

@@ -68,11 +68,11 @@ def test_dynamic_tree_keeps_k_paths_and_one_parent_per_node():
         n_children = (nd * present).sum(1)
         assert np.all(n_children <= K)
         nxt_k = depths[d + 1]["k"].reshape(n_seq, K) if d + 1 < gamma else None
+        D_d = 0 if d == 0 else n_seq * (1 + (d - 1) * K)
         for b in range(n_seq):
-            off_d = 0 if d == 0 else 1 + (d - 1) * K
             seen = []
             for i in range(w):
-                dr = b * R1 + off_d + i
+                dr = D_d + b * w + i
                 for m in range(K):
                     c = tree["child_node"][dr, m]
                     if present[b, i] and m < nd[b, i]:
