@@ -92,6 +92,16 @@ def lib():
             L.orc_tree_expand.argtypes = [i32, i32, i32, i32, i32p, i32p, i32p, u64p, u64p, u32p, i32p,
                                           u64p, u64p, u32p, i32p, i32p, u64p, u64p, u32p]
             L.orc_tree_expand.restype = None
+            L.orc_block_j.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32, i64, i32]
+            L.orc_block_j.restype = i32
+            L.orc_block_e.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32, i64, i32, i32]
+            L.orc_block_e.restype = f64
+            L.orc_block_draft_rows.argtypes = [f32p, i64, i64, i64, f64, u64p, u64p, u32p, i32p, i32, i32p, f64p,
+                                               f64p]
+            L.orc_block_draft_rows.restype = None
+            L.orc_hetero_rows.argtypes = [f32p, f32p, i64, i32, i64, f64, u64p, u64p, u32p, i32p, i32p, i32p,
+                                          u32p, i32p, f64p, f64p]
+            L.orc_hetero_rows.restype = None
             L.orc_truncate_rows.argtypes = [f32p, i64, i64, i64, f64, i32, f64, f32p, f64p]
             L.orc_truncate_rows.restype = None
             L.orc_set_threads.argtypes = [ctypes.c_int]
@@ -290,3 +300,45 @@ def tree_expand(n_seq, K, gamma, depth, d, key, ctx, pos, row_k, tree):
                           _ptr(tree["child_node"], ctypes.c_int32), _ptr(tree["node_key"], ctypes.c_uint64),
                           _ptr(tree["node_ctx"], ctypes.c_uint64), _ptr(tree["node_pos"], ctypes.c_uint32))
     return nk, nc, npos, nkk
+
+
+def block_j(key: int, ctx: int, pos: int, i: int, B: int) -> int:
+    """Block J_i of token i's smallest augmented arrival."""
+    return int(lib().orc_block_j(key, ctx, pos, int(i), int(B)))
+
+
+def block_e(key: int, ctx: int, pos: int, i: int, b: int, B: int) -> float:
+    """First arrival E_(i,b) of augmented point (i, b)."""
+    return float(lib().orc_block_e(key, ctx, pos, int(i), int(b), int(B)))
+
+
+def block_draft_rows(q_logits, key, ctx, pos, block, B: int, T: float = 1.0):
+    """Proposal races per row: (x, key, margin)."""
+    q = _c(q_logits, np.float32)
+    n, V = q.shape
+    key, ctx, pos, block = _c(key, np.uint64), _c(ctx, np.uint64), _c(pos, np.uint32), _c(block, np.int32)
+    x = np.zeros(n, np.int32)
+    k, m = np.zeros(n, np.float64), np.zeros(n, np.float64)
+    lib().orc_block_draft_rows(_ptr(q, ctypes.c_float), n, V, V, float(T), _ptr(key, ctypes.c_uint64),
+                               _ptr(ctx, ctypes.c_uint64), _ptr(pos, ctypes.c_uint32), _ptr(block, ctypes.c_int32),
+                               int(B), _ptr(x, ctypes.c_int32), _ptr(k, ctypes.c_double), _ptr(m, ctypes.c_double))
+    return x, k, m
+
+
+def hetero_rows(p_logits, q_logits, key, ctx, pos, B: int, T: float = 1.0):
+    """One step with B non-identical proposals per context:
+    dict(x [n, B], y, j, word, accept, margin_y, margin_x [n, B])."""
+    p = _c(p_logits, np.float32)
+    n, V = p.shape
+    q = _c(q_logits, np.float32).reshape(n * B, V)
+    key, ctx, pos = _c(key, np.uint64), _c(ctx, np.uint64), _c(pos, np.uint32)
+    x = np.zeros(n * B, np.int32)
+    y, j, acc = np.zeros(n, np.int32), np.zeros(n, np.int32), np.zeros(n, np.int32)
+    word = np.zeros(n, np.uint32)
+    my, mx = np.zeros(n, np.float64), np.zeros(n * B, np.float64)
+    lib().orc_hetero_rows(_ptr(p, ctypes.c_float), _ptr(q, ctypes.c_float), n, int(B), V, float(T),
+                          _ptr(key, ctypes.c_uint64), _ptr(ctx, ctypes.c_uint64), _ptr(pos, ctypes.c_uint32),
+                          _ptr(x, ctypes.c_int32), _ptr(y, ctypes.c_int32), _ptr(j, ctypes.c_int32),
+                          _ptr(word, ctypes.c_uint32), _ptr(acc, ctypes.c_int32), _ptr(my, ctypes.c_double),
+                          _ptr(mx, ctypes.c_double))
+    return dict(x=x.reshape(n, B), y=y, j=j, word=word, accept=acc, margin_y=my, margin_x=mx.reshape(n, B))

@@ -61,6 +61,12 @@
  *                      output function of label(c) ^ ((u + 1) * 0x9E3779B97F4A7C15)
  *                      (a reading: the paper leaves the labeler open),
  *                      position + 1, same key.
+ *   orc_hetero_rows    non-identical proposals Q_0..Q_{B-1} (App. A, the
+ *                      proposition on heterogeneous proposals): one Poisson
+ *                      process on the augmented vocabulary V x [B]; proposal b
+ *                      races Q_b over block b, the target races P(i)/B over all
+ *                      (i, b); Y is accepted iff it equals some X^(b).
+ *   orc_block_draft_rows  proposal b's race alone, per row (tree drafting).
  *   orc_truncate_rows  the logit processing of the experiments (Sec. 6 setup:
  *                      top-k = 50, top-p = 1; truncation leaves a support of at
  *                      most k tokens, Sec. 4.2): tokens outside the top-k /
@@ -597,6 +603,114 @@ void orc_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t depth, con
             next_pos[q] = 0;
             next_k[q] = 0;
         }
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* non-identical proposals (App. A, heterogeneous proposals)           */
+/* ------------------------------------------------------------------ */
+
+/* The augmented race lives on V x [B] (blocks b = 0..B-1).  Its first
+ * arrivals E_(i,b) are B independent Exp(1) per token, generated from three
+ * keyed words by competing exponentials: the minimum of B iid Exp(1) is
+ * Exp(B), it sits in a uniform block independent of its value, and the other
+ * B-1 exceed it by independent Exp(1) amounts.  So, with E'_i the token's
+ * usual first arrival,
+ *     J_i     = floor(B * word(key ^ kBlockJ, i) / 2^32),
+ *     E_(i,b) = E'_i / B                                      for b = J_i,
+ *     E_(i,b) = E'_i / B + exp1(word(key ^ (b+1) kBlockF, i)) otherwise.
+ * B = 1 gives E_(i,0) = E'_i, the identical-proposal source. */
+#define ORC_BLOCK_J 0x3C6EF372FE94F82Bull
+#define ORC_BLOCK_F 0xBB67AE8584CAA73Bull
+
+int32_t orc_block_j(uint64_t key, uint64_t ctx, uint32_t pos, int64_t i, int32_t B)
+{
+    uint32_t w = orc_word(key ^ ORC_BLOCK_J, ctx, pos, i, 1);
+    return (int32_t)(((uint64_t)w * (uint64_t)(uint32_t)B) >> 32);
+}
+
+double orc_block_e(uint64_t key, uint64_t ctx, uint32_t pos, int64_t i, int32_t b, int32_t B)
+{
+    double e = orc_exp1(orc_word(key, ctx, pos, i, 1)) / (double)B;
+    if (b != orc_block_j(key, ctx, pos, i, B))
+        e += orc_exp1(orc_word(key ^ ((uint64_t)(uint32_t)(b + 1) * ORC_BLOCK_F), ctx, pos, i, 1));
+    return e;
+}
+
+/* Proposal b's sample at each row: X = argmin_i ln E_(i,b) - q_i/T over block
+ * b (the race of Q~_b, which puts no mass outside block b); ties to the
+ * smaller token.  x = -1 when no token is usable; margin = second-smallest
+ * minus smallest key (+inf with fewer than two usable tokens). */
+void orc_block_draft_rows(const float* q, int64_t n_rows, int64_t V, int64_t stride, double T, const uint64_t* key,
+                          const uint64_t* ctx, const uint32_t* pos, const int32_t* block, int32_t B, int32_t* x,
+                          double* key_out, double* margin)
+{
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t r = 0; r < n_rows; ++r) {
+        double best = INFINITY, second = INFINITY;
+        int64_t bi = -1;
+        for (int64_t i = 0; i < V; ++i) {
+            double l = (double)q[r * stride + i];
+            if (isnan(l) || l == -INFINITY) continue;
+            double k = log(orc_block_e(key[r], ctx[r], pos[r], i, block[r], B)) - l / T;
+            if (bi < 0 || k < best) { second = best; best = k; bi = i; }
+            else if (k < second) second = k;
+        }
+        x[r] = (int32_t)bi;
+        if (key_out) key_out[r] = bi >= 0 ? best : INFINITY;
+        if (margin) margin[r] = bi >= 0 && second < INFINITY ? second - best : INFINITY;
+    }
+}
+
+/* One step with B proposals at each context c (rows p[c], q[c*B + b]):
+ *   x[c*B + b]  = proposal b's sample (orc_block_draft_rows);
+ *   (y[c], j[c]) = argmin over (i, b) of E_(i,b) / P~(i,b), P~(i,b) = p_i / B,
+ *                  i.e. of ln E_(i,b) - p_i/T (the common ln B - ln Z drops out);
+ *                  ties to the smaller i, then b;
+ *   word[c]     = the watermark word of y: its usual first-arrival word, whose
+ *                  E'_y = B E_(y,j) is the pivot a detector sees;
+ *   accept[c]   = [y in {x[c*B + b]}];  margin_y = the target's key gap. */
+void orc_hetero_rows(const float* p, const float* q, int64_t n_ctx, int32_t B, int64_t V, double T,
+                     const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int32_t* x, int32_t* y,
+                     int32_t* j, uint32_t* word, int32_t* accept, double* margin_y, double* margin_x)
+{
+    int64_t nr = n_ctx * B;
+    uint64_t* rk = malloc((size_t)nr * sizeof(uint64_t));
+    uint64_t* rc = malloc((size_t)nr * sizeof(uint64_t));
+    uint32_t* rp = malloc((size_t)nr * sizeof(uint32_t));
+    int32_t* rb = malloc((size_t)nr * sizeof(int32_t));
+    for (int64_t r = 0; r < nr; ++r) {
+        rk[r] = key[r / B];
+        rc[r] = ctx[r / B];
+        rp[r] = pos[r / B];
+        rb[r] = (int32_t)(r % B);
+    }
+    orc_block_draft_rows(q, nr, V, V, T, rk, rc, rp, rb, B, x, NULL, margin_x);
+    free(rk);
+    free(rc);
+    free(rp);
+    free(rb);
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t c = 0; c < n_ctx; ++c) {
+        double best = INFINITY, second = INFINITY;
+        int64_t bi = -1;
+        int32_t bb = -1;
+        for (int64_t i = 0; i < V; ++i) {
+            double l = (double)p[c * V + i];
+            if (isnan(l) || l == -INFINITY) continue;
+            for (int32_t b = 0; b < B; ++b) {
+                double k = log(orc_block_e(key[c], ctx[c], pos[c], i, b, B)) - l / T;
+                if (bi < 0 || k < best) { second = best; best = k; bi = i; bb = b; }
+                else if (k < second) second = k;
+            }
+        }
+        y[c] = (int32_t)bi;
+        j[c] = bb;
+        word[c] = bi >= 0 ? orc_word(key[c], ctx[c], pos[c], bi, 1) : 0u;
+        int32_t acc = 0;
+        for (int32_t b = 0; b < B; ++b) acc |= (bi >= 0 && x[c * B + b] == (int32_t)bi);
+        accept[c] = acc;
+        if (margin_y) margin_y[c] = bi >= 0 && second < INFINITY ? second - best : INFINITY;
     }
 }
 
