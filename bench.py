@@ -231,6 +231,9 @@ def main():
     if args.workload == "dynamic":
         run_dynamic(args, rank, world, dev)
         return
+    if args.workload == "hetero":
+        run_hetero(args, rank, world, dev)
+        return
     wl = synth.make_workload(args.workload, device=dev, n_seq=args.n_seq)
     t = wl.tree
     g = lambda x: torch.as_tensor(np.asarray(x)).to(dev).contiguous()
@@ -573,6 +576,110 @@ def run_dynamic(args, rank, world, dev):
             "gpu_launches": args.steps * (2 * gamma + 1), "clocks": clocks,
             "mean_accept_len": float(vout["accept_len"].float().mean().item()),
             "mean_draft_nodes_per_seq": float((b.row_k[:b.n_draft] > 0).sum().item()) / n_seq,
+        }))
+
+
+def run_hetero(args, rank, world, dev):
+    """Non-identical proposals (the augmented race on V x [B], B = 8 draft models): per step
+    gamma x (pps_draft_hetero over the n_seq x B proposal rows + pps_hetero_expand), then
+    pps_verify_tree over every node slot of the merged chains.  n_seq=64, V=128256, B=8,
+    gamma=5 (41 node slots and 40 proposal rows per sequence), bf16 logits: target rows as
+    zipf_k8; proposal b's rows = the target row of its static slot + N(0, (0.5 + 0.25 b)^2)
+    (the drafters' outputs are inputs)."""
+    from paper_2609_21858_gb300 import pps, synth, tree
+    n_seq, V, B, gamma = args.n_seq or 64, 128256, 8, 5
+    g = torch.Generator(device=dev)
+    g.manual_seed(3)
+    b = tree.HeteroTreeBuilder(n_seq, B, gamma, dev)
+    p = synth._zipf(g, b.n_nodes, V, 1.0, True, dev).to(torch.bfloat16)
+    N1 = 1 + B * gamma
+    sig = (0.5 + 0.25 * torch.arange(B, device=dev, dtype=torch.float32)).repeat(n_seq)[:, None]
+    q = []
+    for d in range(gamma):
+        # row (s, b) of depth d reads node (s, d, b)'s target row (the root at depth 0)
+        off = 0 if d == 0 else 1 + (d - 1) * B
+        w = torch.arange(B, device=dev) if d > 0 else torch.zeros(B, dtype=torch.long, device=dev)
+        slots = (torch.arange(n_seq, device=dev)[:, None] * N1 + off + w[None, :]).ravel()
+        q.append((p[slots].float() + sig * torch.randn(slots.numel(), V, generator=g, device=dev))
+                 .to(torch.bfloat16))
+    rk = torch.as_tensor(synth.splitmix64_stream(30, 2 * n_seq).view(np.int64), device=dev)
+    root_key, root_ctx = rk[:n_seq], rk[n_seq:]
+    root_pos = torch.full((n_seq,), 100, dtype=torch.int32, device=dev)
+    ws_v = pps.workspace(b.n_nodes, n_seq, dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    W = gamma + 1
+    vout = dict(winner=torch.empty(b.n_nodes, dtype=torch.int32, device=dev),
+                word=torch.empty(b.n_nodes, dtype=torch.int32, device=dev),
+                accept_len=torch.empty(n_seq, dtype=torch.int32, device=dev),
+                n_emitted=torch.empty(n_seq, dtype=torch.int32, device=dev),
+                emitted=torch.empty(n_seq, W, dtype=torch.int32, device=dev),
+                score=torch.empty(n_seq, W, dtype=torch.float32, device=dev),
+                score_sum=torch.empty(n_seq, dtype=torch.float64, device=dev))
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        b.run(root_key, root_ctx, root_pos, lambda d, *_: q[d], stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+        b.verify(p, ws=ws_v, out=vout, status=status, stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    assert int(status.item()) == 0, f"status flags {int(status.item())}"
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk = Clocks(dev.index or 0)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    clk.start()
+    time.sleep(0.3)
+    e0.record(stream)
+    for k in range(args.steps):
+        step(evs[k])
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = clk.stop()
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
+    t_draft = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    t_verify = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    n_prop = gamma * n_seq * B
+    rows = n_prop + b.n_nodes
+    nbytes = rows * V * 2
+    peak, peak_kind = _peaks()
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    hz = (clocks.get("sm_mhz") or 2070.0) * 1e6
+    mul_peak = sms * WIDE_MULS_PER_SM_CLK * hz / 1e12
+    tok_draft = n_prop * V
+    mul_ach = tok_draft * WIDE_MULS_PER_TOKEN / (t_draft / 1e3) / 1e12
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": rows * world / (ms / 1e3), "unit": "rows/s", "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded Zipf-rank logits; no model, no dataset)",
+            "config": {"workload": f"non-identical proposals: n_seq={n_seq}, V={V}, B={B} proposals, "
+                                   f"gamma={gamma}, {n_prop} proposal rows + {b.n_nodes} node slots per step",
+                       "rows_per_step": rows, "l2": f"inputs ({nbytes / 1e9:.2f} GB) larger than L2, no flush",
+                       "parallelism": f"replicas x{world}"},
+            "gb_per_s": nbytes / (ms / 1e3) / 1e9,
+            "roofline": {"bound": "alu", "achieved": mul_ach, "peak": mul_peak, "unit": "T wide-mul/s",
+                         "frac": mul_ach / mul_peak, "traffic": None,
+                         "kernel": "race_kernel, proposal rows (pps_draft_hetero) incl. the expansions",
+                         "ms": t_draft,
+                         "peak_kind": f"derived: {sms} SMs x {WIDE_MULS_PER_SM_CLK} 32x32->64 multiplies/clk x "
+                                      f"{hz / 1e6:.0f} MHz (median sampled SM clock)",
+                         "work": f"{WIDE_MULS_PER_TOKEN} wide multiplies per token x {tok_draft} tokens"},
+            "roofline_hbm": {"bound": "hbm", "achieved_draft": n_prop * V * 2 / (t_draft / 1e3) / 1e9,
+                             "achieved_verify": b.n_nodes * V * 2 / (t_verify / 1e3) / 1e9, "peak": peak,
+                             "peak_kind": peak_kind, "ms_verify": t_verify},
+            "gpu_launches": args.steps * (2 * gamma + 1), "clocks": clocks,
+            "mean_accept_len": float(vout["accept_len"].float().mean().item()),
+            "mean_nodes_per_seq": float((b.node_ctx != 0).sum().item()) / n_seq,
         }))
 
 

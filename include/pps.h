@@ -227,6 +227,90 @@ pps_status pps_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t dept
                            uint32_t* node_pos, pps_stream_t stream);
 
 /*
+ * Non-identical proposals (App. A, the proposition on heterogeneous
+ * proposals): B draft models Q_0..Q_{B-1} each propose one token per context
+ * from one Poisson process on the augmented vocabulary V x [B].  Proposal b
+ * is the race of Q_b over block b; the target is the race of P(i)/B over all
+ * of V x [B], whose token Y is accepted iff it equals some proposal.
+ *
+ * The augmented source (this library's reading; the paper fixes only that
+ * the points of V x [B] carry one common Poisson process): the B first
+ * arrivals of token i are generated by competing exponentials,
+ *   E_(i,b) = E'_i / B                    for b = J_i,
+ *   E_(i,b) = E'_i / B + F_(i,b)          otherwise,
+ * E'_i = -ln u of word w(i, 1) under the row's key (the plain source),
+ * J_i = floor(B w' / 2^32), w' = token i's word under key ^ 0x3C6EF372FE94F82B,
+ * F_(i,b) = -ln u of token i's word under key ^ (b + 1) * 0xBB67AE8584CAA73B
+ * (the least of B iid Exp(1) is Exp(B), in a uniform block independent of
+ * its value; the rest exceed it by iid Exp(1)).  Consequences: the target's Y
+ * is exactly the plain race winner on P (pps_verify_tree), its watermark word
+ * and the detector (pps_wm_score / pps_wm_detect) are unchanged, and J = J_Y
+ * (pps_hetero_block).
+ */
+#define PPS_MAX_BLOCKS 32
+
+/*
+ * pps_draft_hetero -- proposal rows: row r is proposal b = row_block[r] at
+ * its context, X = argmin_i ln E_(i,b) - logit_i / T (ties to the smaller
+ * token).  Arguments as pps_draft_list with K = 1, plus:
+ * row_block    [n_rows] proposal index of each row, 0 <= b < n_blocks (other
+ *              values are read as block indices of the same source; no memory
+ *              is indexed by them)
+ * n_blocks     B, 1 <= B <= PPS_MAX_BLOCKS (B = 1 is the plain race)
+ * out_tok      [n_rows] X, -1 if no token is usable
+ * out_key      nullable [n_rows] its key s = ln E_(X,b) - logit_X / T (fp32)
+ * ws, ws_bytes workspace of pps_workspace_size(n_rows, vocab, 1, 0) bytes
+ */
+pps_status pps_draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t row_stride,
+                            pps_row_ids ids, float temperature, const int32_t* row_block, int32_t n_blocks,
+                            int32_t* out_tok, float* out_key, uint32_t* status, void* ws, size_t ws_bytes,
+                            pps_stream_t stream);
+
+/*
+ * pps_hetero_expand -- one depth of the draft tree of B proposals, each
+ * drafting a chain of gamma tokens (each row drafted by pps_draft_hetero);
+ * chains that agree share nodes, so node c's draft list D(c) is the set of
+ * distinct tokens its proposals drew, and pps_verify_tree walks the tree with
+ * K = B.  A proposal at node o of depth d that drew x moves to the child
+ * (d+1, f), f = the first proposal at o that drew x.  Child identity: the same
+ * key, position + 1, label SplitMix64-output(label(c) ^ (x + 1) *
+ * 0x9E3779B97F4A7C15) (as pps_tree_expand).
+ *
+ * Fixed-capacity layout (K = B in pps_tree_expand's formulas):
+ *   nodes        N1 = 1 + B*gamma per sequence; node (s, d, o) =
+ *                s*N1 + (d == 0 ? 0 : 1 + (d-1)*B + o); seq_off[s] = s*N1;
+ *                node (s, d+1, b) is used iff proposal b is the first to reach it
+ *   node lists   depth-major, n_seq*(1 + B*(gamma-1)) rows of stride B: depth
+ *                d's rows start at L_d = n_seq*(d == 0 ? 0 : 1 + (d-1)*B),
+ *                w_d = (d == 0 ? 1 : B) per sequence, node (s, d, o) owns list
+ *                row L_d + s*w_d + o (its node_draft_row)
+ *   proposal rows depth-major, n_seq*B per depth: row (s, b) = s*B + b
+ * Inputs (depth d's proposal rows): draft_tok [n_seq*B] (pps_draft_hetero
+ * outputs), rows (their identities), row_owner [n_seq*B]: the node (s, d, o)
+ * of each row as o (0 at depth 0), -1 = proposal stopped (it drew nothing at
+ * an earlier depth).  A row with draft_tok < 0 stops its proposal.
+ * Outputs: list_tok, child_node [n_lists, B] and list_ndistinct [n_lists]:
+ * depth d's lists (tokens in proposal order, -1 past ndistinct; every list
+ * row of the depth is written, 0 entries for unused nodes); node_key,
+ * node_ctx, node_pos [n_seq*N1]: depth d+1's nodes (zeros for unused ones);
+ * next_key, next_ctx, next_pos, next_owner [n_seq*B]: depth d+1's proposal
+ * rows (only when depth + 1 < gamma; nullable otherwise).  All device pointers.
+ */
+pps_status pps_hetero_expand(int32_t n_seq, int32_t n_blocks, int32_t gamma, int32_t depth, const int32_t* draft_tok,
+                             pps_row_ids rows, const int32_t* row_owner, uint64_t* next_key, uint64_t* next_ctx,
+                             uint32_t* next_pos, int32_t* next_owner, int32_t* list_tok, int32_t* list_ndistinct,
+                             int32_t* child_node, uint64_t* node_key, uint64_t* node_ctx, uint32_t* node_pos,
+                             pps_stream_t stream);
+
+/*
+ * pps_hetero_block -- the block J = J_Y of the target's augmented point
+ * (Y, J) for n tokens Y (e.g. pps_verify_tree winners) under their contexts'
+ * identities; -1 where Y < 0.  1 <= n_blocks <= PPS_MAX_BLOCKS.
+ */
+pps_status pps_hetero_block(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_blocks, int32_t* out_block,
+                            pps_stream_t stream);
+
+/*
  * pps_wm_score -- detector pass (detector algorithm of App. E; Eq. 2):
  * regenerate the first-arrival word of every observed token under its
  * context's identity and score it, A_t = -ln(1 - u_t).

@@ -92,6 +92,9 @@ def lib():
             L.orc_tree_expand.argtypes = [i32, i32, i32, i32, i32p, i32p, i32p, u64p, u64p, u32p, i32p,
                                           u64p, u64p, u32p, i32p, i32p, u64p, u64p, u32p]
             L.orc_tree_expand.restype = None
+            L.orc_hetero_expand.argtypes = [i32, i32, i32, i32, i32p, u64p, u64p, u32p, i32p, u64p, u64p, u32p,
+                                            i32p, i32p, i32p, i32p, u64p, u64p, u32p]
+            L.orc_hetero_expand.restype = None
             L.orc_block_j.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32, i64, i32]
             L.orc_block_j.restype = i32
             L.orc_block_e.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32, i64, i32, i32]
@@ -342,3 +345,32 @@ def hetero_rows(p_logits, q_logits, key, ctx, pos, B: int, T: float = 1.0):
                           _ptr(word, ctypes.c_uint32), _ptr(acc, ctypes.c_int32), _ptr(my, ctypes.c_double),
                           _ptr(mx, ctypes.c_double))
     return dict(x=x.reshape(n, B), y=y, j=j, word=word, accept=acc, margin_y=my, margin_x=mx.reshape(n, B))
+
+
+def hetero_expand(n_seq, B, gamma, depth, tok, key, ctx, pos, owner, tree):
+    """One depth of the tree of B proposals; `tok` = the proposals' draws at this depth's
+    rows, `tree` = dict(list_tok, child_node [n_lists, B], list_nd [n_lists],
+    node_key/ctx/pos [n_seq*N1]), updated in place.
+    Returns (next_key, next_ctx, next_pos, next_owner) of depth+1's rows."""
+    n = n_seq * B
+    nk, nc = np.zeros(n, np.uint64), np.zeros(n, np.uint64)
+    npos, no = np.zeros(n, np.uint32), np.zeros(n, np.int32)
+    tok, owner = _c(tok, np.int32), _c(owner, np.int32)
+    key, ctx, pos = _c(key, np.uint64), _c(ctx, np.uint64), _c(pos, np.uint32)
+    lib().orc_hetero_expand(n_seq, int(B), int(gamma), int(depth), _ptr(tok, ctypes.c_int32),
+                            _ptr(key, ctypes.c_uint64), _ptr(ctx, ctypes.c_uint64), _ptr(pos, ctypes.c_uint32),
+                            _ptr(owner, ctypes.c_int32), _ptr(nk, ctypes.c_uint64), _ptr(nc, ctypes.c_uint64),
+                            _ptr(npos, ctypes.c_uint32), _ptr(no, ctypes.c_int32),
+                            _ptr(tree["list_tok"], ctypes.c_int32), _ptr(tree["list_nd"], ctypes.c_int32),
+                            _ptr(tree["child_node"], ctypes.c_int32), _ptr(tree["node_key"], ctypes.c_uint64),
+                            _ptr(tree["node_ctx"], ctypes.c_uint64), _ptr(tree["node_pos"], ctypes.c_uint32))
+    return nk, nc, npos, no
+
+
+def hetero_tree(n_seq, B, gamma):
+    """Empty oracle tree arrays of the multi-proposal layout."""
+    N1 = 1 + B * gamma
+    nl = n_seq * (1 + B * (gamma - 1))
+    return dict(list_tok=np.full((nl, B), -1, np.int32), child_node=np.full((nl, B), -1, np.int32),
+                list_nd=np.zeros(nl, np.int32), node_key=np.zeros(n_seq * N1, np.uint64),
+                node_ctx=np.zeros(n_seq * N1, np.uint64), node_pos=np.zeros(n_seq * N1, np.uint32))

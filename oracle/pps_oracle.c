@@ -714,6 +714,82 @@ void orc_hetero_rows(const float* p, const float* q, int64_t n_ctx, int32_t B, i
     }
 }
 
+/* One depth of the draft tree of B proposals, each drafting a chain (the
+ * proposition's one-step coupling applied at every node).  Layout of the
+ * fixed-capacity tree, per sequence s: node (s, d, o) = s*N1 + (d == 0 ? 0 :
+ * 1 + (d-1)*B + o), N1 = 1 + B*gamma; node lists depth-major, depth d's rows
+ * from L_d = n_seq*(d == 0 ? 0 : 1 + (d-1)*B), w_d = (d == 0 ? 1 : B) per
+ * sequence, node (s, d, o) owning list row L_d + s*w_d + o; proposal rows
+ * (s, b) = s*B + b per depth.  A proposal at node o (owner[r]; -1 = stopped)
+ * that drew token x (x < 0 stops it) moves to the child (d+1, f), f = the
+ * smallest proposal at the same node that drew x.  Node o's list: the tokens
+ * of the proposals b with first[b] = b at o, in increasing b, with child
+ * (d+1, b).  Depth d+1's node (s, d+1, b) holds its identities iff b owns it
+ * (zeros otherwise); next rows (key, label(c||x), pos + 1, f) for live
+ * proposals, zeros and owner -1 for stopped ones (written when depth + 1 <
+ * gamma). */
+void orc_hetero_expand(int32_t n_seq, int32_t B, int32_t gamma, int32_t depth, const int32_t* tok,
+                       const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, const int32_t* owner,
+                       uint64_t* next_key, uint64_t* next_ctx, uint32_t* next_pos, int32_t* next_owner,
+                       int32_t* list_tok, int32_t* list_nd, int32_t* child_node, uint64_t* node_key,
+                       uint64_t* node_ctx, uint32_t* node_pos)
+{
+    int64_t N1 = 1 + (int64_t)B * gamma;
+    int32_t w = depth == 0 ? 1 : B;
+    int64_t L_d = depth == 0 ? 0 : (int64_t)n_seq * (1 + (int64_t)(depth - 1) * B);
+    int32_t alive[64], first[64];
+    for (int64_t s = 0; s < n_seq; ++s) {
+        const int64_t r0 = s * B;
+        for (int32_t b = 0; b < B; ++b)
+            alive[b] = owner[r0 + b] >= 0 && owner[r0 + b] < w && tok[r0 + b] >= 0;
+        for (int32_t b = 0; b < B; ++b) {
+            first[b] = -1;
+            if (!alive[b]) continue;
+            for (int32_t t = 0; t <= b; ++t)
+                if (alive[t] && owner[r0 + t] == owner[r0 + b] && tok[r0 + t] == tok[r0 + b]) {
+                    first[b] = t;
+                    break;
+                }
+        }
+        const int64_t child0 = s * N1 + 1 + (int64_t)depth * B;
+        for (int32_t o = 0; o < w; ++o) {
+            const int64_t lr = L_d + s * w + o;
+            int32_t m = 0;
+            for (int32_t t = 0; t < B; ++t)
+                if (alive[t] && owner[r0 + t] == o && first[t] == t) {
+                    list_tok[lr * B + m] = tok[r0 + t];
+                    child_node[lr * B + m] = (int32_t)(child0 + t);
+                    ++m;
+                }
+            list_nd[lr] = m;
+            for (; m < B; ++m) {
+                list_tok[lr * B + m] = -1;
+                child_node[lr * B + m] = -1;
+            }
+        }
+        for (int32_t b = 0; b < B; ++b) {
+            const int64_t r = r0 + b;
+            uint64_t k = 0, lab = 0;
+            uint32_t p = 0;
+            if (alive[b]) {
+                k = key[r];
+                lab = orc_child_label(ctx[r], tok[r]);
+                p = pos[r] + 1u;
+            }
+            const int owns = alive[b] && first[b] == b;
+            node_key[child0 + b] = owns ? k : 0;
+            node_ctx[child0 + b] = owns ? lab : 0;
+            node_pos[child0 + b] = owns ? p : 0u;
+            if (depth + 1 < gamma) {
+                next_key[r] = k;
+                next_ctx[r] = lab;
+                next_pos[r] = p;
+                next_owner[r] = alive[b] ? first[b] : -1;
+            }
+        }
+    }
+}
+
 /* raw words of rows x vocab for a given arrival (bit-exact checks) */
 void orc_words(int64_t n_rows, int64_t V, const uint64_t* key, const uint64_t* ctx, const uint32_t* pos,
                int32_t arrival, uint32_t* out)

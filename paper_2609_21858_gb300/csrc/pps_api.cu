@@ -374,6 +374,64 @@ pps_status pps_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t dept
     return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
 }
 
+pps_status pps_draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t row_stride,
+                            pps_row_ids ids, float temperature, const int32_t* row_block, int32_t n_blocks,
+                            int32_t* out_tok, float* out_key, uint32_t* status, void* ws, size_t ws_bytes,
+                            pps_stream_t stream) {
+    pps_status st = check_rows(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature);
+    if (st != PPS_OK) return st;
+    if (n_blocks < 1 || n_blocks > PPS_MAX_BLOCKS) return PPS_ERR_INVALID_ARG;
+    if (n_rows == 0) return PPS_OK;
+    if (!out_tok || !row_block) return PPS_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < workspace_bytes(n_rows, 0)) return PPS_ERR_WORKSPACE;
+    RaceArgs a = base_args(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature);
+    a.K = 1;
+    a.out_tok = out_tok;
+    a.out_key = out_key;
+    a.status = status;
+    // one block is the plain race (E_(i,0) = E'_i)
+    if (n_blocks > 1) {
+        a.row_block = row_block;
+        a.n_blocks = n_blocks;
+        a.block_shift = std::nextafter((float)std::log2((double)n_blocks), INFINITY);
+    }
+    workspace_carve(ws, n_rows, 0, &a.partials, &a.row_cnt, &a.seq_cnt);
+    const int dt = dtype == PPS_BF16 ? 1 : 0;
+    const bool vec = vec_ok(q_logits, dtype, row_stride);
+    a.G = race_grid(a.total, dt, false, vec, n_blocks > 1);
+    return launch_race(a, dt, false, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_hetero_expand(int32_t n_seq, int32_t n_blocks, int32_t gamma, int32_t depth, const int32_t* draft_tok,
+                             pps_row_ids rows, const int32_t* row_owner, uint64_t* next_key, uint64_t* next_ctx,
+                             uint32_t* next_pos, int32_t* next_owner, int32_t* list_tok, int32_t* list_ndistinct,
+                             int32_t* child_node, uint64_t* node_key, uint64_t* node_ctx, uint32_t* node_pos,
+                             pps_stream_t stream) {
+    if (n_seq < 0 || n_blocks < 1 || n_blocks > PPS_MAX_BLOCKS || gamma < 1 || gamma > 64 || depth < 0 ||
+        depth >= gamma)
+        return PPS_ERR_INVALID_ARG;
+    if (n_seq == 0) return PPS_OK;
+    if (!draft_tok || !rows.key || !rows.ctx_hash || !rows.pos || !row_owner || !list_tok || !list_ndistinct ||
+        !child_node || !node_key || !node_ctx || !node_pos)
+        return PPS_ERR_INVALID_ARG;
+    if (depth + 1 < gamma && (!next_key || !next_ctx || !next_pos || !next_owner)) return PPS_ERR_INVALID_ARG;
+    cudaError_t e = launch_hetero_expand(n_seq, n_blocks, gamma, depth, draft_tok, rows.key, rows.ctx_hash, rows.pos,
+                                         row_owner, next_key, next_ctx, next_pos, next_owner, list_tok,
+                                         list_ndistinct, child_node, node_key, node_ctx, node_pos,
+                                         (cudaStream_t)stream);
+    return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_hetero_block(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_blocks, int32_t* out_block,
+                            pps_stream_t stream) {
+    if (n < 0 || n_blocks < 1 || n_blocks > PPS_MAX_BLOCKS) return PPS_ERR_INVALID_ARG;
+    if (n == 0) return PPS_OK;
+    if (!tokens || !ids.key || !ids.ctx_hash || !ids.pos || !out_block) return PPS_ERR_INVALID_ARG;
+    cudaError_t e = launch_hetero_block(n, n_blocks, tokens, ids.key, ids.ctx_hash, ids.pos, out_block,
+                                        (cudaStream_t)stream);
+    return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
 pps_status pps_philox_words(pps_row_ids ids, int64_t n_rows, int64_t vocab, int32_t arrival, uint32_t* out,
                             pps_stream_t stream) {
     if (n_rows < 0 || vocab < 1 || arrival < 1) return PPS_ERR_INVALID_ARG;

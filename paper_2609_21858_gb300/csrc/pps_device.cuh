@@ -238,6 +238,55 @@ __device__ __forceinline__ double key64(uint32_t w, float l, float T) {
     return log(exp1_f64(w)) - ld / (double)T;
 }
 
+// ------------------------------------------------------------------ augmented source
+//
+// Non-identical proposals (App. A, heterogeneous proposals): proposal b of B
+// races over block b of the augmented vocabulary V x [B], the target over all
+// of it with P(i)/B.  The B first arrivals of token i are generated by
+// competing exponentials (the least of B iid Exp(1) is Exp(B), lies in a
+// uniform block independent of its value, and the others exceed it by iid
+// Exp(1) amounts):
+//     E_(i,b) = E'_i / B                 in block J_i = floor(B wJ / 2^32),
+//     E_(i,b) = E'_i / B + F_(i,b)       in the other blocks,
+// with E'_i the token's first arrival (its word under the key), wJ its word
+// under key ^ kBlockJ and F_(i,b) = Exp(1) from its word under
+// key ^ (b + 1) kBlockF.  The target's augmented argmin is therefore the
+// plain race on P, and a proposal's key is at least the plain key - log2 B.
+constexpr uint64_t kBlockJ = 0x3C6EF372FE94F82Bull;
+constexpr uint64_t kBlockF = 0xBB67AE8584CAA73Bull;
+constexpr double kLog2Log2e = 0.5287663729448976;  // log2(log2 e)
+
+struct Blk {
+    int b = 0;          // the row's block (its proposal)
+    int B = 1;          // number of blocks (1: the plain race)
+    float shift = 0.f;  // >= log2 B: the filter tests plain keys against theta + shift
+};
+
+__device__ __forceinline__ int block_j(uint32_t wj, int B) { return (int)__umulhi(wj, (uint32_t)B); }
+
+// E_(i,b) in fp64 for token i with first-arrival word w
+static __device__ __noinline__ double block_e64(uint64_t key, uint64_t ctx, uint32_t pos, int64_t i, uint32_t w, int b,
+                                         int B) {
+    double e = exp1_f64(w) / (double)B;
+    if (b != block_j(word_of(key ^ kBlockJ, ctx, pos, i, 1), B))
+        e += exp1_f64(word_of(key ^ ((uint64_t)(uint32_t)(b + 1) * kBlockF), ctx, pos, i, 1));
+    return e;
+}
+
+// the list key of a block arrival, in key32's units (log2 E + log2 log2 e - l c),
+// evaluated in fp64 and rounded once: within key_err_bound of the exact key
+// for B <= 32 (|log2 E| < 39); NaN logits map to +inf
+__device__ __forceinline__ float block_key32(double e, float l, float c) {
+    if (l != l) return __int_as_float(0x7f800000);
+    return (float)(log2(e) + kLog2Log2e - (double)l * (double)c);
+}
+// the fp64 race key s = ln E_(i,b) - l/T
+__device__ __forceinline__ double block_key64(double e, float l, float T) {
+    double ld = (double)l;
+    if (ld != ld) return __longlong_as_double(0x7ff0000000000000ll);
+    return log(e) - ld / (double)T;
+}
+
 // Aaronson score A = -ln(1 - u) (Eq. 2), fp64 and accurate fp32
 __device__ __forceinline__ double score64(uint32_t w) {
     if (w < 0x80000000u) return -log1p(-(((double)w + 0.5) * 0x1p-32));

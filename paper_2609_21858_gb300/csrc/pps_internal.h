@@ -69,6 +69,11 @@ struct RaceArgs {
     int64_t nv;     // 16-byte vectors per row (last one may be partial)
     int64_t total;  // n_rows * nv
     int G;
+    // proposal rows of the augmented race (draft side only; row_block NULL = off):
+    // row r is proposal row_block[r] of n_blocks, block_shift >= log2 n_blocks
+    const int32_t* row_block;
+    int n_blocks;
+    float block_shift;
     // truncation (truncated race only): top-k in [1, kTopMax], top-p in (0, 1]
     int top_k;
     float top_p;
@@ -85,7 +90,7 @@ void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials
 
 // launchers (pps_race.cu)
 cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
-int race_grid(int64_t total, int dtype, bool verify, bool vec);
+int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk = false);
 cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
 int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec);
 
@@ -103,6 +108,13 @@ cudaError_t launch_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t 
                                const uint32_t* pos, const int32_t* row_k, uint64_t* next_key, uint64_t* next_ctx,
                                uint32_t* next_pos, int32_t* next_k, int32_t* child_node, uint64_t* node_key,
                                uint64_t* node_ctx, uint32_t* node_pos, cudaStream_t stream);
+cudaError_t launch_hetero_expand(int32_t n_seq, int32_t B, int32_t gamma, int32_t depth, const int32_t* tok,
+                                 const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, const int32_t* owner,
+                                 uint64_t* next_key, uint64_t* next_ctx, uint32_t* next_pos, int32_t* next_owner,
+                                 int32_t* list_tok, int32_t* list_nd, int32_t* child_node, uint64_t* node_key,
+                                 uint64_t* node_ctx, uint32_t* node_pos, cudaStream_t stream);
+cudaError_t launch_hetero_block(int64_t n, int32_t B, const int32_t* tok, const uint64_t* key, const uint64_t* ctx,
+                                const uint32_t* pos, int32_t* out, cudaStream_t stream);
 cudaError_t launch_words(const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int64_t n_rows, int64_t V,
                          int32_t arrival, uint32_t* out, cudaStream_t stream);
 cudaError_t launch_selftest(uint64_t w_begin, uint64_t w_end, float* out, cudaStream_t stream);

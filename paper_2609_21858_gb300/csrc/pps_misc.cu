@@ -283,6 +283,90 @@ __global__ void tree_expand_kernel(int32_t n_seq, int32_t K, int32_t gamma, int3
         }
 }
 
+// One depth of the draft tree of B non-identical proposals (layout in pps.h):
+// warp s takes sequence s, lane b proposal b.  A proposal at node o of depth
+// d that drew token x moves to child (d+1, f), f = the first proposal at the
+// same node that drew x; node o's list holds the distinct tokens of its
+// proposals in proposal order, each with that child.
+__global__ void hetero_expand_kernel(int32_t n_seq, int32_t B, int32_t gamma, int32_t depth,
+                                     const int32_t* __restrict__ tok, const uint64_t* __restrict__ key,
+                                     const uint64_t* __restrict__ ctx, const uint32_t* __restrict__ pos,
+                                     const int32_t* __restrict__ owner, uint64_t* next_key, uint64_t* next_ctx,
+                                     uint32_t* next_pos, int32_t* next_owner, int32_t* list_tok, int32_t* list_nd,
+                                     int32_t* child_node, uint64_t* node_key, uint64_t* node_ctx,
+                                     uint32_t* node_pos) {
+    const int lane = threadIdx.x & 31;
+    const int64_t s = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (s >= n_seq) return;
+    const int64_t N1 = 1 + (int64_t)B * gamma;
+    const int w = depth == 0 ? 1 : B;
+    // node lists are numbered depth-major: depth d's start at L_d = n_seq (1 + (d-1) B)
+    const int64_t L_d = depth == 0 ? 0 : (int64_t)n_seq * (1 + (int64_t)(depth - 1) * B);
+    const int64_t child0 = s * N1 + 1 + (int64_t)depth * B;  // node (s, d+1, 0)
+    const int64_t r = s * B + lane;
+    int o = -1, x = -1;
+    if (lane < B) {
+        o = owner[r];
+        x = tok[r];
+    }
+    const bool alive = lane < B && o >= 0 && o < w && x >= 0;
+    int first = alive ? lane : -1;
+    for (int t = 0; t < B; ++t) {
+        const int ot = __shfl_sync(FULL, o, t), xt = __shfl_sync(FULL, x, t);
+        const bool at = __shfl_sync(FULL, (int)alive, t) != 0;
+        if (alive && at && t < first && ot == o && xt == x) first = t;
+    }
+    // lane o writes the list of node (s, d, o)
+    const int64_t lr = L_d + s * w + lane;
+    int m = 0;
+    for (int t = 0; t < B; ++t) {
+        const int ot = __shfl_sync(FULL, o, t), xt = __shfl_sync(FULL, x, t), ft = __shfl_sync(FULL, first, t);
+        const bool at = __shfl_sync(FULL, (int)alive, t) != 0;
+        if (lane < w && at && ot == lane && ft == t) {
+            list_tok[lr * B + m] = xt;
+            child_node[lr * B + m] = (int32_t)(child0 + t);
+            ++m;
+        }
+    }
+    if (lane < w) {
+        for (int q = m; q < B; ++q) {
+            list_tok[lr * B + q] = -1;
+            child_node[lr * B + q] = -1;
+        }
+        list_nd[lr] = m;
+    }
+    // depth d+1: node (s, d+1, b) is proposal b's when it is the first to reach it
+    if (lane < B) {
+        uint64_t k = 0, lab = 0;
+        uint32_t p = 0;
+        if (alive) {
+            k = key[r];
+            lab = mix64(ctx[r] ^ ((uint64_t)(uint32_t)(x + 1) * 0x9E3779B97F4A7C15ull));
+            p = pos[r] + 1u;
+        }
+        const bool owns = alive && first == lane;
+        node_key[child0 + lane] = owns ? k : 0;
+        node_ctx[child0 + lane] = owns ? lab : 0;
+        node_pos[child0 + lane] = owns ? p : 0u;
+        if (depth + 1 < gamma) {
+            next_key[r] = k;
+            next_ctx[r] = lab;
+            next_pos[r] = p;
+            next_owner[r] = alive ? first : -1;
+        }
+    }
+}
+
+// block J of the augmented race's winning point (Y, J) for each token
+__global__ void hetero_block_kernel(int64_t n, int32_t B, const int32_t* __restrict__ tok,
+                                    const uint64_t* __restrict__ key, const uint64_t* __restrict__ ctx,
+                                    const uint32_t* __restrict__ pos, int32_t* __restrict__ out) {
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += (int64_t)gridDim.x * blockDim.x) {
+        const int32_t y = tok[t];
+        out[t] = y >= 0 ? block_j(word_of(key[t] ^ kBlockJ, ctx[t], pos[t], y, 1), B) : -1;
+    }
+}
+
 __global__ void words_kernel(const uint64_t* __restrict__ key, const uint64_t* __restrict__ ctx,
                              const uint32_t* __restrict__ pos, int64_t n_rows, int64_t V, int32_t arrival,
                              uint32_t* __restrict__ out) {
@@ -368,6 +452,28 @@ cudaError_t launch_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t 
     tree_expand_kernel<<<(unsigned)blocks, 256, 0, stream>>>(n_seq, K, gamma, depth, tok, mult, ndist, key, ctx, pos,
                                                               row_k, next_key, next_ctx, next_pos, next_k, child_node,
                                                               node_key, node_ctx, node_pos);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_hetero_expand(int32_t n_seq, int32_t B, int32_t gamma, int32_t depth, const int32_t* tok,
+                                 const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, const int32_t* owner,
+                                 uint64_t* next_key, uint64_t* next_ctx, uint32_t* next_pos, int32_t* next_owner,
+                                 int32_t* list_tok, int32_t* list_nd, int32_t* child_node, uint64_t* node_key,
+                                 uint64_t* node_ctx, uint32_t* node_pos, cudaStream_t stream) {
+    if (n_seq == 0) return cudaSuccess;
+    const int64_t blocks = ((int64_t)n_seq * 32 + 255) / 256;
+    hetero_expand_kernel<<<(unsigned)blocks, 256, 0, stream>>>(n_seq, B, gamma, depth, tok, key, ctx, pos, owner,
+                                                                next_key, next_ctx, next_pos, next_owner, list_tok,
+                                                                list_nd, child_node, node_key, node_ctx, node_pos);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_hetero_block(int64_t n, int32_t B, const int32_t* tok, const uint64_t* key, const uint64_t* ctx,
+                                const uint32_t* pos, int32_t* out, cudaStream_t stream) {
+    if (n == 0) return cudaSuccess;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    hetero_block_kernel<<<(unsigned)blocks, 256, 0, stream>>>(n, B, tok, key, ctx, pos, out);
     return cudaGetLastError();
 }
 

@@ -244,16 +244,17 @@ struct WarpList {
         kp = kp_;
         k = k_;
     }
-    // lower tf to b (no effect when b >= tf)
-    __device__ __forceinline__ void bound(float b) {
+    // lower tf to b (no effect when b >= tf); the filter tests plain keys
+    // against tf + shift (shift = 0 except for proposal rows of the augmented race)
+    __device__ __forceinline__ void bound(float b, float shift = 0.f) {
         tf = fminf(tf, b);
-        tz = filter_tz(tf);
+        tz = filter_tz(tf + shift);
     }
     // after the list changed: tf <= min(th, (entry k-1) + filter_slack)
-    __device__ __forceinline__ void refresh() {
+    __device__ __forceinline__ void refresh(float shift = 0.f) {
         th = __shfl_sync(FULL, lk, kp - 1);
         thi = __shfl_sync(FULL, li, kp - 1);
-        bound(fminf(th, filter_slack(__shfl_sync(FULL, lk, k - 1))));
+        bound(fminf(th, filter_slack(__shfl_sync(FULL, lk, k - 1))), shift);
     }
 };
 
@@ -263,7 +264,8 @@ struct WarpList {
 // sorted across the warp and merged.  Ends when no lane has a key below it,
 // so the threshold is always current.
 template <int VW>
-__device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], int64_t i0, int lane) {
+__device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], int64_t i0, int lane,
+                                                float shift = 0.f) {
     while (true) {
         float bk = kInf;
         int bi = INT_MAX, be = -1;
@@ -297,23 +299,32 @@ __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], in
 #pragma unroll
         for (int e = 0; e < VW; ++e)
             if (e == be) pk[e] = kInf;
-        L.refresh();
+        L.refresh(shift);
     }
 }
 
 // Filter, key and offer the 4 tokens of one Philox block (counter cb, tokens
-// 4cb..4cb+3, logits l[]) for the lanes with `mine`.
+// 4cb..4cb+3, logits l[]) for the lanes with `mine`.  BLK: the rows are
+// proposal b's race over block b of the augmented source; survivors of the
+// (shifted) plain filter are keyed with their block arrival.
+template <bool BLK>
 __device__ __forceinline__ void block_survivors(WarpList& L, const RowPhilox& rp, bool mine, uint32_t cb,
-                                                const float (&l)[4], unsigned valid, float c, int lane) {
+                                                const float (&l)[4], unsigned valid, float c, int lane, const Blk& bk,
+                                                uint64_t key, uint64_t ctx, uint32_t pos) {
     float pk[4] = {kInf, kInf, kInf, kInf};
     if (mine) {
         const uint4 q = rp.block(cb);
         const uint32_t wq[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e)
-            if (((valid >> e) & 1u) && filter_pass(wq[e], l[e], c, L.tz)) pk[e] = key32(wq[e], l[e], c);
+            if (((valid >> e) & 1u) && filter_pass(wq[e], l[e], c, L.tz)) {
+                if constexpr (BLK)
+                    pk[e] = block_key32(block_e64(key, ctx, pos, (int64_t)4 * cb + e, wq[e], bk.b, bk.B), l[e], c);
+                else
+                    pk[e] = key32(wq[e], l[e], c);
+            }
     }
-    offer_survivors<4>(L, pk, (int64_t)4 * cb, lane);
+    offer_survivors<4>(L, pk, (int64_t)4 * cb, lane, bk.shift);
 }
 
 // ---------------------------------------------------------------- rare paths (out of line)
@@ -329,9 +340,9 @@ constexpr int kQueueCap = 32 + 32 * 2 * PPS_UNITS;
 // Work off the queue: lane j regenerates the words of queued block j (32 at
 // a time), reloads its four logits, keys the tokens over the filter cut and
 // offers them.  Out of line; the fast scan itself makes no calls.
-template <int DT>
+template <int DT, bool BLK>
 __device__ __noinline__ SlowState flush_queue(SlowState st, const uint32_t* q, int qn, const char* row, float c,
-                                              uint64_t key, uint64_t ctx, uint32_t pos) {
+                                              uint64_t key, uint64_t ctx, uint32_t pos, Blk bk) {
     const int lane = threadIdx.x & 31;
     RowPhilox rp;
     rp.init(key, ctx, pos);
@@ -355,7 +366,7 @@ __device__ __noinline__ SlowState flush_queue(SlowState st, const uint32_t* q, i
                 l[3] = __uint_as_float(v.w);
             }
         }
-        block_survivors(st.L, rp, mine, cb, l, 0xfu, c, lane);
+        block_survivors<BLK>(st.L, rp, mine, cb, l, 0xfu, c, lane, bk, key, ctx, pos);
     }
     __syncwarp();
     return st;
@@ -364,9 +375,10 @@ __device__ __noinline__ SlowState flush_queue(SlowState st, const uint32_t* q, i
 // Scalar-load path, one vector per lane at a time: the last partial
 // iteration of a segment, the ragged vector of a row, and unaligned rows.
 // Tokens with a logit below `floor` take no part (-inf: none excluded).
-template <int DT>
+template <int DT, bool BLK = false>
 __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64_t V, int64_t base, int64_t v1,
-                                            float c, uint64_t key, uint64_t ctx, uint32_t pos, float floor) {
+                                            float c, uint64_t key, uint64_t ctx, uint32_t pos, float floor,
+                                            Blk bk = Blk{}) {
     constexpr int VW = DT == 1 ? 8 : 4;
     const int lane = threadIdx.x & 31;
     RowPhilox rp;
@@ -399,7 +411,7 @@ __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64
 #pragma unroll
                 for (int e = 0; e < 4; ++e) pass |= ((vh >> e) & 1u) && filter_pass(wq[e], l[e], c, st.L.tz);
             }
-            if (__any_sync(FULL, pass)) block_survivors(st.L, rp, pass, cb, l, vh, c, lane);
+            if (__any_sync(FULL, pass)) block_survivors<BLK>(st.L, rp, pass, cb, l, vh, c, lane, bk, key, ctx, pos);
         }
     }
     return st;
@@ -412,9 +424,10 @@ __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64
 // row's k-th key is at most their largest, and the slack keeps every token
 // that could tie with it (tf itself is recorded as a drop bound).  Without
 // it every block of the first iteration would pass the filter and be queued.
-template <int DT>
+// BLK: the lane's smallest plain key is replaced by that token's block key.
+template <int DT, bool BLK>
 __device__ __noinline__ float seed_theta(const char* row, int64_t v0, float c, uint64_t key, uint64_t ctx,
-                                         uint32_t pos, int k) {
+                                         uint32_t pos, int k, Blk blk) {
     const int lane = threadIdx.x & 31;
     RowPhilox rp;
     rp.init(key, ctx, pos);
@@ -442,6 +455,9 @@ __device__ __noinline__ float seed_theta(const char* row, int64_t v0, float c, u
             }
         }
     }
+    if constexpr (BLK)
+        bk = block_key32(block_e64(key, ctx, pos, bi, word_of(key, ctx, pos, bi, 1), blk.b, blk.B),
+                         load_logit<DT>(row, bi), c);
     warp_sort(bk, bi, lane);
     return filter_slack(__shfl_sync(FULL, bk, k - 1));
 }
@@ -559,9 +575,10 @@ __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* ro
 
 // Stream vectors [v0, v1) of one row through the warp's list: full
 // iterations through the fast loop, the rest through the scalar tail.
-template <int DT, bool VEC>
+template <int DT, bool VEC, bool BLK>
 __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int64_t V, int64_t v0, int64_t v1,
-                                               float c, uint64_t key, uint64_t ctx, uint32_t pos, uint32_t* q) {
+                                               float c, uint64_t key, uint64_t ctx, uint32_t pos, uint32_t* q,
+                                               const Blk& bk) {
     constexpr int VW = DT == 1 ? 8 : 4;
     constexpr int STEP = (DT == 1 ? 32 : 64) * PPS_UNITS;  // vectors per fast-loop iteration
     const int64_t nfull = V / VW;                           // vectors holding VW tokens
@@ -570,19 +587,19 @@ __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int
     SlowState st{L};
     int64_t base = v0;
     if (n_it > 0) {
-        st.L.bound(seed_theta<DT>(row, v0, c, key, ctx, pos, st.L.k));
+        st.L.bound(seed_theta<DT, BLK>(row, v0, c, key, ctx, pos, st.L.k, bk), bk.shift);
         int64_t it = 0;
         int qn = 0;
         while (it < n_it) {
             RowPhilox rp;
             rp.init(key, ctx, pos);
             it = fast_scan<DT>(rp, row, v0, it, n_it, c, st.L.tz, q, qn);
-            if (qn > 0) st = flush_queue<DT>(st, q, qn, row, c, key, ctx, pos);
+            if (qn > 0) st = flush_queue<DT, BLK>(st, q, qn, row, c, key, ctx, pos, bk);
             qn = 0;
         }
         base = v0 + n_it * STEP;
     }
-    if (base < v1) st = tail_loop<DT>(st, row, V, base, v1, c, key, ctx, pos, -kInf);
+    if (base < v1) st = tail_loop<DT, BLK>(st, row, V, base, v1, c, key, ctx, pos, -kInf, bk);
     L = st.L;
 }
 
@@ -665,16 +682,17 @@ __device__ __forceinline__ void emit_row(const RaceArgs& a, int64_t r, double dk
         size_t o = (size_t)r * K + lane;
         a.out_tok[o] = lane < kr ? tok : -1;
         if (a.out_key) a.out_key[o] = (mine && lane < kr) ? sk : kInf;
-        a.out_mult[o] = lane < kr ? mult : 0;
+        if (a.out_mult) a.out_mult[o] = lane < kr ? mult : 0;
         if (a.out_samples) a.out_samples[o] = lane < kr ? sample : -1;
     }
-    if (lane == 0) a.out_nd[r] = nd;
+    if (lane == 0 && a.out_nd) a.out_nd[r] = nd;
 }
 
 // Warp 0 finishes row r from its complete list (lk, li) and the drop bound.
-template <int DT, bool VERIFY>
+// BLK: the near-tie keys are those of the row's block arrivals.
+template <int DT, bool VERIFY, bool BLK = false>
 __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk, int li, float theta_drop, int kr,
-                                          int kp, int lane) {
+                                          int kp, int lane, Blk bk = Blk{}) {
     const int nvalid = __popc(__ballot_sync(FULL, lane < kp && lk < kInf));
     const float tau = nvalid >= kr ? __shfl_sync(FULL, lk, kr - 1) : kInf;
     bool complete;
@@ -701,7 +719,10 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
     if (need_exact) {
         if (lane < nvalid) {
             uint32_t w = word_of(key, ctx, pos, li, 1);
-            dk = key64(w, logit_at<DT>(a, r, li), a.T);
+            if constexpr (BLK)
+                dk = block_key64(block_e64(key, ctx, pos, li, w, bk.b, bk.B), logit_at<DT>(a, r, li), a.T);
+            else
+                dk = key64(w, logit_at<DT>(a, r, li), a.T);
         }
         warp_sort_d(dk, li, lane);
         sk = (float)dk;
@@ -828,9 +849,9 @@ __device__ __noinline__ void sequence_ticket(const RaceArgs& a, int64_t r, int l
     __syncwarp();
 }
 
-template <int DT, bool VERIFY>
+template <int DT, bool VERIFY, bool BLK>
 __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_t gw, int64_t NW, int64_t v0,
-                                        int64_t v1, const WarpList L, int kr, int kp) {
+                                            int64_t v1, const WarpList L, int kr, int kp, Blk bk) {
     const int lane = threadIdx.x & 31;
     const int64_t nv = a.nv;
     float lk = L.lk;
@@ -868,7 +889,7 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
         }
     }
     if (final_here) {
-        finalize_row<DT, VERIFY>(a, r, lk, li, theta_drop, kr, kp, lane);
+        finalize_row<DT, VERIFY, BLK>(a, r, lk, li, theta_drop, kr, kp, lane, bk);
         if constexpr (VERIFY) sequence_ticket(a, r, lane);
     }
 }
@@ -881,7 +902,7 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
 // sequence's walk is run by the warp that finishes its last node.  No warp
 // ever waits for another and the kernel has no block-wide barrier.
 
-template <int DT, bool VERIFY, bool VEC>
+template <int DT, bool VERIFY, bool VEC, bool BLK>
 __global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(const RaceArgs a) {
     __shared__ uint32_t s_queue[kQueueCap];
     const int64_t NW = a.G;
@@ -903,35 +924,46 @@ __global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(con
         const uint32_t pos = __ldg(a.pos + r);
         const char* row = reinterpret_cast<const char*>(a.logits) + (size_t)r * (size_t)a.stride * esz;
 
+        Blk bk;
+        if constexpr (BLK) {
+            bk.b = __ldg(a.row_block + r);
+            bk.B = a.n_blocks;
+            bk.shift = a.block_shift;
+        }
         WarpList L;
         L.reset(kp, kr);
-        stream_segment<DT, VEC>(L, row, a.V, v0, v1, c, key, ctx, pos, s_queue);
+        stream_segment<DT, VEC, BLK>(L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk);
 
-        finish_segment<DT, VERIFY>(a, r, gw, NW, v0, v1, L, kr, kp);
+        finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk);
     }
 }
 
 
 #include "pps_trunc.cuh"
 
-int race_grid(int64_t total, int dtype, bool verify, bool vec) {
-    static int sms = 0, occ[2][2][2] = {};
+// the race kernel instance: dtype x (verify | block draft | draft) x vec
+static const void* race_fn(int dtype, bool verify, bool blk, bool vec) {
+    if (dtype == 1) {
+        if (verify) return vec ? (const void*)race_kernel<1, true, true, false> : (const void*)race_kernel<1, true, false, false>;
+        if (blk) return vec ? (const void*)race_kernel<1, false, true, true> : (const void*)race_kernel<1, false, false, true>;
+        return vec ? (const void*)race_kernel<1, false, true, false> : (const void*)race_kernel<1, false, false, false>;
+    }
+    if (verify) return vec ? (const void*)race_kernel<0, true, true, false> : (const void*)race_kernel<0, true, false, false>;
+    if (blk) return vec ? (const void*)race_kernel<0, false, true, true> : (const void*)race_kernel<0, false, false, true>;
+    return vec ? (const void*)race_kernel<0, false, true, false> : (const void*)race_kernel<0, false, false, false>;
+}
+
+int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk) {
+    static int sms = 0, occ[2][3][2] = {};
     int dev = 0;
     cudaGetDevice(&dev);
     if (sms == 0) {
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         if (sms <= 0) sms = 1;
     }
-    int& o = occ[dtype][verify][vec];
+    int& o = occ[dtype][verify ? 1 : (blk ? 2 : 0)][vec];
     if (o == 0) {
-        const void* fn = nullptr;
-        if (dtype == 1)
-            fn = verify ? (vec ? (const void*)race_kernel<1, true, true> : (const void*)race_kernel<1, true, false>)
-                        : (vec ? (const void*)race_kernel<1, false, true> : (const void*)race_kernel<1, false, false>);
-        else
-            fn = verify ? (vec ? (const void*)race_kernel<0, true, true> : (const void*)race_kernel<0, true, false>)
-                        : (vec ? (const void*)race_kernel<0, false, true> : (const void*)race_kernel<0, false, false>);
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, kThreads, 0);
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, race_fn(dtype, verify, blk && !verify, vec), kThreads, 0);
         if (o <= 0) o = 1;
     }
     int64_t g = (int64_t)sms * o;
@@ -944,21 +976,28 @@ int race_grid(int64_t total, int dtype, bool verify, bool vec) {
 
 cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream) {
     dim3 grid(a.G), block(kThreads);
+    const bool blk = !verify && a.row_block != nullptr;
     if (dtype == 1) {
         if (verify) {
-            if (vec) race_kernel<1, true, true><<<grid, block, 0, stream>>>(a);
-            else race_kernel<1, true, false><<<grid, block, 0, stream>>>(a);
+            if (vec) race_kernel<1, true, true, false><<<grid, block, 0, stream>>>(a);
+            else race_kernel<1, true, false, false><<<grid, block, 0, stream>>>(a);
+        } else if (blk) {
+            if (vec) race_kernel<1, false, true, true><<<grid, block, 0, stream>>>(a);
+            else race_kernel<1, false, false, true><<<grid, block, 0, stream>>>(a);
         } else {
-            if (vec) race_kernel<1, false, true><<<grid, block, 0, stream>>>(a);
-            else race_kernel<1, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) race_kernel<1, false, true, false><<<grid, block, 0, stream>>>(a);
+            else race_kernel<1, false, false, false><<<grid, block, 0, stream>>>(a);
         }
     } else {
         if (verify) {
-            if (vec) race_kernel<0, true, true><<<grid, block, 0, stream>>>(a);
-            else race_kernel<0, true, false><<<grid, block, 0, stream>>>(a);
+            if (vec) race_kernel<0, true, true, false><<<grid, block, 0, stream>>>(a);
+            else race_kernel<0, true, false, false><<<grid, block, 0, stream>>>(a);
+        } else if (blk) {
+            if (vec) race_kernel<0, false, true, true><<<grid, block, 0, stream>>>(a);
+            else race_kernel<0, false, false, true><<<grid, block, 0, stream>>>(a);
         } else {
-            if (vec) race_kernel<0, false, true><<<grid, block, 0, stream>>>(a);
-            else race_kernel<0, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) race_kernel<0, false, true, false><<<grid, block, 0, stream>>>(a);
+            else race_kernel<0, false, false, false><<<grid, block, 0, stream>>>(a);
         }
     }
     return cudaGetLastError();

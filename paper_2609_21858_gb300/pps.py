@@ -21,6 +21,7 @@ DISTINCT, IID = 0, 1
 FLAG_GUARD, FLAG_LOGIT_RANGE = 1, 2
 MAX_K = 32
 MAX_TOP_K = 64
+MAX_BLOCKS = 32
 
 _lock = threading.Lock()
 _lib = None
@@ -76,6 +77,14 @@ def lib():
             L.pps_wm_detect.argtypes = [vp, RowIds, i64, i32, vp, ctypes.c_int, ctypes.c_double, vp, vp, vp, vp]
             L.pps_wm_detect.restype = ctypes.c_int
             L.pps_wm_score.restype = ctypes.c_int
+            L.pps_draft_hetero.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, vp, i32, vp, vp, vp, vp,
+                                           sz, vp]
+            L.pps_draft_hetero.restype = ctypes.c_int
+            L.pps_hetero_expand.argtypes = [i32, i32, i32, i32, vp, RowIds, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp,
+                                            vp, vp]
+            L.pps_hetero_expand.restype = ctypes.c_int
+            L.pps_hetero_block.argtypes = [vp, RowIds, i64, i32, vp, vp]
+            L.pps_hetero_block.restype = ctypes.c_int
             L.pps_philox_words.argtypes = [RowIds, i64, i64, i32, vp, vp]
             L.pps_philox_words.restype = ctypes.c_int
             L.pps_selftest_philox_rate.argtypes = [u64, vp, i32, vp]
@@ -273,6 +282,51 @@ def tree_expand(K: int, gamma: int, depth: int, draft, rows_key, rows_ctx, rows_
                                  _ptr(child_node), _ptr(nodes["key"]), _ptr(nodes["ctx"]), _ptr(nodes["pos"]),
                                  _stream(stream))
     _check("pps_tree_expand", code)
+
+
+def draft_hetero(q_logits, key, ctx, pos, row_block, n_blocks: int, temperature: float = 1.0, ws=None, status=None,
+                 out_tok=None, out_key=None, stream=None):
+    """pps_draft_hetero: proposal row_block[r] of n_blocks at each row (non-identical
+    proposals on the augmented source).  Returns the [n_rows] int32 tokens."""
+    n, V, stride = _rows(q_logits)
+    dev = q_logits.device
+    if out_tok is None:
+        out_tok = torch.empty(n, dtype=torch.int32, device=dev)
+    if ws is None:
+        ws = workspace(n, 0, dev)
+    if row_block.dtype != torch.int32 or not row_block.is_cuda or not row_block.is_contiguous():
+        raise TypeError("row_block must be a contiguous CUDA int32 tensor")
+    code = lib().pps_draft_hetero(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
+                                  float(temperature), _ptr(row_block), int(n_blocks), _ptr(out_tok), _ptr(out_key),
+                                  _ptr(status), _ptr(ws), ws.numel(), _stream(stream))
+    _check("pps_draft_hetero", code)
+    return out_tok
+
+
+def hetero_expand(n_blocks: int, gamma: int, depth: int, draft_tok, rows_key, rows_ctx, rows_pos, row_owner,
+                  nxt, lists: dict, nodes: dict, stream=None):
+    """pps_hetero_expand: depth `depth` of the tree of n_blocks proposals.  Writes
+    lists = dict(tok, ndist, child) of the depth's nodes, nodes = dict(key, ctx, pos) of
+    the next depth's nodes and nxt = dict(key, ctx, pos, owner) of the next depth's
+    proposal rows (None at the last depth) in place."""
+    n_seq = row_owner.numel() // n_blocks
+    nx = nxt or {}
+    code = lib().pps_hetero_expand(n_seq, int(n_blocks), int(gamma), int(depth), _ptr(draft_tok),
+                                   _ids(rows_key, rows_ctx, rows_pos), _ptr(row_owner), _ptr(nx.get("key")),
+                                   _ptr(nx.get("ctx")), _ptr(nx.get("pos")), _ptr(nx.get("owner")),
+                                   _ptr(lists["tok"]), _ptr(lists["ndist"]), _ptr(lists["child"]),
+                                   _ptr(nodes["key"]), _ptr(nodes["ctx"]), _ptr(nodes["pos"]), _stream(stream))
+    _check("pps_hetero_expand", code)
+
+
+def hetero_block(tokens, key, ctx, pos, n_blocks: int, out=None, stream=None):
+    """pps_hetero_block: the block J of the target's augmented point for each token."""
+    n = tokens.numel()
+    if out is None:
+        out = torch.empty(n, dtype=torch.int32, device=tokens.device)
+    code = lib().pps_hetero_block(_ptr(tokens), _ids(key, ctx, pos), n, int(n_blocks), _ptr(out), _stream(stream))
+    _check("pps_hetero_block", code)
+    return out
 
 
 SCORE_AARONSON, SCORE_U, SCORE_LI, SCORE_POWER_LAW = 0, 1, 2, 3

@@ -142,3 +142,37 @@ def test_tree_expand_validates_shape_arguments():
                dict(tok=None)):
         assert expand(**kw) == pps.ERR_INVALID_ARG, kw
     assert expand(n_seq=0) == pps.OK
+
+
+def test_hetero_entry_points_validate_arguments():
+    L = pps.lib()
+    fake = ctypes.c_void_p(256)
+    ids = pps.RowIds(256, 256, 256)
+    ws = pps.workspace_size(8, 0, 1, 0)
+
+    def draft(n_rows=8, V=100, stride=100, T=1.0, block=fake, B=4, tok=fake, ws_bytes=ws, dtype=pps.BF16):
+        return L.pps_draft_hetero(fake, dtype, n_rows, V, stride, ids, T, block, B, tok, None, None, fake, ws_bytes,
+                                  None)
+
+    for kw in (dict(B=0), dict(B=33), dict(stride=99), dict(T=0.0), dict(block=None), dict(tok=None),
+               dict(n_rows=-1), dict(V=0)):
+        assert draft(**kw) == pps.ERR_INVALID_ARG, kw
+    assert draft(ws_bytes=ws - 1) == pps.ERR_WORKSPACE
+    assert draft(dtype=7) == pps.ERR_UNSUPPORTED
+    assert draft(n_rows=0) == pps.OK
+
+    def expand(n_seq=4, B=4, gamma=3, depth=0, tok=fake, nxt=fake):
+        return L.pps_hetero_expand(n_seq, B, gamma, depth, tok, ids, fake, nxt, nxt, nxt, nxt, fake, fake, fake,
+                                   fake, fake, fake, None)
+
+    for kw in (dict(B=0), dict(B=33), dict(gamma=0), dict(gamma=65), dict(depth=-1), dict(depth=3), dict(n_seq=-1),
+               dict(tok=None), dict(nxt=None)):
+        assert expand(**kw) == pps.ERR_INVALID_ARG, kw
+    assert expand(n_seq=0) == pps.OK
+
+    def block(n=5, B=3, tok=fake, out=fake):
+        return L.pps_hetero_block(tok, ids, n, B, out, None)
+
+    for kw in (dict(B=0), dict(B=33), dict(n=-1), dict(tok=None), dict(out=None)):
+        assert block(**kw) == pps.ERR_INVALID_ARG, kw
+    assert block(n=0) == pps.OK

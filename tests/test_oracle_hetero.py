@@ -211,3 +211,69 @@ def test_block_streams_never_alias():
     wj = {oracle.word(key ^ cj, ctx, pos, i) for i in range(64)}
     wf = {oracle.word(key ^ (((b + 1) * cf) % 2 ** 64), ctx, pos, i) for b in range(4) for i in range(64)}
     assert not (ws & wj) and not (ws & wf) and not (wj & wf)
+
+
+# ---------------------------------------------------------------- the multi-proposal tree
+
+def _draw(b, d, ctx, Vs):
+    # a deterministic stand-in for proposal b's race at context ctx: few tokens, so chains agree often
+    h = oracle.mix64(int(ctx) ^ ((b + 1) * 0x9E3779B97F4A7C15 % 2 ** 64) ^ (d * 0x632BE59BD9B4E019 % 2 ** 64))
+    return -1 if h % 13 == 0 else int(h % Vs)
+
+
+@pytest.mark.parametrize("B,gamma,Vs", [(1, 3, 3), (3, 4, 2), (5, 3, 3), (8, 5, 2), (32, 2, 4)])
+def test_tree_is_the_trie_of_the_proposal_chains(B, gamma, Vs):
+    # brute force: each proposal's chain, then the distinct prefixes per depth
+    n_seq = 6
+    key, ctx, pos = _ids(n_seq, B * 10 + gamma)
+    tree = oracle.hetero_tree(n_seq, B, gamma)
+    N1 = 1 + B * gamma
+    roots = np.arange(n_seq) * N1
+    tree["node_key"][roots], tree["node_ctx"][roots], tree["node_pos"][roots] = key, ctx, pos
+    rk, rc, rp = np.repeat(key, B), np.repeat(ctx, B), np.repeat(pos, B)
+    owner = np.zeros(n_seq * B, np.int32)
+    for d in range(gamma):
+        tok = np.array([_draw(r % B, d, rc[r], Vs) if owner[r] >= 0 else 7 for r in range(n_seq * B)], np.int32)
+        rk, rc, rp, owner = oracle.hetero_expand(n_seq, B, gamma, d, tok, rk, rc, rp, owner, tree)
+    L = [0] + [n_seq * (1 + (d - 1) * B) for d in range(1, gamma + 1)]
+    for s in range(n_seq):
+        chains = []
+        for b in range(B):
+            c, ch = int(ctx[s]), []
+            for d in range(gamma):
+                x = _draw(b, d, c, Vs)
+                if x < 0:
+                    break
+                ch.append(x)
+                c = oracle.child_label(c, x)
+            chains.append(ch)
+        # walk the oracle's tree along every prefix and compare lists with the brute force
+        for d in range(gamma):
+            prefixes = sorted({tuple(ch[:d]) for ch in chains if len(ch) >= d})
+            nodes_at_d = []
+            for pre in prefixes:
+                node, lrow = s * N1, L[0] + s
+                for t, x in enumerate(pre):
+                    m = list(tree["list_tok"][lrow][:tree["list_nd"][lrow]]).index(x)
+                    node = tree["child_node"][lrow][m]
+                    o = node - s * N1 - 1 - t * B
+                    lrow = L[t + 1] + s * B + o if t + 1 < gamma else -1
+                nodes_at_d.append(node)
+                through = [b for b in range(B) if len(chains[b]) > d and tuple(chains[b][:d]) == pre]
+                want = []
+                for b in through:
+                    if chains[b][d] not in want:
+                        want.append(chains[b][d])
+                got = list(tree["list_tok"][lrow][:tree["list_nd"][lrow]])
+                assert got == want, (s, pre, got, want)
+                # the node's identity is the fold of the labeler along its prefix
+                lab = int(ctx[s])
+                for x in pre:
+                    lab = oracle.child_label(lab, x)
+                assert int(tree["node_ctx"][node]) == lab and int(tree["node_pos"][node]) == int(pos[s]) + d
+                assert int(tree["node_key"][node]) == int(key[s])
+            assert len(set(nodes_at_d)) == len(prefixes)
+        # unused node slots and list rows are empty
+        used = {tuple(ch[:d]) for ch in chains for d in range(1, len(ch) + 1)}
+        n_used = int(np.count_nonzero(tree["node_ctx"][s * N1 + 1:(s + 1) * N1]))
+        assert n_used == len(used)
