@@ -402,6 +402,13 @@ pps_status pps_philox_words(pps_row_ids ids, int64_t n_rows, int64_t vocab, int3
  * difference to out_max_err[0] (device float, must hold 0 before the call). */
 pps_status pps_selftest_key_error(uint64_t w_begin, uint64_t w_end, float* out_max_err, pps_stream_t stream);
 
+/* Self-test of the fp32 logarithm inside the block key of pps_draft_hetero:
+ * over every fp32 x in [x_lo, x_hi) (0 < x_lo <= x_hi, finite) it compares
+ * lg2.approx(x) with an fp64 log2 and writes the largest absolute difference
+ * to out_max_err[0] (device float, must hold 0 before the call).  The block
+ * key's error bound assumes at most 2^-17 over [2^-40, 2^7). */
+pps_status pps_selftest_lg2_error(float x_lo, float x_hi, float* out_max_err, pps_stream_t stream);
+
 /* Throughput self-test of the keyed source alone: generates n_blocks Philox
  * blocks (4 words each) with the streaming kernels' row-specialised
  * generator, in a grid of out_len / 256 CTAs of 256 threads, and writes one

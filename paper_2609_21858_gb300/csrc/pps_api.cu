@@ -445,6 +445,14 @@ pps_status pps_selftest_key_error(uint64_t w_begin, uint64_t w_end, float* out_m
     return launch_selftest(w_begin, w_end, out_max_err, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
 }
 
+pps_status pps_selftest_lg2_error(float x_lo, float x_hi, float* out_max_err, pps_stream_t stream) {
+    if (!out_max_err || !(x_lo > 0.0f) || !(x_hi >= x_lo) || !std::isfinite(x_hi)) return PPS_ERR_INVALID_ARG;
+    uint32_t b0, b1;
+    std::memcpy(&b0, &x_lo, 4);
+    std::memcpy(&b1, &x_hi, 4);
+    return launch_selftest_lg2(b0, b1, out_max_err, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
 pps_status pps_selftest_philox_rate(uint64_t n_blocks, uint32_t* out, int32_t out_len, pps_stream_t stream) {
     if (!out || out_len < 256 || n_blocks == 0) return PPS_ERR_INVALID_ARG;
     return launch_philox_rate(n_blocks, out, out_len, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;

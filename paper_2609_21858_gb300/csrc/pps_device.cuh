@@ -254,37 +254,59 @@ __device__ __forceinline__ double key64(uint32_t w, float l, float T) {
 // plain race on P, and a proposal's key is at least the plain key - log2 B.
 constexpr uint64_t kBlockJ = 0x3C6EF372FE94F82Bull;
 constexpr uint64_t kBlockF = 0xBB67AE8584CAA73Bull;
-constexpr double kLog2Log2e = 0.5287663729448976;  // log2(log2 e)
+
+// Extra error of the fp32 block key below over the plain key's bound: the
+// key is lg2.approx(fl(y' / B) [+ y_F]) - l c with y = -log2 u from
+// neg_log2_u.  With M = the bound on |key_x32(w) - log2(-log2 u)| (kErrAbs,
+// measured over all words) and e the absolute error of lg2.approx (at most
+// 2^-17 over every fp32 input of the key's range [2^-40, 2^7), measured by
+// pps_selftest_lg2_error: about 4.0e-6), each y has relative error
+// <= (M + e) ln 2, the scaling and the sum add three roundings, and the outer
+// lg2.approx adds e: |error| <= M + 2e + 3 * 2^-24 / ln 2 < 1.9e-5.
+constexpr float kBlkErr = 4.0e-5f;
 
 struct Blk {
     int b = 0;          // the row's block (its proposal)
     int B = 1;          // number of blocks (1: the plain race)
+    float invB = 1.f;   // 1 / B (fp32)
     float shift = 0.f;  // >= log2 B: the filter tests plain keys against theta + shift
+    float eb = 0.f;     // extra list-key error (kBlkErr for block rows)
 };
 
 __device__ __forceinline__ int block_j(uint32_t wj, int B) { return (int)__umulhi(wj, (uint32_t)B); }
 
-// E_(i,b) in fp64 for token i with first-arrival word w
-static __device__ __noinline__ double block_e64(uint64_t key, uint64_t ctx, uint32_t pos, int64_t i, uint32_t w, int b,
-                                         int B) {
-    double e = exp1_f64(w) / (double)B;
-    if (b != block_j(word_of(key ^ kBlockJ, ctx, pos, i, 1), B))
-        e += exp1_f64(word_of(key ^ ((uint64_t)(uint32_t)(b + 1) * kBlockF), ctx, pos, i, 1));
-    return e;
+// J_i and, when J_i != b, the word of the excess F_(i,b)
+__device__ __forceinline__ int block_words(uint64_t key, uint64_t ctx, uint32_t pos, int64_t i, int b, int B,
+                                           uint32_t& wf) {
+    const int J = block_j(word_of(key ^ kBlockJ, ctx, pos, i, 1), B);
+    wf = J != b ? word_of(key ^ ((uint64_t)(uint32_t)(b + 1) * kBlockF), ctx, pos, i, 1) : 0u;
+    return J;
 }
 
-// the list key of a block arrival, in key32's units (log2 E + log2 log2 e - l c),
-// evaluated in fp64 and rounded once: within key_err_bound of the exact key
-// for B <= 32 (|log2 E| < 39); NaN logits map to +inf
-__device__ __forceinline__ float block_key32(double e, float l, float c) {
-    if (l != l) return __int_as_float(0x7f800000);
-    return (float)(log2(e) + kLog2Log2e - (double)l * (double)c);
+// the fp32 list key of block arrival E_(i,b) (key32's units: log2 E + log2 log2 e
+// - l c), within key_err_bound + kBlkErr of the exact value; NaN logits -> +inf
+__device__ __forceinline__ float block_key32(uint32_t w, int J, uint32_t wf, int b, float invB, float l, float c) {
+    float y = neg_log2_u(w) * invB;
+    if (J != b) y += neg_log2_u(wf);
+    const float k = fmaf(-l, c, lg2_approx(y));
+    return k != k ? __int_as_float(0x7f800000) : k;
 }
-// the fp64 race key s = ln E_(i,b) - l/T
-__device__ __forceinline__ double block_key64(double e, float l, float T) {
-    double ld = (double)l;
+
+// the fp64 race key s = ln E_(i,b) - l/T (near ties)
+__device__ __forceinline__ double block_key64(uint32_t w, int J, uint32_t wf, int b, int B, float l, float T) {
+    const double ld = (double)l;
     if (ld != ld) return __longlong_as_double(0x7ff0000000000000ll);
+    double e = exp1_f64(w) / (double)B;
+    if (J != b) e += exp1_f64(wf);
     return log(e) - ld / (double)T;
+}
+
+// list key of token i of a block row (words regenerated; out of line: rare path)
+static __device__ __noinline__ float block_key_of(uint64_t key, uint64_t ctx, uint32_t pos, int64_t i, uint32_t w,
+                                                  float l, float c, int b, int B, float invB) {
+    uint32_t wf;
+    const int J = block_words(key, ctx, pos, i, b, B, wf);
+    return block_key32(w, J, wf, b, invB, l, c);
 }
 
 // Aaronson score A = -ln(1 - u) (Eq. 2), fp64 and accurate fp32

@@ -118,6 +118,7 @@ cudaError_t launch_hetero_block(int64_t n, int32_t B, const int32_t* tok, const 
 cudaError_t launch_words(const uint64_t* key, const uint64_t* ctx, const uint32_t* pos, int64_t n_rows, int64_t V,
                          int32_t arrival, uint32_t* out, cudaStream_t stream);
 cudaError_t launch_selftest(uint64_t w_begin, uint64_t w_end, float* out, cudaStream_t stream);
+cudaError_t launch_selftest_lg2(uint32_t b0, uint32_t b1, float* out, cudaStream_t stream);
 cudaError_t launch_philox_rate(uint64_t n_blocks, uint32_t* out, int out_len, cudaStream_t stream);
 
 }  // namespace pps

@@ -394,6 +394,21 @@ __global__ void selftest_kernel(uint64_t w0, uint64_t w1, float* out) {
     if ((threadIdx.x & 31) == 0) atomicMax(reinterpret_cast<unsigned int*>(out), __float_as_uint(worst));
 }
 
+// largest |lg2.approx(x) - log2 x| over the positive fp32 x with bit patterns
+// in [b0, b1) (every input of the block key's outer logarithm)
+__global__ void selftest_lg2_kernel(uint32_t b0, uint32_t b1, float* out) {
+    float worst = 0.0f;
+    for (uint64_t b = (uint64_t)b0 + (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; b < b1;
+         b += (uint64_t)gridDim.x * blockDim.x) {
+        const float x = __uint_as_float((uint32_t)b);
+        const float d = (float)fabs((double)lg2_approx(x) - log2((double)x));
+        worst = fmaxf(worst, d);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) worst = fmaxf(worst, __shfl_xor_sync(FULL, worst, o));
+    if ((threadIdx.x & 31) == 0) atomicMax(reinterpret_cast<unsigned int*>(out), __float_as_uint(worst));
+}
+
 // Philox-only throughput: every thread generates blocks c0 = t, t + stride, ...
 // with the row-specialised generator of the streaming kernels and folds the
 // words into one value, so the kernel is bound by the Philox multiplies alone
@@ -493,6 +508,14 @@ cudaError_t launch_selftest(uint64_t w_begin, uint64_t w_end, float* out, cudaSt
     uint64_t blocks = (n + 255) / 256;
     if (blocks > 152 * 64) blocks = 152 * 64;
     selftest_kernel<<<(unsigned)blocks, 256, 0, stream>>>(w_begin, w_end, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_selftest_lg2(uint32_t b0, uint32_t b1, float* out, cudaStream_t stream) {
+    if (b1 <= b0) return cudaSuccess;
+    uint64_t blocks = ((uint64_t)(b1 - b0) + 255) / 256;
+    if (blocks > 152 * 64) blocks = 152 * 64;
+    selftest_lg2_kernel<<<(unsigned)blocks, 256, 0, stream>>>(b0, b1, out);
     return cudaGetLastError();
 }
 

@@ -250,11 +250,12 @@ struct WarpList {
         tf = fminf(tf, b);
         tz = filter_tz(tf + shift);
     }
-    // after the list changed: tf <= min(th, (entry k-1) + filter_slack)
-    __device__ __forceinline__ void refresh(float shift = 0.f) {
+    // after the list changed: tf <= min(th, (entry k-1) + filter_slack), the
+    // slack widened by 4 eb for keys with extra error eb
+    __device__ __forceinline__ void refresh(float shift = 0.f, float eb = 0.f) {
         th = __shfl_sync(FULL, lk, kp - 1);
         thi = __shfl_sync(FULL, li, kp - 1);
-        bound(fminf(th, filter_slack(__shfl_sync(FULL, lk, k - 1))), shift);
+        bound(fminf(th, filter_slack(__shfl_sync(FULL, lk, k - 1)) + 4.0f * eb), shift);
     }
 };
 
@@ -265,7 +266,7 @@ struct WarpList {
 // so the threshold is always current.
 template <int VW>
 __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], int64_t i0, int lane,
-                                                float shift = 0.f) {
+                                                float shift = 0.f, float eb = 0.f) {
     while (true) {
         float bk = kInf;
         int bi = INT_MAX, be = -1;
@@ -299,14 +300,15 @@ __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], in
 #pragma unroll
         for (int e = 0; e < VW; ++e)
             if (e == be) pk[e] = kInf;
-        L.refresh(shift);
+        L.refresh(shift, eb);
     }
 }
 
 // Filter, key and offer the 4 tokens of one Philox block (counter cb, tokens
 // 4cb..4cb+3, logits l[]) for the lanes with `mine`.  BLK: the rows are
 // proposal b's race over block b of the augmented source; survivors of the
-// (shifted) plain filter are keyed with their block arrival.
+// (shifted) plain filter are keyed with their block arrival (fp32, error
+// bound widened by bk.eb).
 template <bool BLK>
 __device__ __forceinline__ void block_survivors(WarpList& L, const RowPhilox& rp, bool mine, uint32_t cb,
                                                 const float (&l)[4], unsigned valid, float c, int lane, const Blk& bk,
@@ -315,16 +317,30 @@ __device__ __forceinline__ void block_survivors(WarpList& L, const RowPhilox& rp
     if (mine) {
         const uint4 q = rp.block(cb);
         const uint32_t wq[4] = {q.x, q.y, q.z, q.w};
+        unsigned pm = 0;
 #pragma unroll
         for (int e = 0; e < 4; ++e)
-            if (((valid >> e) & 1u) && filter_pass(wq[e], l[e], c, L.tz)) {
-                if constexpr (BLK)
-                    pk[e] = block_key32(block_e64(key, ctx, pos, (int64_t)4 * cb + e, wq[e], bk.b, bk.B), l[e], c);
-                else
-                    pk[e] = key32(wq[e], l[e], c);
+            if (((valid >> e) & 1u) && filter_pass(wq[e], l[e], c, L.tz)) pm |= 1u << e;
+        if constexpr (BLK) {
+            if (pm) {
+                // the block's J words and block-b excess words, four tokens per Philox block
+                const uint64_t kj = key ^ kBlockJ, kf = key ^ ((uint64_t)(uint32_t)(bk.b + 1) * kBlockF);
+                const uint4 jq = philox(cb, pos, (uint32_t)ctx, (uint32_t)(ctx >> 32), (uint32_t)kj,
+                                        (uint32_t)(kj >> 32));
+                const uint4 fq = philox(cb, pos, (uint32_t)ctx, (uint32_t)(ctx >> 32), (uint32_t)kf,
+                                        (uint32_t)(kf >> 32));
+                const uint32_t wj[4] = {jq.x, jq.y, jq.z, jq.w}, wf[4] = {fq.x, fq.y, fq.z, fq.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if ((pm >> e) & 1u) pk[e] = block_key32(wq[e], block_j(wj[e], bk.B), wf[e], bk.b, bk.invB, l[e], c);
             }
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                if ((pm >> e) & 1u) pk[e] = key32(wq[e], l[e], c);
+        }
     }
-    offer_survivors<4>(L, pk, (int64_t)4 * cb, lane, bk.shift);
+    offer_survivors<4>(L, pk, (int64_t)4 * cb, lane, bk.shift, bk.eb);
 }
 
 // ---------------------------------------------------------------- rare paths (out of line)
@@ -456,10 +472,10 @@ __device__ __noinline__ float seed_theta(const char* row, int64_t v0, float c, u
         }
     }
     if constexpr (BLK)
-        bk = block_key32(block_e64(key, ctx, pos, bi, word_of(key, ctx, pos, bi, 1), blk.b, blk.B),
-                         load_logit<DT>(row, bi), c);
+        bk = block_key_of(key, ctx, pos, bi, word_of(key, ctx, pos, bi, 1), load_logit<DT>(row, bi), c, blk.b,
+                          blk.B, blk.invB);
     warp_sort(bk, bi, lane);
-    return filter_slack(__shfl_sync(FULL, bk, k - 1));
+    return filter_slack(__shfl_sync(FULL, bk, k - 1)) + 4.0f * blk.eb;
 }
 
 // ---------------------------------------------------------------- the fast loop
@@ -695,13 +711,15 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
                                           int kp, int lane, Blk bk = Blk{}) {
     const int nvalid = __popc(__ballot_sync(FULL, lane < kp && lk < kInf));
     const float tau = nvalid >= kr ? __shfl_sync(FULL, lk, kr - 1) : kInf;
+    // list-key error bound (block rows: widened by bk.eb)
+    auto err = [&](float k) { return BLK ? key_err_bound(k) + bk.eb : key_err_bound(k); };
     bool complete;
     if (nvalid < kr)
         complete = theta_drop == kInf;
     else if (tau == -kInf)
         complete = true;
     else
-        complete = theta_drop == kInf || theta_drop > tau + key_err_bound(tau) + key_err_bound(theta_drop);
+        complete = theta_drop == kInf || theta_drop > tau + err(tau) + err(theta_drop);
     if (lane == 0 && a.status) {
         unsigned f = complete ? 0u : PPS_FLAG_GUARD;
         if (nvalid >= kr && tau > -kInf && fabsf(tau) > 65536.0f) f |= PPS_FLAG_LOGIT_RANGE;
@@ -710,7 +728,7 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
     // near ties among the first min(nvalid, kr+1) entries
     float nk = __shfl_down_sync(FULL, lk, 1);
     int lim = min(nvalid, kr + 1);
-    bool close = lane + 1 < lim && !(nk - lk > key_err_bound(lk) + key_err_bound(nk));
+    bool close = lane + 1 < lim && !(nk - lk > err(lk) + err(nk));
     const bool need_exact = (__ballot_sync(FULL, close) != 0) || (!VERIFY && a.iid);
     const uint64_t key = a.key[r], ctx = a.ctx[r];
     const uint32_t pos = a.pos[r];
@@ -719,9 +737,11 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
     if (need_exact) {
         if (lane < nvalid) {
             uint32_t w = word_of(key, ctx, pos, li, 1);
-            if constexpr (BLK)
-                dk = block_key64(block_e64(key, ctx, pos, li, w, bk.b, bk.B), logit_at<DT>(a, r, li), a.T);
-            else
+            if constexpr (BLK) {
+                uint32_t wf;
+                const int J = block_words(key, ctx, pos, li, bk.b, bk.B, wf);
+                dk = block_key64(w, J, wf, bk.b, bk.B, logit_at<DT>(a, r, li), a.T);
+            } else
                 dk = key64(w, logit_at<DT>(a, r, li), a.T);
         }
         warp_sort_d(dk, li, lane);
@@ -928,7 +948,9 @@ __global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(con
         if constexpr (BLK) {
             bk.b = __ldg(a.row_block + r);
             bk.B = a.n_blocks;
+            bk.invB = 1.0f / (float)a.n_blocks;
             bk.shift = a.block_shift;
+            bk.eb = kBlkErr;
         }
         WarpList L;
         L.reset(kp, kr);

@@ -89,6 +89,8 @@ def lib():
             L.pps_philox_words.restype = ctypes.c_int
             L.pps_selftest_philox_rate.argtypes = [u64, vp, i32, vp]
             L.pps_selftest_philox_rate.restype = ctypes.c_int
+            L.pps_selftest_lg2_error.argtypes = [f32, f32, vp, vp]
+            L.pps_selftest_lg2_error.restype = ctypes.c_int
             L.pps_selftest_key_error.argtypes = [u64, u64, vp, vp]
             L.pps_selftest_key_error.restype = ctypes.c_int
             _lib = L
@@ -362,6 +364,14 @@ def philox_words(key, ctx, pos, vocab: int, arrival: int = 1, stream=None):
 def selftest_key_error(w_begin: int = 0, w_end: int = 1 << 32, stream=None) -> float:
     out = torch.zeros(1, dtype=torch.float32, device="cuda")
     _check("pps_selftest_key_error", lib().pps_selftest_key_error(w_begin, w_end, _ptr(out), _stream(stream)))
+    return float(out.item())
+
+
+def selftest_lg2_error(x_lo: float = 2.0 ** -40, x_hi: float = 2.0 ** 7, stream=None) -> float:
+    """Largest |lg2.approx(x) - log2 x| over every fp32 x in [x_lo, x_hi)."""
+    out = torch.zeros(1, dtype=torch.float32, device="cuda")
+    _check("pps_selftest_lg2_error", lib().pps_selftest_lg2_error(float(x_lo), float(x_hi), _ptr(out),
+                                                                  _stream(stream)))
     return float(out.item())
 
 

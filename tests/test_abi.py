@@ -80,6 +80,9 @@ def test_validation_rejects_bad_arguments_without_a_gpu():
     assert L.pps_wm_score(fake, ids, 10, 0, fake, fake, None, None) == pps.ERR_INVALID_ARG
     assert L.pps_philox_words(ids, 1, 10, 0, fake, None) == pps.ERR_INVALID_ARG
     assert L.pps_selftest_key_error(0, (1 << 32) + 1, fake, None) == pps.ERR_INVALID_ARG
+    assert L.pps_selftest_lg2_error(0.0, 1.0, fake, None) == pps.ERR_INVALID_ARG
+    assert L.pps_selftest_lg2_error(2.0, 1.0, fake, None) == pps.ERR_INVALID_ARG
+    assert L.pps_selftest_lg2_error(1.0, 2.0, None, None) == pps.ERR_INVALID_ARG
 
 
 def test_workspace_size_grows_with_rows_and_sequences():

@@ -114,6 +114,12 @@ def test_full_size_proposal_rows_sampled():
         assert om[i] < FLIP_MARGIN
 
 
+def test_block_key_logarithm_error_is_within_its_bound():
+    # the fp32 block key's bound (kBlkErr) assumes lg2.approx errs by at most 2^-17
+    # over the key's whole input range; checked over every fp32 input there
+    assert pps.selftest_lg2_error(2.0 ** -40, 2.0 ** 7) <= 2.0 ** -17
+
+
 def test_winner_blocks_match_the_oracle():
     n = 5000
     rng = np.random.default_rng(2)
