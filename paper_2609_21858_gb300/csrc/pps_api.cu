@@ -393,7 +393,6 @@ pps_status pps_draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_row
     if (n_blocks > 1) {
         a.row_block = row_block;
         a.n_blocks = n_blocks;
-        a.block_shift = std::nextafter((float)std::log2((double)n_blocks), INFINITY);
     }
     workspace_carve(ws, n_rows, 0, &a.partials, &a.row_cnt, &a.seq_cnt);
     const int dt = dtype == PPS_BF16 ? 1 : 0;

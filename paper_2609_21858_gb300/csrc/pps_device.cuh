@@ -266,11 +266,11 @@ constexpr uint64_t kBlockF = 0xBB67AE8584CAA73Bull;
 constexpr float kBlkErr = 4.0e-5f;
 
 struct Blk {
-    int b = 0;          // the row's block (its proposal)
-    int B = 1;          // number of blocks (1: the plain race)
-    float invB = 1.f;   // 1 / B (fp32)
-    float shift = 0.f;  // >= log2 B: the filter tests plain keys against theta + shift
-    float eb = 0.f;     // extra list-key error (kBlkErr for block rows)
+    int b = 0;  // the row's block (its proposal)
+    int B = 1;  // number of blocks (1: the plain race)
+    // the filter tests plain keys against theta + shift, shift = ceil(log2 B) >= log2 B
+    __device__ __forceinline__ float shift() const { return (float)(32 - __clz(B - 1)); }
+    __device__ __forceinline__ float invB() const { return 1.0f / (float)B; }
 };
 
 __device__ __forceinline__ int block_j(uint32_t wj, int B) { return (int)__umulhi(wj, (uint32_t)B); }

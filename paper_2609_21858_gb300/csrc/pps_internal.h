@@ -70,10 +70,9 @@ struct RaceArgs {
     int64_t total;  // n_rows * nv
     int G;
     // proposal rows of the augmented race (draft side only; row_block NULL = off):
-    // row r is proposal row_block[r] of n_blocks, block_shift >= log2 n_blocks
+    // row r is proposal row_block[r] of n_blocks
     const int32_t* row_block;
     int n_blocks;
-    float block_shift;
     // truncation (truncated race only): top-k in [1, kTopMax], top-p in (0, 1]
     int top_k;
     float top_p;

@@ -43,6 +43,9 @@
 #ifndef PPS_RACE_MIN_BLOCKS
 #define PPS_RACE_MIN_BLOCKS 12  // one-warp CTAs resident per SM (register budget 168, no spills)
 #endif
+#ifndef PPS_BLOCK_MIN_BLOCKS
+#define PPS_BLOCK_MIN_BLOCKS 12  // the same for proposal rows of the augmented race (16 spills)
+#endif
 
 namespace pps {
 
@@ -308,7 +311,7 @@ __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], in
 // 4cb..4cb+3, logits l[]) for the lanes with `mine`.  BLK: the rows are
 // proposal b's race over block b of the augmented source; survivors of the
 // (shifted) plain filter are keyed with their block arrival (fp32, error
-// bound widened by bk.eb).
+// bound widened by kBlkErr).
 template <bool BLK>
 __device__ __forceinline__ void block_survivors(WarpList& L, const RowPhilox& rp, bool mine, uint32_t cb,
                                                 const float (&l)[4], unsigned valid, float c, int lane, const Blk& bk,
@@ -332,7 +335,8 @@ __device__ __forceinline__ void block_survivors(WarpList& L, const RowPhilox& rp
                 const uint32_t wj[4] = {jq.x, jq.y, jq.z, jq.w}, wf[4] = {fq.x, fq.y, fq.z, fq.w};
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
-                    if ((pm >> e) & 1u) pk[e] = block_key32(wq[e], block_j(wj[e], bk.B), wf[e], bk.b, bk.invB, l[e], c);
+                    if ((pm >> e) & 1u)
+                        pk[e] = block_key32(wq[e], block_j(wj[e], bk.B), wf[e], bk.b, bk.invB(), l[e], c);
             }
         } else {
 #pragma unroll
@@ -340,7 +344,7 @@ __device__ __forceinline__ void block_survivors(WarpList& L, const RowPhilox& rp
                 if ((pm >> e) & 1u) pk[e] = key32(wq[e], l[e], c);
         }
     }
-    offer_survivors<4>(L, pk, (int64_t)4 * cb, lane, bk.shift, bk.eb);
+    offer_survivors<4>(L, pk, (int64_t)4 * cb, lane, BLK ? bk.shift() : 0.f, BLK ? kBlkErr : 0.f);
 }
 
 // ---------------------------------------------------------------- rare paths (out of line)
@@ -473,9 +477,9 @@ __device__ __noinline__ float seed_theta(const char* row, int64_t v0, float c, u
     }
     if constexpr (BLK)
         bk = block_key_of(key, ctx, pos, bi, word_of(key, ctx, pos, bi, 1), load_logit<DT>(row, bi), c, blk.b,
-                          blk.B, blk.invB);
+                          blk.B, blk.invB());
     warp_sort(bk, bi, lane);
-    return filter_slack(__shfl_sync(FULL, bk, k - 1)) + 4.0f * blk.eb;
+    return filter_slack(__shfl_sync(FULL, bk, k - 1)) + (BLK ? 4.0f * kBlkErr : 0.f);
 }
 
 // ---------------------------------------------------------------- the fast loop
@@ -603,7 +607,7 @@ __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int
     SlowState st{L};
     int64_t base = v0;
     if (n_it > 0) {
-        st.L.bound(seed_theta<DT, BLK>(row, v0, c, key, ctx, pos, st.L.k, bk), bk.shift);
+        st.L.bound(seed_theta<DT, BLK>(row, v0, c, key, ctx, pos, st.L.k, bk), BLK ? bk.shift() : 0.f);
         int64_t it = 0;
         int qn = 0;
         while (it < n_it) {
@@ -711,8 +715,8 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
                                           int kp, int lane, Blk bk = Blk{}) {
     const int nvalid = __popc(__ballot_sync(FULL, lane < kp && lk < kInf));
     const float tau = nvalid >= kr ? __shfl_sync(FULL, lk, kr - 1) : kInf;
-    // list-key error bound (block rows: widened by bk.eb)
-    auto err = [&](float k) { return BLK ? key_err_bound(k) + bk.eb : key_err_bound(k); };
+    // list-key error bound (block rows: widened by kBlkErr)
+    auto err = [&](float k) { return BLK ? key_err_bound(k) + kBlkErr : key_err_bound(k); };
     bool complete;
     if (nvalid < kr)
         complete = theta_drop == kInf;
@@ -923,7 +927,7 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
 // ever waits for another and the kernel has no block-wide barrier.
 
 template <int DT, bool VERIFY, bool VEC, bool BLK>
-__global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(const RaceArgs a) {
+__global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RACE_MIN_BLOCKS) race_kernel(const RaceArgs a) {
     __shared__ uint32_t s_queue[kQueueCap];
     const int64_t NW = a.G;
     const int64_t gw = blockIdx.x;
@@ -948,9 +952,6 @@ __global__ void __launch_bounds__(kThreads, PPS_RACE_MIN_BLOCKS) race_kernel(con
         if constexpr (BLK) {
             bk.b = __ldg(a.row_block + r);
             bk.B = a.n_blocks;
-            bk.invB = 1.0f / (float)a.n_blocks;
-            bk.shift = a.block_shift;
-            bk.eb = kBlkErr;
         }
         WarpList L;
         L.reset(kp, kr);
