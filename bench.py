@@ -211,6 +211,8 @@ def main():
     ap.add_argument("--top-p", type=float, default=1.0, help="then to its top-p set (with --top-k)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--eager", action="store_true",
+                    help="tree workloads: launch every call from Python instead of replaying a CUDA graph")
     args = ap.parse_args()
 
     rank, world, local = dist_init()
@@ -533,29 +535,18 @@ def run_dynamic(args, rank, world, dev):
                 emitted=torch.empty(n_seq, W, dtype=torch.int32, device=dev),
                 score=torch.empty(n_seq, W, dtype=torch.float32, device=dev),
                 score_sum=torch.empty(n_seq, dtype=torch.float64, device=dev))
-    stream = torch.cuda.current_stream(dev)
-
     def step():
-        b.run(root_key, root_ctx, root_pos, lambda d, *_: q[d], stream=stream)
-        b.verify(p, ws=ws_v, out=vout, status=status, stream=stream)
+        b.run(root_key, root_ctx, root_pos, lambda d, *_: q[d])
+        b.verify(p, ws=ws_v, out=vout, status=status)
 
     for _ in range(max(3, args.warmup)):
         step()
     torch.cuda.synchronize(dev)
     assert int(status.item()) == 0, f"status flags {int(status.item())}"
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    clk = Clocks(dev.index or 0)
+    run = step if args.eager else graph_of(step, dev).replay
     barrier(world)
-    torch.cuda.synchronize(dev)
-    clk.start()
-    time.sleep(0.3)
-    e0.record(stream)
-    for _ in range(args.steps):
-        step()
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    clocks = clk.stop()
-    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
+    ms, clocks = timed_replays(run, args.steps, dev, Clocks(dev.index or 0))
+    ms = max_over_ranks(ms, world)
     rows = b.n_draft + b.n_nodes
     nbytes = rows * V * 2
     peak, peak_kind = _peaks()
@@ -569,7 +560,8 @@ def run_dynamic(args, rank, world, dev):
             "config": {"workload": f"dynamic IID tree: B={n_seq}, V={V}, K={K}, gamma={gamma}, "
                                    f"{b.n_nodes} node slots + {b.n_draft} draft rows per step",
                        "rows_per_step": rows, "l2": f"inputs ({nbytes / 1e9:.2f} GB) larger than L2, no flush",
-                       "parallelism": f"replicas x{world}"},
+                       "parallelism": f"replicas x{world}",
+                       "launch": "eager" if args.eager else "CUDA graph of the step's library calls"},
             "gb_per_s": gbs,
             "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
                          "traffic": None, "peak_kind": peak_kind, "algorithmic_bytes": nbytes},
@@ -577,6 +569,40 @@ def run_dynamic(args, rank, world, dev):
             "mean_accept_len": float(vout["accept_len"].float().mean().item()),
             "mean_draft_nodes_per_seq": float((b.row_k[:b.n_draft] > 0).sum().item()) / n_seq,
         }))
+
+
+def graph_of(fn, dev):
+    """Capture fn() (library calls on the current stream) into a CUDA graph, after warm-up
+    runs on the capture's side stream."""
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(torch.cuda.current_stream(dev))
+    with torch.cuda.stream(side):
+        for _ in range(3):
+            fn()
+    torch.cuda.current_stream(dev).wait_stream(side)
+    torch.cuda.synchronize(dev)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        fn()
+    torch.cuda.synchronize(dev)
+    return g
+
+
+def timed_replays(fn, steps, dev, clk=None):
+    """Mean device time of `steps` calls of fn on the current stream (CUDA events)."""
+    stream = torch.cuda.current_stream(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+    if clk is not None:
+        clk.start()
+        time.sleep(0.3)
+    e0.record(stream)
+    for _ in range(steps):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = clk.stop() if clk is not None else None
+    return e0.elapsed_time(e1) / steps, clocks
 
 
 def run_hetero(args, rank, world, dev):
@@ -615,38 +641,30 @@ def run_hetero(args, rank, world, dev):
                 emitted=torch.empty(n_seq, W, dtype=torch.int32, device=dev),
                 score=torch.empty(n_seq, W, dtype=torch.float32, device=dev),
                 score_sum=torch.empty(n_seq, dtype=torch.float64, device=dev))
-    stream = torch.cuda.current_stream(dev)
+    def draft():
+        b.run(root_key, root_ctx, root_pos, lambda d, *_: q[d])
 
-    def step(ev=None):
-        if ev is not None:
-            ev[0].record(stream)
-        b.run(root_key, root_ctx, root_pos, lambda d, *_: q[d], stream=stream)
-        if ev is not None:
-            ev[1].record(stream)
-        b.verify(p, ws=ws_v, out=vout, status=status, stream=stream)
-        if ev is not None:
-            ev[2].record(stream)
+    def verify():
+        b.verify(p, ws=ws_v, out=vout, status=status)
+
+    def step():
+        draft()
+        verify()
 
     for _ in range(max(3, args.warmup)):
         step()
     torch.cuda.synchronize(dev)
     assert int(status.item()) == 0, f"status flags {int(status.item())}"
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    clk = Clocks(dev.index or 0)
+    if args.eager:
+        run, run_d, run_v = step, draft, verify
+    else:
+        run, run_d, run_v = (graph_of(f, dev).replay for f in (step, draft, verify))
     barrier(world)
-    torch.cuda.synchronize(dev)
-    clk.start()
-    time.sleep(0.3)
-    e0.record(stream)
-    for k in range(args.steps):
-        step(evs[k])
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    clocks = clk.stop()
-    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
-    t_draft = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
-    t_verify = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    ms, clocks = timed_replays(run, args.steps, dev, Clocks(dev.index or 0))
+    ms = max_over_ranks(ms, world)
+    # the two phases alone (the draft phase: gamma proposal-row races + expansions)
+    t_draft, _ = timed_replays(run_d, args.steps, dev)
+    t_verify, _ = timed_replays(run_v, args.steps, dev)
     n_prop = gamma * n_seq * B
     rows = n_prop + b.n_nodes
     nbytes = rows * V * 2
@@ -665,7 +683,8 @@ def run_hetero(args, rank, world, dev):
             "config": {"workload": f"non-identical proposals: n_seq={n_seq}, V={V}, B={B} proposals, "
                                    f"gamma={gamma}, {n_prop} proposal rows + {b.n_nodes} node slots per step",
                        "rows_per_step": rows, "l2": f"inputs ({nbytes / 1e9:.2f} GB) larger than L2, no flush",
-                       "parallelism": f"replicas x{world}"},
+                       "parallelism": f"replicas x{world}",
+                       "launch": "eager" if args.eager else "CUDA graph of the step's library calls"},
             "gb_per_s": nbytes / (ms / 1e3) / 1e9,
             "roofline": {"bound": "alu", "achieved": mul_ach, "peak": mul_peak, "unit": "T wide-mul/s",
                          "frac": mul_ach / mul_peak, "traffic": None,
