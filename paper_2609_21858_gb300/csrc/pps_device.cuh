@@ -151,45 +151,6 @@ struct RowPhilox {
         }
         return make_uint4(x0, x1, x2, x3);
     }
-
-    // NB blocks at counters c0[b], computed round-major so that the NB
-    // independent multiply chains are interleaved instruction by instruction
-    template <int NB>
-    __device__ __forceinline__ void blocks(const uint32_t (&c0)[NB], uint4 (&out)[NB]) const {
-        uint32_t x0[NB], x1[NB], x2[NB], x3[NB];
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            uint32_t hi0, lo0;
-            mulhilo(kPhiloxM0, c0[b], hi0, lo0);
-            x3[b] = lo0;
-            x2[b] = hi0 ^ r1_c3k;
-        }
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            uint32_t h1, l1;
-            mulhilo(kPhiloxM1, x2[b], h1, l1);
-            x0[b] = h1 ^ r2_f;
-            x1[b] = l1;
-            x2[b] = x3[b] ^ r2_gh;
-            x3[b] = r2_lo0;
-        }
-#pragma unroll
-        for (int r = 0; r < 8; ++r) {
-#pragma unroll
-            for (int b = 0; b < NB; ++b) {
-                uint32_t a0, b0, a1, b1;
-                mulhilo(kPhiloxM0, x0[b], a0, b0);
-                mulhilo(kPhiloxM1, x2[b], a1, b1);
-                const uint32_t n0 = a1 ^ x1[b] ^ rk0[r], n2 = a0 ^ x3[b] ^ rk1[r];
-                x0[b] = n0;
-                x1[b] = b1;
-                x2[b] = n2;
-                x3[b] = b0;
-            }
-        }
-#pragma unroll
-        for (int b = 0; b < NB; ++b) out[b] = make_uint4(x0[b], x1[b], x2[b], x3[b]);
-    }
 };
 
 // ------------------------------------------------------------------ transforms
@@ -386,6 +347,13 @@ __device__ __forceinline__ bool filter_pass(uint32_t w, float l, float c, float 
 }
 __device__ __forceinline__ float filter_tz(float theta) {
     return theta + (kFilterMargin + kLog2Ln2 + kFilterScaleLog2);
+}
+
+// packed bf16 max (a NaN half yields the other operand's half)
+__device__ __forceinline__ uint32_t bf2_max(uint32_t a, uint32_t b) {
+    uint32_t r;
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
 }
 
 // bf16 -> fp32 (exact)

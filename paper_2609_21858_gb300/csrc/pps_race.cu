@@ -34,8 +34,8 @@
 #ifndef PPS_PREFETCH
 #define PPS_PREFETCH 0  // 1: load the next iteration's vectors one iteration ahead (costs registers)
 #endif
-#ifndef PPS_INTERLEAVE
-#define PPS_INTERLEAVE 0  // 1: Philox blocks of an iteration computed round-major
+#ifndef PPS_VECFILTER
+#define PPS_VECFILTER 1  // 1: one filter test per 16-byte vector on verify rows and fp32 rows
 #endif
 #ifndef PPS_PACKED
 #define PPS_PACKED 0  // 1: pairs of filter sums with packed fp32x2 fma/add
@@ -520,7 +520,10 @@ __device__ __forceinline__ float block_filter_max(const uint4& w, const float (&
 // no calls: it returns the iteration after which the queue holds 32 or more
 // blocks (n_it when it ran to the end), so that nothing it keeps in
 // registers (the row's round keys above all) lives across a call.
-template <int DT>
+// VF: test each 16-byte vector once (verify rows, where one key is kept, and
+// fp32 rows); otherwise each Philox block's four tokens (the vector test
+// passes up to 8x more often under the looser bound of a K-list).
+template <int DT, bool VF>
 __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* row, int64_t v0, int64_t it0,
                                              int64_t n_it, float c, float tz, uint32_t* q, int& qn) {
     constexpr int NB = 2 * PPS_UNITS;          // Philox blocks per lane per iteration
@@ -550,27 +553,40 @@ __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* ro
         p += STEP;
 #endif
         unsigned bm = 0;
-#if PPS_INTERLEAVE
-        uint32_t cb[NB];
-        uint4 wb[NB];
+        if constexpr (VF && PPS_VECFILTER) {
+            // One test per 16-byte vector: the filter sum rises with the word and
+            // the logit, so the vector's largest word with its largest logit
+            // passes whenever one of its tokens would; the ex2 error is taken at
+            // the larger argument, as in the per-token test, so the same margin
+            // covers it.  A passing vector queues its Philox blocks for the
+            // per-token test.
 #pragma unroll
-        for (int b = 0; b < NB; ++b) cb[b] = cl + block_offset<DT>(b);
-        rp.blocks<NB>(cb, wb);
+            for (int k = 0; k < ND; ++k) {
+                if constexpr (DT == 1) {
+                    const uint4 w0 = rp.block(cl + block_offset<DT>(2 * k));
+                    const uint4 w1 = rp.block(cl + block_offset<DT>(2 * k + 1));
+                    const uint32_t wm =
+                        max(max(max(w0.x, w0.y), max(w0.z, w0.w)), max(max(w1.x, w1.y), max(w1.z, w1.w)));
+                    const uint32_t m2 = bf2_max(bf2_max(d[k].x, d[k].y), bf2_max(d[k].z, d[k].w));
+                    const float lm = fmaxf(bf16_lo(m2), bf16_hi(m2));
+                    bm |= (filter_pass(wm, lm, c, tz) ? 3u : 0u) << (2 * k);
+                } else {
+                    const uint4 w = rp.block(cl + block_offset<DT>(k));
+                    const uint32_t wm = max(max(w.x, w.y), max(w.z, w.w));
+                    const float lm = fmaxf(fmaxf(__uint_as_float(d[k].x), __uint_as_float(d[k].y)),
+                                           fmaxf(__uint_as_float(d[k].z), __uint_as_float(d[k].w)));
+                    bm |= (filter_pass(wm, lm, c, tz) ? 1u : 0u) << k;
+                }
+            }
+        } else {
 #pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            float l[4];
-            block_logits<DT>(d, b, l);
-            bm |= (unsigned)(block_filter_max(wb[b], l, c, tz) >= kFilterCut) << b;
+            for (int b = 0; b < NB; ++b) {
+                const uint4 w = rp.block(cl + block_offset<DT>(b));
+                float l[4];
+                block_logits<DT>(d, b, l);
+                bm |= (unsigned)(block_filter_max(w, l, c, tz) >= kFilterCut) << b;
+            }
         }
-#else
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            const uint4 w = rp.block(cl + block_offset<DT>(b));
-            float l[4];
-            block_logits<DT>(d, b, l);
-            bm |= (unsigned)(block_filter_max(w, l, c, tz) >= kFilterCut) << b;
-        }
-#endif
         if (__any_sync(FULL, bm != 0)) {
             // append this lane's flagged blocks at its offset in the warp's batch
             const int n = __popc(bm);
@@ -595,7 +611,7 @@ __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* ro
 
 // Stream vectors [v0, v1) of one row through the warp's list: full
 // iterations through the fast loop, the rest through the scalar tail.
-template <int DT, bool VEC, bool BLK>
+template <int DT, bool VEC, bool BLK, bool VF>
 __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int64_t V, int64_t v0, int64_t v1,
                                                float c, uint64_t key, uint64_t ctx, uint32_t pos, uint32_t* q,
                                                const Blk& bk) {
@@ -613,7 +629,7 @@ __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int
         while (it < n_it) {
             RowPhilox rp;
             rp.init(key, ctx, pos);
-            it = fast_scan<DT>(rp, row, v0, it, n_it, c, st.L.tz, q, qn);
+            it = fast_scan<DT, VF>(rp, row, v0, it, n_it, c, st.L.tz, q, qn);
             if (qn > 0) st = flush_queue<DT, BLK>(st, q, qn, row, c, key, ctx, pos, bk);
             qn = 0;
         }
@@ -955,7 +971,7 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
         }
         WarpList L;
         L.reset(kp, kr);
-        stream_segment<DT, VEC, BLK>(L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk);
+        stream_segment<DT, VEC, BLK, VERIFY || DT == 0>(L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk);
 
         finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk);
     }

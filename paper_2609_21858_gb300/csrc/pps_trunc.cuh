@@ -212,12 +212,6 @@ __device__ __forceinline__ void top_offer(TopList& L, float (&cv)[N], const int 
 
 // ---------------------------------------------------------------- vector helpers
 
-__device__ __forceinline__ uint32_t bf2_max(uint32_t a, uint32_t b) {
-    uint32_t r;
-    asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));  // a NaN half yields the other operand's half
-    return r;
-}
-
 // any half of the bf16 pair m >= the bf16 pair t2 (NaN halves compare false)
 __device__ __forceinline__ bool bf2_any_ge(uint32_t m, uint32_t t2) {
     uint32_t r;
