@@ -29,7 +29,10 @@
 #include "pps_internal.h"
 
 #ifndef PPS_UNITS
-#define PPS_UNITS 3  // 8-token units per lane per fast-loop iteration (2 Philox blocks each)
+#define PPS_UNITS 3  // 8-token units per lane per fast-loop iteration (2 Philox blocks each), draft rows
+#endif
+#ifndef PPS_UNITS_VERIFY
+#define PPS_UNITS_VERIFY 4  // the same for verify rows
 #endif
 #ifndef PPS_PREFETCH
 #define PPS_PREFETCH 0  // 1: load the next iteration's vectors one iteration ahead (costs registers)
@@ -354,8 +357,9 @@ struct SlowState {
 };
 
 // Blocks flagged by the fast scan wait in a per-warp queue of Philox block
-// counters in shared memory (one iteration adds at most 32 x 2 x PPS_UNITS).
-constexpr int kQueueCap = 32 + 32 * 2 * PPS_UNITS;
+// counters in shared memory (one iteration adds at most 32 x 2 x units).
+constexpr int kMaxUnits = PPS_UNITS > PPS_UNITS_VERIFY ? PPS_UNITS : PPS_UNITS_VERIFY;
+constexpr int kQueueCap = 32 + 32 * 2 * kMaxUnits;
 
 // Work off the queue: lane j regenerates the words of queued block j (32 at
 // a time), reloads its four logits, keys the tokens over the filter cut and
@@ -511,10 +515,10 @@ __device__ __forceinline__ float block_filter_max(const uint4& w, const float (&
 }
 
 // Fast scan over iterations [it0, n_it) of the full vectors starting at
-// vector v0 of a row.  Each iteration covers PPS_UNITS x 32 (bf16) or x 64
-// (fp32) vectors; every lane takes PPS_UNITS units of 8 tokens = 2 x
-// PPS_UNITS Philox blocks with counters cl + block_offset(b), cl advancing by
-// 64 x PPS_UNITS, so that many independent multiply chains are in flight per
+// vector v0 of a row.  Each iteration covers U x 32 (bf16) or x 64 (fp32)
+// vectors; every lane takes U units of 8 tokens = 2 x U Philox blocks with
+// counters cl + block_offset(b), cl advancing by 64 x U, so that many
+// independent multiply chains are in flight per
 // lane.  A lane keeps only the per-block maxima of the filter sums; a block
 // with a token over the cut is appended to the warp's queue.  The scan makes
 // no calls: it returns the iteration after which the queue holds 32 or more
@@ -523,15 +527,15 @@ __device__ __forceinline__ float block_filter_max(const uint4& w, const float (&
 // VF: test each 16-byte vector once (verify rows, where one key is kept, and
 // fp32 rows); otherwise each Philox block's four tokens (the vector test
 // passes up to 8x more often under the looser bound of a K-list).
-template <int DT, bool VF>
+template <int DT, bool VF, int U>
 __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* row, int64_t v0, int64_t it0,
                                              int64_t n_it, float c, float tz, uint32_t* q, int& qn) {
-    constexpr int NB = 2 * PPS_UNITS;          // Philox blocks per lane per iteration
+    constexpr int NB = 2 * U;                  // Philox blocks per lane per iteration
     constexpr int ND = DT == 1 ? NB / 2 : NB;  // 16-byte vectors per lane per iteration
     constexpr int STEP = 32 * ND;              // vectors per iteration
     const int lane = threadIdx.x & 31;
     const uint4* p = reinterpret_cast<const uint4*>(row) + v0 + it0 * STEP + lane;
-    uint32_t cl = (DT == 1 ? (uint32_t)(2 * (v0 + lane)) : (uint32_t)(v0 + lane)) + (uint32_t)(it0 * 64 * PPS_UNITS);
+    uint32_t cl = (DT == 1 ? (uint32_t)(2 * (v0 + lane)) : (uint32_t)(v0 + lane)) + (uint32_t)(it0 * 64 * U);
 #if PPS_PREFETCH
     uint4 nx[ND];
 #pragma unroll
@@ -604,19 +608,19 @@ __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* ro
             qn += total;
             if (qn >= 32) return it + 1;
         }
-        cl += 64 * PPS_UNITS;
+        cl += 64 * U;
     }
     return n_it;
 }
 
 // Stream vectors [v0, v1) of one row through the warp's list: full
 // iterations through the fast loop, the rest through the scalar tail.
-template <int DT, bool VEC, bool BLK, bool VF>
+template <int DT, bool VEC, bool BLK, bool VF, int U>
 __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int64_t V, int64_t v0, int64_t v1,
                                                float c, uint64_t key, uint64_t ctx, uint32_t pos, uint32_t* q,
                                                const Blk& bk) {
     constexpr int VW = DT == 1 ? 8 : 4;
-    constexpr int STEP = (DT == 1 ? 32 : 64) * PPS_UNITS;  // vectors per fast-loop iteration
+    constexpr int STEP = (DT == 1 ? 32 : 64) * U;  // vectors per fast-loop iteration
     const int64_t nfull = V / VW;                           // vectors holding VW tokens
     const int64_t vend = VEC ? min(v1, nfull) : v0;
     const int64_t n_it = vend > v0 ? (vend - v0) / STEP : 0;
@@ -629,7 +633,7 @@ __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int
         while (it < n_it) {
             RowPhilox rp;
             rp.init(key, ctx, pos);
-            it = fast_scan<DT, VF>(rp, row, v0, it, n_it, c, st.L.tz, q, qn);
+            it = fast_scan<DT, VF, U>(rp, row, v0, it, n_it, c, st.L.tz, q, qn);
             if (qn > 0) st = flush_queue<DT, BLK>(st, q, qn, row, c, key, ctx, pos, bk);
             qn = 0;
         }
@@ -971,7 +975,8 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
         }
         WarpList L;
         L.reset(kp, kr);
-        stream_segment<DT, VEC, BLK, VERIFY || DT == 0>(L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk);
+        stream_segment<DT, VEC, BLK, VERIFY || DT == 0, VERIFY ? PPS_UNITS_VERIFY : PPS_UNITS>(
+            L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk);
 
         finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk);
     }
