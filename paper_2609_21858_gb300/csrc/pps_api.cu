@@ -14,7 +14,7 @@ namespace pps {
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 size_t workspace_bytes(int64_t n_rows, int32_t n_seq) {
-    return align256(kSlotBytes * (size_t)(n_rows + (int64_t)kGridMax)) + align256(sizeof(uint32_t) * (size_t)n_rows) +
+    return align256(kSlotBytes * (size_t)(n_rows + (int64_t)kGridMax)) + align256(sizeof(uint32_t) * 2 * (size_t)n_rows) +
            align256(sizeof(uint32_t) * (size_t)(n_seq > 0 ? n_seq : 0));
 }
 
@@ -23,8 +23,8 @@ void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials
     char* p = static_cast<char*>(ws);
     *partials = reinterpret_cast<Partial*>(p);
     p += align256(kSlotBytes * (size_t)(n_rows + (int64_t)kGridMax));
-    *row_cnt = reinterpret_cast<uint32_t*>(p);
-    p += align256(sizeof(uint32_t) * (size_t)n_rows);
+    *row_cnt = reinterpret_cast<uint32_t*>(p);  // [n_rows] arrival counters, then [n_rows] shared row bounds
+    p += align256(sizeof(uint32_t) * 2 * (size_t)n_rows);
     *seq_cnt = reinterpret_cast<uint32_t*>(p);
 }
 
@@ -72,7 +72,7 @@ static RaceArgs base_args(const void* logits, pps_dtype dtype, int64_t n_rows, i
 // device address; the address is looked up per device with
 // cudaGetSymbolAddress and cached.
 constexpr size_t kNoAllocPartialBytes = sizeof(Partial) * (size_t)(PPS_NOALLOC_MAX_ROWS + PPS_NOALLOC_MAX_WARPS);
-constexpr size_t kNoAllocCounterBytes = sizeof(uint32_t) * (size_t)PPS_NOALLOC_MAX_ROWS;
+constexpr size_t kNoAllocCounterBytes = sizeof(uint32_t) * 2 * (size_t)PPS_NOALLOC_MAX_ROWS;
 constexpr size_t kNoAllocScratchBytes = kNoAllocPartialBytes + kNoAllocCounterBytes;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
@@ -158,6 +158,7 @@ static pps_status draft_list(const void* q_logits, pps_dtype dtype, int64_t n_ro
     a.out_samples = out_samples;
     a.status = status;
     workspace_carve(ws, n_rows, 0, &a.partials, &a.row_cnt, &a.seq_cnt);
+    a.row_bound = a.row_cnt + n_rows;
     a.tpartials = reinterpret_cast<TruncPartial*>(a.partials);
     a.top_k = top_k;
     a.top_p = top_p;
@@ -230,6 +231,7 @@ static pps_status verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_n
     a.out_ss = out_score_sum;
     a.status = status;
     workspace_carve(ws, n_nodes, n_seq, &a.partials, &a.row_cnt, &a.seq_cnt);
+    a.row_bound = a.row_cnt + n_nodes;
     a.tpartials = reinterpret_cast<TruncPartial*>(a.partials);
     a.top_k = top_k;
     a.top_p = top_p;
@@ -292,8 +294,8 @@ pps_status pps_draft_list_noalloc(const void* q_logits, pps_dtype dtype, int64_t
     if (st != PPS_OK) return st;
     char* base = static_cast<char*>(scratch);
     uint32_t* row_cnt = reinterpret_cast<uint32_t*>(base + kNoAllocPartialBytes);
-    // the arrival counters must start at zero; the partial lists need no clearing
-    if (cudaMemsetAsync(row_cnt, 0, sizeof(uint32_t) * (size_t)n_rows, (cudaStream_t)stream) != cudaSuccess)
+    // the arrival counters and shared row bounds must start at zero; the partial lists need no clearing
+    if (cudaMemsetAsync(row_cnt, 0, sizeof(uint32_t) * 2 * (size_t)n_rows, (cudaStream_t)stream) != cudaSuccess)
         return PPS_ERR_CUDA;
     RaceArgs a = base_args(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature);
     a.K = K;
@@ -307,6 +309,7 @@ pps_status pps_draft_list_noalloc(const void* q_logits, pps_dtype dtype, int64_t
     a.status = status;
     a.partials = reinterpret_cast<Partial*>(base);
     a.row_cnt = row_cnt;
+    a.row_bound = row_cnt + n_rows;
     a.seq_cnt = nullptr;
     const int dt = dtype == PPS_BF16 ? 1 : 0;
     const bool vec = vec_ok(q_logits, dtype, row_stride);
@@ -395,6 +398,7 @@ pps_status pps_draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_row
         a.n_blocks = n_blocks;
     }
     workspace_carve(ws, n_rows, 0, &a.partials, &a.row_cnt, &a.seq_cnt);
+    a.row_bound = a.row_cnt + n_rows;
     const int dt = dtype == PPS_BF16 ? 1 : 0;
     const bool vec = vec_ok(q_logits, dtype, row_stride);
     a.G = race_grid(a.total, dt, false, vec, n_blocks > 1);

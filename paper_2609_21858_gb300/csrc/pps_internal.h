@@ -80,6 +80,7 @@ struct RaceArgs {
     Partial* partials;   // [n_rows + kGridMax]: slot (warp + row)
     TruncPartial* tpartials;  // the same slots, for the truncated race
     uint32_t* row_cnt;   // [n_rows]
+    uint32_t* row_bound; // [n_rows] shared filter bound of a row cut between warps (0 = none)
     uint32_t* seq_cnt;   // [n_seq]
 };
 

@@ -37,6 +37,9 @@
 #ifndef PPS_PREFETCH
 #define PPS_PREFETCH 0  // 1: load the next iteration's vectors one iteration ahead (costs registers)
 #endif
+#ifndef PPS_ROWBOUND
+#define PPS_ROWBOUND 1  // 1: warps that share a row share its filter bound through the workspace
+#endif
 #ifndef PPS_VECFILTER
 #define PPS_VECFILTER 1  // 1: one filter test per 16-byte vector on verify rows and fp32 rows
 #endif
@@ -54,6 +57,18 @@ namespace pps {
 
 #define FULL 0xffffffffu
 constexpr float kInf = __builtin_huge_valf();
+
+// Shared row bound: a float kept as ~(order-preserving bits), so that atomicMax
+// keeps the smallest bound and the zeroed word reads as none (+inf).
+__device__ __forceinline__ uint32_t bound_enc(float f) {
+    const uint32_t b = __float_as_uint(f);
+    return ~((b & 0x80000000u) ? ~b : (b | 0x80000000u));
+}
+__device__ __forceinline__ float bound_dec(uint32_t e) {
+    if (e == 0u) return kInf;
+    const uint32_t o = ~e;
+    return __uint_as_float((o & 0x80000000u) ? (o & 0x7fffffffu) : ~o);
+}
 
 __device__ __forceinline__ bool lex_less(float ak, int ai, float bk, int bi) {
     return ak < bk || (ak == bk && ai < bi);
@@ -265,6 +280,14 @@ struct WarpList {
     }
 };
 
+// Publish filter_slack of the list's k-th key (widened by eb) as a filter bound
+// for every warp of the row: the row's k-th key is at most this list's, so
+// the bound passes the completeness test of any segment that adopts it.
+__device__ __forceinline__ void publish_bound(uint32_t* slot, const WarpList& L, float eb, int lane) {
+    const float pub = filter_slack(__shfl_sync(FULL, L.lk, L.k - 1)) + eb * 4.0f;
+    if (lane == 0 && pub < kInf) atomicMax(slot, bound_enc(pub));
+}
+
 // Offer the keyed survivors of one lane (pk[e] for token i0 + e, +inf = none)
 // to the warp list: each round every lane offers its smallest remaining key
 // below the threshold; up to three offers are inserted one by one, more are
@@ -318,7 +341,7 @@ __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], in
 template <bool BLK>
 __device__ __forceinline__ void block_survivors(WarpList& L, const RowPhilox& rp, bool mine, uint32_t cb,
                                                 const float (&l)[4], unsigned valid, float c, int lane, const Blk& bk,
-                                                uint64_t key, uint64_t ctx, uint32_t pos) {
+                                                uint64_t key, uint64_t ctx, uint32_t pos, uint32_t* slot) {
     float pk[4] = {kInf, kInf, kInf, kInf};
     if (mine) {
         const uint4 q = rp.block(cb);
@@ -348,6 +371,7 @@ __device__ __forceinline__ void block_survivors(WarpList& L, const RowPhilox& rp
         }
     }
     offer_survivors<4>(L, pk, (int64_t)4 * cb, lane, BLK ? bk.shift() : 0.f, BLK ? kBlkErr : 0.f);
+    if (slot != nullptr) publish_bound(slot, L, BLK ? kBlkErr : 0.f, lane);
 }
 
 // ---------------------------------------------------------------- rare paths (out of line)
@@ -366,7 +390,7 @@ constexpr int kQueueCap = 32 + 32 * 2 * kMaxUnits;
 // offers them.  Out of line; the fast scan itself makes no calls.
 template <int DT, bool BLK>
 __device__ __noinline__ SlowState flush_queue(SlowState st, const uint32_t* q, int qn, const char* row, float c,
-                                              uint64_t key, uint64_t ctx, uint32_t pos, Blk bk) {
+                                              uint64_t key, uint64_t ctx, uint32_t pos, Blk bk, uint32_t* slot) {
     const int lane = threadIdx.x & 31;
     RowPhilox rp;
     rp.init(key, ctx, pos);
@@ -390,7 +414,7 @@ __device__ __noinline__ SlowState flush_queue(SlowState st, const uint32_t* q, i
                 l[3] = __uint_as_float(v.w);
             }
         }
-        block_survivors<BLK>(st.L, rp, mine, cb, l, 0xfu, c, lane, bk, key, ctx, pos);
+        block_survivors<BLK>(st.L, rp, mine, cb, l, 0xfu, c, lane, bk, key, ctx, pos, slot);
     }
     __syncwarp();
     return st;
@@ -402,7 +426,7 @@ __device__ __noinline__ SlowState flush_queue(SlowState st, const uint32_t* q, i
 template <int DT, bool BLK = false>
 __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64_t V, int64_t base, int64_t v1,
                                             float c, uint64_t key, uint64_t ctx, uint32_t pos, float floor,
-                                            Blk bk = Blk{}) {
+                                            Blk bk = Blk{}, uint32_t* slot = nullptr) {
     constexpr int VW = DT == 1 ? 8 : 4;
     const int lane = threadIdx.x & 31;
     RowPhilox rp;
@@ -435,7 +459,8 @@ __device__ __noinline__ SlowState tail_loop(SlowState st, const char* row, int64
 #pragma unroll
                 for (int e = 0; e < 4; ++e) pass |= ((vh >> e) & 1u) && filter_pass(wq[e], l[e], c, st.L.tz);
             }
-            if (__any_sync(FULL, pass)) block_survivors<BLK>(st.L, rp, pass, cb, l, vh, c, lane, bk, key, ctx, pos);
+            if (__any_sync(FULL, pass))
+                block_survivors<BLK>(st.L, rp, pass, cb, l, vh, c, lane, bk, key, ctx, pos, slot);
         }
     }
     return st;
@@ -527,9 +552,13 @@ __device__ __forceinline__ float block_filter_max(const uint4& w, const float (&
 // VF: test each 16-byte vector once (verify rows, where one key is kept, and
 // fp32 rows); otherwise each Philox block's four tokens (the vector test
 // passes up to 8x more often under the looser bound of a K-list).
+// slot (nullable): the row's shared bound, read every iteration; a smaller one
+// lowers the filter threshold and is returned in tfa (the caller records it as
+// this segment's drop bound).
 template <int DT, bool VF, int U>
 __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* row, int64_t v0, int64_t it0,
-                                             int64_t n_it, float c, float tz, uint32_t* q, int& qn) {
+                                             int64_t n_it, float c, float tz, uint32_t* q, int& qn,
+                                             const uint32_t* slot, float shift, float& tfa) {
     constexpr int NB = 2 * U;                  // Philox blocks per lane per iteration
     constexpr int ND = DT == 1 ? NB / 2 : NB;  // 16-byte vectors per lane per iteration
     constexpr int STEP = 32 * ND;              // vectors per iteration
@@ -556,6 +585,8 @@ __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* ro
         for (int k = 0; k < ND; ++k) d[k] = ldg_stream(p + 32 * k);
         p += STEP;
 #endif
+        uint32_t shared_bound = 0u;
+        if (slot != nullptr) asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(shared_bound) : "l"(slot));
         unsigned bm = 0;
         if constexpr (VF && PPS_VECFILTER) {
             // One test per 16-byte vector: the filter sum rises with the word and
@@ -591,6 +622,13 @@ __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* ro
                 bm |= (unsigned)(block_filter_max(w, l, c, tz) >= kFilterCut) << b;
             }
         }
+        if (slot != nullptr) {
+            const float g = bound_dec(shared_bound);
+            if (g < tfa) {
+                tfa = g;
+                tz = filter_tz(g + shift);
+            }
+        }
         if (__any_sync(FULL, bm != 0)) {
             // append this lane's flagged blocks at its offset in the warp's batch
             const int n = __popc(bm);
@@ -618,7 +656,7 @@ __device__ __forceinline__ int64_t fast_scan(const RowPhilox& rp, const char* ro
 template <int DT, bool VEC, bool BLK, bool VF, int U>
 __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int64_t V, int64_t v0, int64_t v1,
                                                float c, uint64_t key, uint64_t ctx, uint32_t pos, uint32_t* q,
-                                               const Blk& bk) {
+                                               const Blk& bk, uint32_t* slot) {
     constexpr int VW = DT == 1 ? 8 : 4;
     constexpr int STEP = (DT == 1 ? 32 : 64) * U;  // vectors per fast-loop iteration
     const int64_t nfull = V / VW;                           // vectors holding VW tokens
@@ -627,19 +665,24 @@ __device__ __forceinline__ void stream_segment(WarpList& L, const char* row, int
     SlowState st{L};
     int64_t base = v0;
     if (n_it > 0) {
-        st.L.bound(seed_theta<DT, BLK>(row, v0, c, key, ctx, pos, st.L.k, bk), BLK ? bk.shift() : 0.f);
+        const float shift = BLK ? bk.shift() : 0.f;
+        const float seed = seed_theta<DT, BLK>(row, v0, c, key, ctx, pos, st.L.k, bk);
+        st.L.bound(seed, shift);
+        if (slot != nullptr && (threadIdx.x & 31) == 0 && seed < kInf) atomicMax(slot, bound_enc(seed));
         int64_t it = 0;
         int qn = 0;
         while (it < n_it) {
             RowPhilox rp;
             rp.init(key, ctx, pos);
-            it = fast_scan<DT, VF, U>(rp, row, v0, it, n_it, c, st.L.tz, q, qn);
-            if (qn > 0) st = flush_queue<DT, BLK>(st, q, qn, row, c, key, ctx, pos, bk);
+            float tfa = st.L.tf;
+            it = fast_scan<DT, VF, U>(rp, row, v0, it, n_it, c, st.L.tz, q, qn, slot, shift, tfa);
+            st.L.bound(tfa, shift);
+            if (qn > 0) st = flush_queue<DT, BLK>(st, q, qn, row, c, key, ctx, pos, bk, slot);
             qn = 0;
         }
         base = v0 + n_it * STEP;
     }
-    if (base < v1) st = tail_loop<DT, BLK>(st, row, V, base, v1, c, key, ctx, pos, -kInf, bk);
+    if (base < v1) st = tail_loop<DT, BLK>(st, row, V, base, v1, c, key, ctx, pos, -kInf, bk, slot);
     L = st.L;
 }
 
@@ -917,7 +960,10 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
         if (lane == 0) {
             unsigned t = atomicAdd(a.row_cnt + r, 1u);
             last = t == (unsigned)(last_w - first_w);
-            if (last) a.row_cnt[r] = 0u;
+            if (last) {
+                a.row_cnt[r] = 0u;
+                if (a.row_bound) a.row_bound[r] = 0u;
+            }
         }
         final_here = __shfl_sync(FULL, last, 0) != 0;
         if (final_here) {
@@ -975,8 +1021,13 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
         }
         WarpList L;
         L.reset(kp, kr);
+        // a row cut between warps shares its filter bound (verify and proposal rows: on K-list
+        // draft rows the extra registers cost more occupancy than the shared bound saves)
+        uint32_t* slot = nullptr;
+        if constexpr (PPS_ROWBOUND && (VERIFY || BLK))
+            if (a.row_bound && (v0 > 0 || v1 < nv)) slot = a.row_bound + r;
         stream_segment<DT, VEC, BLK, VERIFY || DT == 0, VERIFY ? PPS_UNITS_VERIFY : PPS_UNITS>(
-            L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk);
+            L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk, slot);
 
         finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk);
     }
