@@ -641,11 +641,13 @@ def run_hetero(args, rank, world, dev):
                 emitted=torch.empty(n_seq, W, dtype=torch.int32, device=dev),
                 score=torch.empty(n_seq, W, dtype=torch.float32, device=dev),
                 score_sum=torch.empty(n_seq, dtype=torch.float64, device=dev))
+    tk, tp = args.top_k, args.top_p
+
     def draft():
-        b.run(root_key, root_ctx, root_pos, lambda d, *_: q[d])
+        b.run(root_key, root_ctx, root_pos, lambda d, *_: q[d], top_k=tk, top_p=tp)
 
     def verify():
-        b.verify(p, ws=ws_v, out=vout, status=status)
+        b.verify(p, ws=ws_v, out=vout, status=status, top_k=tk, top_p=tp)
 
     def step():
         draft()
@@ -674,6 +676,19 @@ def run_hetero(args, rank, world, dev):
     mul_peak = sms * WIDE_MULS_PER_SM_CLK * hz / 1e12
     tok_draft = n_prop * V
     mul_ach = tok_draft * WIDE_MULS_PER_TOKEN / (t_draft / 1e3) / 1e12
+    trunc = f", top-k {tk}, top-p {tp}" if tk > 0 else ""
+    roof = {"bound": "alu", "achieved": mul_ach, "peak": mul_peak, "unit": "T wide-mul/s",
+            "frac": mul_ach / mul_peak, "traffic": None,
+            "kernel": "race_kernel, proposal rows (pps_draft_hetero) incl. the expansions", "ms": t_draft,
+            "peak_kind": f"derived: {sms} SMs x {WIDE_MULS_PER_SM_CLK} 32x32->64 multiplies/clk x "
+                         f"{hz / 1e6:.0f} MHz (median sampled SM clock)",
+            "work": f"{WIDE_MULS_PER_TOKEN} wide multiplies per token x {tok_draft} tokens"}
+    if tk > 0:
+        # truncated rows: the scan keys no token outside the top-k set, so HBM bounds it
+        gbs_d = n_prop * V * 2 / (t_draft / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": gbs_d, "peak": peak, "unit": "GB/s", "frac": gbs_d / peak,
+                "traffic": None, "kernel": "trunc_kernel, proposal rows (pps_draft_hetero_trunc) incl. the expansions",
+                "ms": t_draft, "peak_kind": peak_kind, "algorithmic_bytes": n_prop * V * 2}
     if rank == 0:
         print(json.dumps({
             "metric": METRIC, "value": rows * world / (ms / 1e3), "unit": "rows/s", "n_gpus": world,
@@ -681,18 +696,12 @@ def run_hetero(args, rank, world, dev):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded Zipf-rank logits; no model, no dataset)",
             "config": {"workload": f"non-identical proposals: n_seq={n_seq}, V={V}, B={B} proposals, "
-                                   f"gamma={gamma}, {n_prop} proposal rows + {b.n_nodes} node slots per step",
+                                   f"gamma={gamma}, {n_prop} proposal rows + {b.n_nodes} node slots per step{trunc}",
                        "rows_per_step": rows, "l2": f"inputs ({nbytes / 1e9:.2f} GB) larger than L2, no flush",
                        "parallelism": f"replicas x{world}",
                        "launch": "eager" if args.eager else "CUDA graph of the step's library calls"},
             "gb_per_s": nbytes / (ms / 1e3) / 1e9,
-            "roofline": {"bound": "alu", "achieved": mul_ach, "peak": mul_peak, "unit": "T wide-mul/s",
-                         "frac": mul_ach / mul_peak, "traffic": None,
-                         "kernel": "race_kernel, proposal rows (pps_draft_hetero) incl. the expansions",
-                         "ms": t_draft,
-                         "peak_kind": f"derived: {sms} SMs x {WIDE_MULS_PER_SM_CLK} 32x32->64 multiplies/clk x "
-                                      f"{hz / 1e6:.0f} MHz (median sampled SM clock)",
-                         "work": f"{WIDE_MULS_PER_TOKEN} wide multiplies per token x {tok_draft} tokens"},
+            "roofline": roof,
             "roofline_hbm": {"bound": "hbm", "achieved_draft": n_prop * V * 2 / (t_draft / 1e3) / 1e9,
                              "achieved_verify": b.n_nodes * V * 2 / (t_verify / 1e3) / 1e9, "peak": peak,
                              "peak_kind": peak_kind, "ms_verify": t_verify},

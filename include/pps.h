@@ -79,7 +79,8 @@ const char* pps_status_string(pps_status s);
 
 /* Bytes of workspace pps_draft_list / pps_verify_tree need for n_rows rows and
  * n_seq sequences (n_seq = 0 for pps_draft_list).  The workspace holds
- * per-row partial candidate lists and arrival counters; it must be zeroed once
+ * per-row partial candidate lists, arrival counters and the shared filter
+ * bounds of rows cut between CTAs; it must be zeroed once
  * before its first use (pps_workspace_clear or cudaMemset) and is left zeroed
  * by every call that returns PPS_OK and runs to completion.  One workspace
  * must not be used by two calls that run concurrently. */
@@ -265,6 +266,17 @@ pps_status pps_draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_row
                             pps_row_ids ids, float temperature, const int32_t* row_block, int32_t n_blocks,
                             int32_t* out_tok, float* out_key, uint32_t* status, void* ws, size_t ws_bytes,
                             pps_stream_t stream);
+
+/*
+ * pps_draft_hetero_trunc -- pps_draft_hetero with the logit processing of the
+ * truncated calls (top_k, top_p as pps_draft_list_trunc) applied to each
+ * proposal row before its race: proposal b races its truncated Q_b over
+ * block b.  PPS_ERR_INVALID_ARG for top_k or top_p out of range.
+ */
+pps_status pps_draft_hetero_trunc(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab,
+                                  int64_t row_stride, pps_row_ids ids, float temperature, int32_t top_k, float top_p,
+                                  const int32_t* row_block, int32_t n_blocks, int32_t* out_tok, float* out_key,
+                                  uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream);
 
 /*
  * pps_hetero_expand -- one depth of the draft tree of B proposals, each

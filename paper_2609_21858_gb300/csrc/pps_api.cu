@@ -377,10 +377,10 @@ pps_status pps_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t dept
     return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
 }
 
-pps_status pps_draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t row_stride,
-                            pps_row_ids ids, float temperature, const int32_t* row_block, int32_t n_blocks,
-                            int32_t* out_tok, float* out_key, uint32_t* status, void* ws, size_t ws_bytes,
-                            pps_stream_t stream) {
+static pps_status draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab,
+                               int64_t row_stride, pps_row_ids ids, float temperature, int32_t top_k, float top_p,
+                               const int32_t* row_block, int32_t n_blocks, int32_t* out_tok, float* out_key,
+                               uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream) {
     pps_status st = check_rows(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature);
     if (st != PPS_OK) return st;
     if (n_blocks < 1 || n_blocks > PPS_MAX_BLOCKS) return PPS_ERR_INVALID_ARG;
@@ -399,10 +399,38 @@ pps_status pps_draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_row
     }
     workspace_carve(ws, n_rows, 0, &a.partials, &a.row_cnt, &a.seq_cnt);
     a.row_bound = a.row_cnt + n_rows;
+    a.tpartials = reinterpret_cast<TruncPartial*>(a.partials);
+    a.top_k = top_k;
+    a.top_p = top_p;
     const int dt = dtype == PPS_BF16 ? 1 : 0;
     const bool vec = vec_ok(q_logits, dtype, row_stride);
-    a.G = race_grid(a.total, dt, false, vec, n_blocks > 1);
-    return launch_race(a, dt, false, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+    cudaError_t e;
+    if (top_k > 0) {
+        a.G = trunc_grid(a.total, a.n_rows, dt, false, vec, n_blocks > 1);
+        e = launch_trunc(a, dt, false, vec, (cudaStream_t)stream);
+    } else {
+        a.G = race_grid(a.total, dt, false, vec, n_blocks > 1);
+        e = launch_race(a, dt, false, vec, (cudaStream_t)stream);
+    }
+    return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+pps_status pps_draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab, int64_t row_stride,
+                            pps_row_ids ids, float temperature, const int32_t* row_block, int32_t n_blocks,
+                            int32_t* out_tok, float* out_key, uint32_t* status, void* ws, size_t ws_bytes,
+                            pps_stream_t stream) {
+    return draft_hetero(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature, 0, 1.0f, row_block, n_blocks,
+                        out_tok, out_key, status, ws, ws_bytes, stream);
+}
+
+pps_status pps_draft_hetero_trunc(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab,
+                                  int64_t row_stride, pps_row_ids ids, float temperature, int32_t top_k, float top_p,
+                                  const int32_t* row_block, int32_t n_blocks, int32_t* out_tok, float* out_key,
+                                  uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream) {
+    pps_status st = check_trunc(top_k, top_p);
+    if (st != PPS_OK) return st;
+    return draft_hetero(q_logits, dtype, n_rows, vocab, row_stride, ids, temperature, top_k, top_p, row_block,
+                        n_blocks, out_tok, out_key, status, ws, ws_bytes, stream);
 }
 
 pps_status pps_hetero_expand(int32_t n_seq, int32_t n_blocks, int32_t gamma, int32_t depth, const int32_t* draft_tok,

@@ -92,7 +92,7 @@ void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials
 cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
 int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk = false);
 cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
-int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec);
+int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec, bool blk = false);
 
 // launchers (pps_misc.cu)
 // detection score kind and its constants (pps_device.cuh score_kind32)

@@ -1102,24 +1102,28 @@ cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cud
 // like k ln(segment / k), and a row finished by one warp needs no merge):
 // with at most as many rows as resident warps, each row gets the same number
 // of warps s; with more rows, the grid is the resident one.
-int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec) {
-    static int sms = 0, occ[2][2][2] = {};
+static const void* trunc_fn(int dtype, bool verify, bool blk, bool vec) {
+    if (dtype == 1) {
+        if (verify) return vec ? (const void*)trunc_kernel<1, true, true, false> : (const void*)trunc_kernel<1, true, false, false>;
+        if (blk) return vec ? (const void*)trunc_kernel<1, false, true, true> : (const void*)trunc_kernel<1, false, false, true>;
+        return vec ? (const void*)trunc_kernel<1, false, true, false> : (const void*)trunc_kernel<1, false, false, false>;
+    }
+    if (verify) return vec ? (const void*)trunc_kernel<0, true, true, false> : (const void*)trunc_kernel<0, true, false, false>;
+    if (blk) return vec ? (const void*)trunc_kernel<0, false, true, true> : (const void*)trunc_kernel<0, false, false, true>;
+    return vec ? (const void*)trunc_kernel<0, false, true, false> : (const void*)trunc_kernel<0, false, false, false>;
+}
+
+int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec, bool blk) {
+    static int sms = 0, occ[2][3][2] = {};
     int dev = 0;
     cudaGetDevice(&dev);
     if (sms == 0) {
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         if (sms <= 0) sms = 1;
     }
-    int& o = occ[dtype][verify][vec];
+    int& o = occ[dtype][verify ? 1 : (blk ? 2 : 0)][vec];
     if (o == 0) {
-        const void* fn = nullptr;
-        if (dtype == 1)
-            fn = verify ? (vec ? (const void*)trunc_kernel<1, true, true> : (const void*)trunc_kernel<1, true, false>)
-                        : (vec ? (const void*)trunc_kernel<1, false, true> : (const void*)trunc_kernel<1, false, false>);
-        else
-            fn = verify ? (vec ? (const void*)trunc_kernel<0, true, true> : (const void*)trunc_kernel<0, true, false>)
-                        : (vec ? (const void*)trunc_kernel<0, false, true> : (const void*)trunc_kernel<0, false, false>);
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, kThreads, 0);
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, trunc_fn(dtype, verify, blk && !verify, vec), kThreads, 0);
         if (o <= 0) o = 1;
     }
     int64_t g = (int64_t)sms * o;
@@ -1133,21 +1137,28 @@ int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec) 
 
 cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream) {
     dim3 grid(a.G), block(kThreads);
+    const bool blk = !verify && a.row_block != nullptr;
     if (dtype == 1) {
         if (verify) {
-            if (vec) trunc_kernel<1, true, true><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<1, true, false><<<grid, block, 0, stream>>>(a);
+            if (vec) trunc_kernel<1, true, true, false><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<1, true, false, false><<<grid, block, 0, stream>>>(a);
+        } else if (blk) {
+            if (vec) trunc_kernel<1, false, true, true><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<1, false, false, true><<<grid, block, 0, stream>>>(a);
         } else {
-            if (vec) trunc_kernel<1, false, true><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<1, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) trunc_kernel<1, false, true, false><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<1, false, false, false><<<grid, block, 0, stream>>>(a);
         }
     } else {
         if (verify) {
-            if (vec) trunc_kernel<0, true, true><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<0, true, false><<<grid, block, 0, stream>>>(a);
+            if (vec) trunc_kernel<0, true, true, false><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<0, true, false, false><<<grid, block, 0, stream>>>(a);
+        } else if (blk) {
+            if (vec) trunc_kernel<0, false, true, true><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<0, false, false, true><<<grid, block, 0, stream>>>(a);
         } else {
-            if (vec) trunc_kernel<0, false, true><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<0, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) trunc_kernel<0, false, true, false><<<grid, block, 0, stream>>>(a);
+            else trunc_kernel<0, false, false, false><<<grid, block, 0, stream>>>(a);
         }
     }
     return cudaGetLastError();

@@ -696,9 +696,9 @@ __device__ __forceinline__ void merge_low_f(float& xk, int& xi, float yk, int yi
         }
     }
 }
-template <int DT, bool VERIFY>
+template <int DT, bool VERIFY, bool BLK>
 __device__ __noinline__ void finalize_trunc(const RaceArgs& a, int64_t r, const TopList& L, int kr, int kp,
-                                            float* s_val) {
+                                            float* s_val, Blk bk) {
     const int lane = threadIdx.x & 31;
     const int k = a.top_k;
     const float lk = L.entry(k - 1);  // l_(k); -inf when the row has fewer than k usable tokens
@@ -721,8 +721,8 @@ __device__ __noinline__ void finalize_trunc(const RaceArgs& a, int64_t r, const 
         WarpList W;
         W.reset(kp, kr);
         SlowState st{W};
-        st = tail_loop<DT>(st, row, a.V, 0, a.nv, a.c, key, ctx, pos, lk);
-        finalize_row<DT, VERIFY>(a, r, st.L.lk, st.L.li, fminf(st.L.th, st.L.tf), kr, kp, lane);
+        st = tail_loop<DT, BLK>(st, row, a.V, 0, a.nv, a.c, key, ctx, pos, lk, bk);
+        finalize_row<DT, VERIFY, BLK>(a, r, st.L.lk, st.L.li, fminf(st.L.th, st.L.tf), kr, kp, lane, bk);
         return;
     }
     // S = the list's entries with logit >= keep: the race's fp32 keys, the 32
@@ -730,19 +730,25 @@ __device__ __noinline__ void finalize_trunc(const RaceArgs& a, int64_t r, const 
     // complete, so nothing was dropped: drop bound +inf)
     float ka = kInf, kb = kInf;
     int ia = L.ai, ib = L.bi;
-    if (L.av > -kInf && L.av >= keep) ka = key32(word_of(key, ctx, pos, ia, 1), L.av, a.c);
-    if (L.bv > -kInf && L.bv >= keep) kb = key32(word_of(key, ctx, pos, ib, 1), L.bv, a.c);
+    // proposal rows of the augmented race: the tokens' block arrivals
+    auto list_key = [&](int i, float l) {
+        const uint32_t w = word_of(key, ctx, pos, i, 1);
+        if constexpr (BLK) return block_key_of(key, ctx, pos, i, w, l, a.c, bk.b, bk.B, bk.invB());
+        return key32(w, l, a.c);
+    };
+    if (L.av > -kInf && L.av >= keep) ka = list_key(ia, L.av);
+    if (L.bv > -kInf && L.bv >= keep) kb = list_key(ib, L.bv);
     if (ka == kInf) ia = INT_MAX;
     if (kb == kInf) ib = INT_MAX;
     warp_sort(ka, ia, lane);
     warp_sort(kb, ib, lane);
     merge_low_f(ka, ia, kb, ib, lane);
-    finalize_row<DT, VERIFY>(a, r, ka, ia, kInf, kr, kp, lane);
+    finalize_row<DT, VERIFY, BLK>(a, r, ka, ia, kInf, kr, kp, lane, bk);
 }
 
-template <int DT, bool VERIFY>
+template <int DT, bool VERIFY, bool BLK>
 __device__ __noinline__ void finish_trunc_segment(const RaceArgs& a, int64_t r, int64_t gw, int64_t NW, int64_t v0,
-                                                  int64_t v1, TopList L, int kr, int kp, float* s_val) {
+                                                  int64_t v1, TopList L, int kr, int kp, float* s_val, Blk bk) {
     const int lane = threadIdx.x & 31;
     const int64_t nv = a.nv;
     bool final_here = v0 == 0 && v1 == nv;
@@ -777,14 +783,14 @@ __device__ __noinline__ void finish_trunc_segment(const RaceArgs& a, int64_t r, 
         }
     }
     if (final_here) {
-        finalize_trunc<DT, VERIFY>(a, r, L, kr, kp, s_val);
+        finalize_trunc<DT, VERIFY, BLK>(a, r, L, kr, kp, s_val, bk);
         if constexpr (VERIFY) sequence_ticket(a, r, lane);
     }
 }
 
 // ---------------------------------------------------------------- the kernel
 
-template <int DT, bool VERIFY, bool VEC>
+template <int DT, bool VERIFY, bool VEC, bool BLK>
 __global__ void __launch_bounds__(kThreads, PPS_TRUNC_MIN_BLOCKS) trunc_kernel(const RaceArgs a) {
     __shared__ float s_val[kTopMax];
     __shared__ float s_cv[kCandCap];
@@ -809,6 +815,11 @@ __global__ void __launch_bounds__(kThreads, PPS_TRUNC_MIN_BLOCKS) trunc_kernel(c
         TopList L;
         L.reset();
         topk_segment<DT, VEC>(L, row, a.V, v0, v1, a.top_k, s_cv, s_ci, s_qv, s_qi);
-        finish_trunc_segment<DT, VERIFY>(a, r, gw, NW, v0, v1, L, kr, kp, s_val);
+        Blk bk;
+        if constexpr (BLK) {
+            bk.b = __ldg(a.row_block + r);
+            bk.B = a.n_blocks;
+        }
+        finish_trunc_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, s_val, bk);
     }
 }

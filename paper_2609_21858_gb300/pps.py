@@ -80,6 +80,9 @@ def lib():
             L.pps_draft_hetero.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, vp, i32, vp, vp, vp, vp,
                                            sz, vp]
             L.pps_draft_hetero.restype = ctypes.c_int
+            L.pps_draft_hetero_trunc.argtypes = [vp, ctypes.c_int, i64, i64, i64, RowIds, f32, i32, f32, vp, i32, vp,
+                                                 vp, vp, vp, sz, vp]
+            L.pps_draft_hetero_trunc.restype = ctypes.c_int
             L.pps_hetero_expand.argtypes = [i32, i32, i32, i32, vp, RowIds, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp,
                                             vp, vp]
             L.pps_hetero_expand.restype = ctypes.c_int
@@ -287,9 +290,10 @@ def tree_expand(K: int, gamma: int, depth: int, draft, rows_key, rows_ctx, rows_
 
 
 def draft_hetero(q_logits, key, ctx, pos, row_block, n_blocks: int, temperature: float = 1.0, ws=None, status=None,
-                 out_tok=None, out_key=None, stream=None):
-    """pps_draft_hetero: proposal row_block[r] of n_blocks at each row (non-identical
-    proposals on the augmented source).  Returns the [n_rows] int32 tokens."""
+                 out_tok=None, out_key=None, stream=None, top_k: int = 0, top_p: float = 1.0):
+    """pps_draft_hetero (pps_draft_hetero_trunc when top_k > 0): proposal row_block[r] of
+    n_blocks at each row (non-identical proposals on the augmented source).  Returns the
+    [n_rows] int32 tokens."""
     n, V, stride = _rows(q_logits)
     dev = q_logits.device
     if out_tok is None:
@@ -298,6 +302,13 @@ def draft_hetero(q_logits, key, ctx, pos, row_block, n_blocks: int, temperature:
         ws = workspace(n, 0, dev)
     if row_block.dtype != torch.int32 or not row_block.is_cuda or not row_block.is_contiguous():
         raise TypeError("row_block must be a contiguous CUDA int32 tensor")
+    if top_k > 0:
+        code = lib().pps_draft_hetero_trunc(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
+                                            float(temperature), int(top_k), float(top_p), _ptr(row_block),
+                                            int(n_blocks), _ptr(out_tok), _ptr(out_key), _ptr(status), _ptr(ws),
+                                            ws.numel(), _stream(stream))
+        _check("pps_draft_hetero_trunc", code)
+        return out_tok
     code = lib().pps_draft_hetero(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
                                   float(temperature), _ptr(row_block), int(n_blocks), _ptr(out_tok), _ptr(out_key),
                                   _ptr(status), _ptr(ws), ws.numel(), _stream(stream))

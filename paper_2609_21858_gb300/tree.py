@@ -141,7 +141,8 @@ class HeteroTreeBuilder:
         n = self.n_seq * self.B
         return slice(d * n, (d + 1) * n)
 
-    def run(self, root_key, root_ctx, root_pos, draft_logits, temperature: float = 1.0, stream=None):
+    def run(self, root_key, root_ctx, root_pos, draft_logits, temperature: float = 1.0, top_k: int = 0,
+            top_p: float = 1.0, stream=None):
         """Draft the trees: per depth one pps_draft_hetero and one pps_hetero_expand."""
         B = self.B
         s0 = self.rows(0)
@@ -156,7 +157,7 @@ class HeteroTreeBuilder:
             s = self.rows(d)
             key, ctx, pos, blk = self.row_key[s], self.row_ctx[s], self.row_pos[s], self.row_block[s]
             pps.draft_hetero(draft_logits(d, key, ctx, pos, blk), key, ctx, pos, blk, B, temperature=temperature,
-                             ws=self.ws, out_tok=self.draft_tok[s], stream=stream)
+                             ws=self.ws, out_tok=self.draft_tok[s], stream=stream, top_k=top_k, top_p=top_p)
             nxt = None
             if d + 1 < self.gamma:
                 sn = self.rows(d + 1)
@@ -165,11 +166,13 @@ class HeteroTreeBuilder:
                               nodes, stream=stream)
         return self
 
-    def verify(self, p_logits, temperature: float = 1.0, ws=None, out=None, status=None, stream=None):
+    def verify(self, p_logits, temperature: float = 1.0, top_k: int = 0, top_p: float = 1.0, ws=None, out=None,
+               status=None, stream=None):
         """The target race over every node slot and the walk (pps_verify_tree, K = B)."""
         return pps.verify_tree(p_logits, self.node_key, self.node_ctx, self.node_pos, self.gamma, self.seq_off,
                                self.node_draft_row, self.list_tok, self.list_nd, self.child_node,
-                               temperature=temperature, ws=ws, out=out, status=status, stream=stream)
+                               temperature=temperature, ws=ws, out=out, status=status, stream=stream, top_k=top_k,
+                               top_p=top_p)
 
 
 def build_hetero(root_key, root_ctx, root_pos, B: int, gamma: int, draft_logits, **kw) -> HeteroTreeBuilder:

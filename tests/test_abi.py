@@ -164,6 +164,13 @@ def test_hetero_entry_points_validate_arguments():
     assert draft(dtype=7) == pps.ERR_UNSUPPORTED
     assert draft(n_rows=0) == pps.OK
 
+    def trunc(top_k=50, top_p=1.0, B=4):
+        return L.pps_draft_hetero_trunc(fake, pps.BF16, 8, 100, 100, ids, 1.0, top_k, top_p, fake, B, fake, None,
+                                        None, fake, ws, None)
+
+    for kw in (dict(top_k=0), dict(top_k=65), dict(top_p=0.0), dict(top_p=1.5), dict(B=0)):
+        assert trunc(**kw) == pps.ERR_INVALID_ARG, kw
+
     def expand(n_seq=4, B=4, gamma=3, depth=0, tok=fake, nxt=fake):
         return L.pps_hetero_expand(n_seq, B, gamma, depth, tok, ids, fake, nxt, nxt, nxt, nxt, fake, fake, fake,
                                    fake, fake, fake, None)

@@ -12,7 +12,7 @@ import torch
 
 import oracle
 from paper_2609_21858_gb300 import pps, synth, tree
-from parity import FLIP_MARGIN, compare_winners, dev_ids
+from parity import FLIP_MARGIN, TOP_P_MARGIN, compare_winners, dev_ids, f32
 
 pytestmark = pytest.mark.gpu
 
@@ -222,3 +222,89 @@ def test_one_step_acceptance_is_the_propositions_coupling():
     assert abs(hit - bound) < 4.5 * sd, (hit, bound)
     assert acc >= hit
     assert acc >= bound - 4.5 * sd
+
+
+# ---------------------------------------------------------------- truncated proposal rows
+
+def _check_trunc_rows(q, key, ctx, pos, blk, B, top_k, top_p, T=1.0):
+    k, c, p = dev_ids(key, ctx, pos)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    x = pps.draft_hetero(q, k, c, p, torch.as_tensor(blk, dtype=torch.int32).cuda(), B, temperature=T,
+                         status=status, top_k=top_k, top_p=top_p)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    # the oracle gets top_p and T as the fp32 values the C ABI receives
+    qm, loose = oracle.truncate_rows(q.float().cpu().numpy(), top_k, f32(top_p), f32(T))
+    ox, _, om = oracle.block_draft_rows(qm, key, ctx, pos, blk, B, f32(T))
+    gx = x.cpu().numpy()
+    for r in np.nonzero(gx != ox)[0]:
+        assert om[r] < FLIP_MARGIN or loose[r] < TOP_P_MARGIN, (r, gx[r], ox[r], om[r], loose[r])
+
+
+@pytest.mark.parametrize("top_k,top_p", [(50, 1.0), (5, 0.9), (64, 0.5), (1, 1.0)])
+@pytest.mark.parametrize("B,V,dtype", [(3, 4099, torch.bfloat16), (8, 1003, torch.float32),
+                                       (32, 20000, torch.bfloat16)])
+def test_truncated_proposal_rows_match_the_oracle(top_k, top_p, B, V, dtype):
+    n = 64
+    ctx = synth.splitmix64_stream(B + V, n)
+    q = torch.as_tensor(synth.label_logits(ctx, V, seed=B)).to(dtype).cuda()
+    key, _, pos = _ids(n, V + 1)
+    blk = (np.arange(n) % B).astype(np.int32)
+    _check_trunc_rows(q, key, ctx, pos, blk, B, top_k, top_p)
+
+
+def test_truncated_proposal_rows_tie_overflow_and_masks():
+    # a top-k tie group larger than the 64-entry list (the exact second pass, with block keys)
+    n, V, B = 24, 32000, 4
+    rng = np.random.default_rng(31)
+    x = rng.normal(0, 1, (n, V)).astype(np.float32)
+    for r in range(0, n, 2):
+        cols = rng.choice(V, 320, replace=False)
+        x[r, cols[:20]] = 8.0 + 0.25 * np.arange(20)
+        x[r, cols[20:]] = 6.0
+    x[1, :] = -np.inf
+    x[3, :-5] = np.nan
+    q = torch.as_tensor(x).to(torch.bfloat16).cuda()
+    key, ctx, pos = _ids(n, 32)
+    blk = rng.integers(0, B, n).astype(np.int32)
+    for tk, tp in ((40, 1.0), (40, 0.6), (10, 0.999999)):
+        _check_trunc_rows(q, key, ctx, pos, blk, B, tk, tp)
+
+
+def test_truncated_hetero_tree_matches_the_oracle():
+    n_seq, B, gamma, V, top_k = 16, 4, 3, 3000, 20
+    rng = np.random.default_rng(40)
+    key = torch.as_tensor(rng.integers(0, 2 ** 63, n_seq, dtype=np.int64)).cuda()
+    ctx = torch.as_tensor(rng.integers(0, 2 ** 63, n_seq, dtype=np.int64)).cuda()
+    pos = torch.as_tensor(rng.integers(0, 5000, n_seq, dtype=np.int32)).cuda()
+    seen = []
+
+    def draft_logits(d, k_, c_, p_, b_):
+        cc, bb = u64(c_), b_.cpu().numpy()
+        lg = np.empty((cc.size, V), np.float32)
+        for b in range(B):
+            lg[bb == b] = synth.label_logits(cc[bb == b], V, seed=200 + b)
+        seen.append((u64(k_), cc, p_.cpu().numpy().view(np.uint32), bb, lg))
+        return torch.as_tensor(lg).cuda()
+
+    t = tree.build_hetero(key, ctx, pos, B, gamma, draft_logits, top_k=top_k, top_p=0.95)
+    torch.cuda.synchronize()
+    for d in range(gamma):
+        gk, gc, gp, gb, lg = seen[d]
+        s = t.rows(d)
+        own = t.row_owner[s].cpu().numpy()
+        qm, loose = oracle.truncate_rows(lg, top_k, f32(0.95), 1.0)
+        ox, _, om = oracle.block_draft_rows(qm, gk, gc, gp, gb, B)
+        gx = t.draft_tok[s].cpu().numpy()
+        for r in np.nonzero((own >= 0) & (gx != ox))[0]:
+            assert om[r] < FLIP_MARGIN or loose[r] < TOP_P_MARGIN
+    plg = synth.label_logits(u64(t.node_ctx), V, seed=13)
+    v = t.verify(torch.as_tensor(plg).cuda(), top_k=top_k, top_p=0.95)
+    torch.cuda.synchronize()
+    pm, ploose = oracle.truncate_rows(plg, top_k, f32(0.95), 1.0)
+    win, wd, _, mg = oracle.target_rows(pm, u64(t.node_key), u64(t.node_ctx), t.node_pos.cpu().numpy().view(np.uint32))
+    gw, gword = v["winner"].cpu().numpy(), v["word"].cpu().numpy().view(np.uint32)
+    compare_winners(gw, gword, win, wd, mg, loose=ploose < TOP_P_MARGIN)
+    ow = oracle.walk(gamma, t.seq_off.cpu().numpy(), t.node_draft_row.cpu().numpy(), t.list_tok.cpu().numpy(),
+                     t.list_nd.cpu().numpy(), t.child_node.cpu().numpy(), gw, gword)
+    assert np.array_equal(v["accept_len"].cpu().numpy(), ow["accept_len"])
