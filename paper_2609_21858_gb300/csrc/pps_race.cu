@@ -40,6 +40,9 @@
 #ifndef PPS_ROWBOUND
 #define PPS_ROWBOUND 1  // 1: warps that share a row share its filter bound through the workspace
 #endif
+#ifndef PPS_IID_FAST
+#define PPS_IID_FAST 1  // 1: IID epilogue in fp32 with a separation check (fp64 only on near ties)
+#endif
 #ifndef PPS_VECFILTER
 #define PPS_VECFILTER 1  // 1: one filter test per 16-byte vector on verify rows and fp32 rows
 #endif
@@ -771,6 +774,83 @@ __device__ __forceinline__ void emit_row(const RaceArgs& a, int64_t r, double dk
     if (lane == 0 && a.out_nd) a.out_nd[r] = nd;
 }
 
+// IID rows whose first-arrival list has no near ties: the multi-arrival
+// scores in fp32, in key32's units (log2 of the summed -log2 u terms, minus
+// l c).  Each term errs by at most its transform's bound (kErrAbs, measured)
+// plus lg2.approx's error, the sum of at most 32 terms adds 31 roundings and
+// the outer lg2.approx its error again, so every score is within
+// key_err_bound + kBlkErr of its exact value (the derivation of kBlkErr covers
+// this sum too).  When every gap between consecutive selected scores, and
+// between the last selected and the best unselected one, exceeds the two
+// bounds, the samples and their order are those of the exact scores and the
+// row is written here; otherwise it returns false and the caller re-keys the
+// row in fp64 (emit_row).
+template <int DT>
+__device__ __noinline__ bool iid_fast(const RaceArgs& a, int64_t r, float lk, int li, int nvalid, int kr, int lane,
+                                      uint64_t key, uint64_t ctx, uint32_t pos) {
+    const int nuse = min(nvalid, kr);
+    const bool mine = lane < nuse;
+    const int tok = mine ? li : -1;
+    const float lt = mine ? logit_at<DT>(a, r, li) : 0.0f;
+    float y = mine ? neg_log2_u(word_of(key, ctx, pos, li, 1)) : 0.0f;
+    float h = mine ? lk : kInf;  // arrival 1's score is the list key itself
+    int j = 1, mult = 0, sample = -1, nsel = 0;
+    float selh = kInf;
+    for (int m = 0; m < kr; ++m) {
+        // warp argmin of (h, tok, j)
+        float bh = h;
+        int bt = mine ? tok : INT_MAX, bj = j, bl = lane;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            const float oh = __shfl_xor_sync(FULL, bh, off);
+            const int ot = __shfl_xor_sync(FULL, bt, off);
+            const int oj = __shfl_xor_sync(FULL, bj, off);
+            const int ol = __shfl_xor_sync(FULL, bl, off);
+            if (oh < bh || (oh == bh && (ot < bt || (ot == bt && oj < bj)))) {
+                bh = oh;
+                bt = ot;
+                bj = oj;
+                bl = ol;
+            }
+        }
+        if (bt == INT_MAX) break;  // fewer usable tokens than samples
+        if (lane == m) {
+            sample = bt;
+            selh = bh;
+        }
+        ++nsel;
+        if (lane == bl) {
+            ++mult;
+            ++j;
+            if (j <= kr) {
+                y += neg_log2_u(word_of(key, ctx, pos, tok, j));
+                h = fmaf(-lt, a.c, lg2_approx(y));
+            } else {
+                h = kInf;
+            }
+        }
+    }
+    float nxt = h;  // the best unselected score
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) nxt = fminf(nxt, __shfl_xor_sync(FULL, nxt, off));
+    const float after = __shfl_down_sync(FULL, selh, 1);
+    const float b = lane + 1 < nsel ? after : nxt;
+    const bool bad = lane < nsel && b < kInf &&
+                     !(b - selh > key_err_bound(selh) + key_err_bound(b) + 2.0f * kBlkErr);
+    if (__any_sync(FULL, bad)) return false;
+    const int nd = __popc(__ballot_sync(FULL, mult > 0));
+    const int K = a.K;
+    if (lane < K) {
+        const size_t o = (size_t)r * K + lane;
+        a.out_tok[o] = lane < kr ? tok : -1;
+        if (a.out_key) a.out_key[o] = (mine && lane < kr) ? key_to_s(lk) : kInf;
+        if (a.out_mult) a.out_mult[o] = lane < kr ? mult : 0;
+        if (a.out_samples) a.out_samples[o] = lane < kr ? sample : -1;
+    }
+    if (lane == 0 && a.out_nd) a.out_nd[r] = nd;
+    return true;
+}
+
 // Warp 0 finishes row r from its complete list (lk, li) and the drop bound.
 // BLK: the near-tie keys are those of the row's block arrivals.
 template <int DT, bool VERIFY, bool BLK = false>
@@ -796,9 +876,14 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
     float nk = __shfl_down_sync(FULL, lk, 1);
     int lim = min(nvalid, kr + 1);
     bool close = lane + 1 < lim && !(nk - lk > err(lk) + err(nk));
-    const bool need_exact = (__ballot_sync(FULL, close) != 0) || (!VERIFY && a.iid);
+    const bool any_close = __ballot_sync(FULL, close) != 0;
     const uint64_t key = a.key[r], ctx = a.ctx[r];
     const uint32_t pos = a.pos[r];
+    if constexpr (!VERIFY && !BLK) {
+        if (a.iid && !any_close && PPS_IID_FAST && iid_fast<DT>(a, r, lk, li, nvalid, kr, lane, key, ctx, pos))
+            return;
+    }
+    const bool need_exact = any_close || (!VERIFY && a.iid);
     double dk = (double)INFINITY;
     float sk = key_to_s(lk);
     if (need_exact) {
