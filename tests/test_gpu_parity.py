@@ -209,6 +209,36 @@ def test_near_ties_are_resolved_exactly():
     assert exact >= n - 2 and int(status.item()) == 0
 
 
+def test_iid_multi_arrival_near_ties_are_resolved_exactly():
+    # fp32 logits built so that a token's second arrival ties another token's first arrival
+    # within ~1e-7: the fp32 IID epilogue must see the tie and hand the row to the fp64 stage
+    n, V, K = 60, 600, 4
+    key, ctx, pos = _rand_ids(n, 71)
+    rng = np.random.default_rng(72)
+    logits = rng.normal(0, 1.0, (n, V)).astype(np.float32)
+    for r in range(n):
+        w1 = oracle.words(key[r:r + 1], ctx[r:r + 1], pos[r:r + 1], V)[0]
+        w2 = oracle.words(key[r:r + 1], ctx[r:r + 1], pos[r:r + 1], V, 2)[0]
+        x = np.array([math.log(oracle.exp1(int(v))) for v in w1])
+        s = x - logits[r]
+        order = np.argsort(s)
+        a, b = order[0], order[1 + r % 3]
+        g2 = math.log(oracle.exp1(int(w1[b])) + oracle.exp1(int(w2[b])))
+        logits[r, b] = np.float32(g2 - s[a] + (1e-7 if r % 2 else -1e-7))
+    L = torch.as_tensor(logits).cuda()
+    ids = dev_ids(key, ctx, pos)
+    d_o = oracle.draft_rows(logits, key, ctx, pos, K, mode=oracle.IID)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    d = pps.draft_list(L, *ids, K, mode=pps.IID, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    for name, want in (("samples", d_o["labels"]), ("mult", d_o["mult"]), ("tok", d_o["tok"])):
+        got = d[name].cpu().numpy()
+        for r in range(n):
+            if d_o["min_gap"][r] > 1e-12:
+                assert list(got[r]) == list(want[r]), (name, r, got[r], want[r])
+
+
 def test_workspace_reuse_is_deterministic():
     wl = synth.make_workload("chain4x4", n_seq=4, vocab=9000, seed=71)
     a = run_gpu(wl)
