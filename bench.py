@@ -16,6 +16,7 @@ from __future__ import annotations
 import argparse
 import json
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -167,6 +168,25 @@ def max_over_ranks(x: float, world: int) -> float:
     return float(t.item())
 
 
+def cpu_model() -> str:
+    """The host CPU's name (x86 'model name', else the Arm implementer/part), for the oracle timing."""
+    try:
+        info = open("/proc/cpuinfo").read()
+        for line in info.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+        parts = {}
+        for line in info.splitlines():
+            if ":" in line:
+                k, v = line.split(":", 1)
+                parts.setdefault(k.strip(), v.strip())
+        if "CPU part" in parts:
+            return f"{platform.machine()} implementer {parts.get('CPU implementer')} part {parts['CPU part']}"
+    except OSError:
+        pass
+    return platform.machine()
+
+
 def oracle_sample(wl, n_draft_rows: int, n_target_rows: int, seed: int = 0, top_k: int = 0, top_p: float = 1.0):
     """Host copies of a bounded sample of the workload's rows and a timer over them."""
     import oracle
@@ -204,6 +224,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="zipf_k8")
+    ap.add_argument("--k", type=int, default=8, help="drafts per root of the ksweep workload (1..32)")
     ap.add_argument("--n-seq", type=int, default=None, help="override the number of sequences (smaller profiling cases)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--n-tokens", type=int, default=10_000_000, help="detector workload size")
@@ -236,7 +257,8 @@ def main():
     if args.workload == "hetero":
         run_hetero(args, rank, world, dev)
         return
-    wl = synth.make_workload(args.workload, device=dev, n_seq=args.n_seq)
+    wl = synth.make_workload(args.workload, device=dev, n_seq=args.n_seq,
+                             K_sweep=args.k if args.workload == "ksweep" else None)
     t = wl.tree
     g = lambda x: torch.as_tensor(np.asarray(x)).to(dev).contiguous()
     row_k, seq_off, ndr, child = g(t.row_k), g(t.seq_off), g(t.node_draft_row), g(t.child_node)
@@ -398,13 +420,21 @@ def main():
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
+        import oracle
         run, nd, nn, cores = oracle_sample(wl, 8, 8, top_k=args.top_k, top_p=args.top_p)
         dt = run()
         reps = max(1, int(args.cpu_seconds / max(dt, 1e-3)))
         tot = sum(run() for _ in range(reps))
+        # the same sample on one thread (a few repetitions), then all threads again
+        oracle.set_threads(1)
+        reps1 = max(1, min(3, int(0.2 * args.cpu_seconds / max(dt * cores, 1e-3))))
+        tot1 = sum(run() for _ in range(reps1))
+        oracle.set_threads(cores)
         cpu = {"value": reps * (nd + nn) / tot, "unit": "rows/s", "cores": cores, "kind": "oracle",
                "sample": f"{nd} draft + {nn} target rows of the same workload, x{reps} repetitions, "
-                         f"{tot:.1f} s on {cores} threads"}
+                         f"{tot:.1f} s on {cores} threads",
+               "single_thread_value": reps1 * (nd + nn) / tot1, "cpu_model": cpu_model(),
+               "nproc": os.cpu_count()}
 
     trunc = f", top-k {args.top_k}, top-p {args.top_p}" if args.top_k > 0 else ""
     if rank == 0:
@@ -714,7 +744,8 @@ def run_hetero(args, rank, world, dev):
 def run_reference(args, world):
     """The CPU oracle on a bounded sample per step, on this host's cores."""
     from paper_2609_21858_gb300 import synth
-    wl = synth.make_workload(args.workload, device="cuda" if torch.cuda.is_available() else "cpu")
+    wl = synth.make_workload(args.workload, device="cuda" if torch.cuda.is_available() else "cpu",
+                             K_sweep=args.k if args.workload == "ksweep" else None)
     t = wl.tree
     run, nd, nn, cores = oracle_sample(wl, 4, 4)
     for _ in range(max(1, min(args.warmup, 2))):
@@ -729,7 +760,8 @@ def run_reference(args, world):
         "config": {"workload": f"{args.workload}: B={t.n_seq}, V={wl.vocab}, K={t.K}, gamma={t.gamma}",
                    "rows_per_step": nd + nn},
         "cpu_baseline": {"value": value, "unit": "rows/s", "cores": cores, "kind": "oracle",
-                         "sample": f"{nd} draft + {nn} target rows per step"},
+                         "sample": f"{nd} draft + {nn} target rows per step", "cpu_model": cpu_model(),
+                         "nproc": os.cpu_count()},
         "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 

@@ -84,11 +84,14 @@ __device__ __forceinline__ bool lex_less_d(double ak, int ai, double bk, int bi)
 // A warp list holds entries (k, i) sorted ascending by (k, i), entry m in
 // lane m; lanes >= kp hold (+inf, INT_MAX).
 
-// insert one warp-uniform entry (serial path for a few survivors)
-__device__ __forceinline__ void list_insert(float& lk, int& li, float ck, int ci, int kp, int lane) {
+// insert one warp-uniform entry (serial path for a few survivors); returns
+// the key left out: the entry pushed out of a full list (+inf if there was
+// room), or ck itself when it does not enter
+__device__ __forceinline__ float list_insert(float& lk, int& li, float ck, int ci, int kp, int lane) {
     bool less = lane < kp && lex_less(ck, ci, lk, li);
     unsigned m = __ballot_sync(FULL, less);
-    if (m == 0) return;
+    if (m == 0) return ck;
+    const float last = __shfl_sync(FULL, lk, kp - 1);
     int p = __ffs(m) - 1;
     float uk = __shfl_up_sync(FULL, lk, 1);
     int ui = __shfl_up_sync(FULL, li, 1);
@@ -103,6 +106,7 @@ __device__ __forceinline__ void list_insert(float& lk, int& li, float ck, int ci
         lk = kInf;
         li = INT_MAX;
     }
+    return last;
 }
 
 // bitonic sort of one entry per lane, ascending
@@ -255,6 +259,7 @@ struct WarpList {
     int thi;
     float tf;  // filter bound: the filter drops only tokens with keys >= tf; never rises
     float tz;  // filter threshold for tf (pps_device.cuh)
+    float mr;  // smallest key of a survivor the list left out (rejected or pushed out)
     int kp;
     int k;     // entries the row needs (kp > k leaves room for near ties)
 
@@ -265,6 +270,7 @@ struct WarpList {
         thi = INT_MAX;
         tf = kInf;
         tz = kInf;
+        mr = kInf;
         kp = kp_;
         k = k_;
     }
@@ -275,12 +281,20 @@ struct WarpList {
         tz = filter_tz(tf + shift);
     }
     // after the list changed: tf <= min(th, (entry k-1) + filter_slack), the
-    // slack widened by 4 eb for keys with extra error eb
+    // slack widened by 4 eb for keys with extra error eb.  A list with no
+    // spare entry (kp = k, i.e. k = 32) keeps tf at the slack bound instead:
+    // the filter passes the keys between entry kp-1 and it, the list leaves
+    // them out and records the smallest in mr, so such a list still proves
+    // itself complete unless entry k and the next key nearly tie.
+    __device__ __forceinline__ bool tight() const { return kp == k; }
     __device__ __forceinline__ void refresh(float shift = 0.f, float eb = 0.f) {
         th = __shfl_sync(FULL, lk, kp - 1);
         thi = __shfl_sync(FULL, li, kp - 1);
-        bound(fminf(th, filter_slack(__shfl_sync(FULL, lk, k - 1)) + 4.0f * eb), shift);
+        const float sl = filter_slack(__shfl_sync(FULL, lk, k - 1)) + 4.0f * eb;
+        bound(tight() ? sl : fminf(th, sl), shift);
     }
+    // every token of the segment left out of the list has a key >= drop()
+    __device__ __forceinline__ float drop() const { return fminf(tight() ? mr : th, tf); }
 };
 
 // Publish filter_slack of the list's k-th key (widened by eb) as a filter bound
@@ -320,19 +334,31 @@ __device__ __forceinline__ void offer_survivors(WarpList& L, float (&pk)[VW], in
                 m &= m - 1;
                 const float ck = __shfl_sync(FULL, bk, src);
                 const int ci = __shfl_sync(FULL, bi, src);
-                list_insert(L.lk, L.li, ck, ci, L.kp, lane);
+                L.mr = fminf(L.mr, list_insert(L.lk, L.li, ck, ci, L.kp, lane));
             }
         } else {
             float ok = valid ? bk : kInf;
             int oi = valid ? bi : INT_MAX;
             warp_sort(ok, oi, lane);
-            warp_merge<false>(L.lk, L.li, ok, oi, L.kp, lane);
+            if (L.tight())
+                L.mr = fminf(L.mr, warp_merge<true>(L.lk, L.li, ok, oi, L.kp, lane));
+            else
+                warp_merge<false>(L.lk, L.li, ok, oi, L.kp, lane);
         }
-        // every offer of this round is now in the list or above its threshold
+        // every offer of this round is now in the list or recorded in mr
 #pragma unroll
         for (int e = 0; e < VW; ++e)
             if (e == be) pk[e] = kInf;
         L.refresh(shift, eb);
+    }
+    // keys not offered (at or above entry kp-1) are left out too
+    float rem = kInf;
+#pragma unroll
+    for (int e = 0; e < VW; ++e) rem = fminf(rem, pk[e]);
+    if (L.tight() && __any_sync(FULL, rem < kInf)) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) rem = fminf(rem, __shfl_xor_sync(FULL, rem, o));
+        L.mr = fminf(L.mr, rem);
     }
 }
 
@@ -387,6 +413,7 @@ struct SlowState {
 // counters in shared memory (one iteration adds at most 32 x 2 x units).
 constexpr int kMaxUnits = PPS_UNITS > PPS_UNITS_VERIFY ? PPS_UNITS : PPS_UNITS_VERIFY;
 constexpr int kQueueCap = 32 + 32 * 2 * kMaxUnits;
+static_assert(kQueueCap >= 1 + 2 * 96, "the queue also serves as the scratch of rescan_row");
 
 // Work off the queue: lane j regenerates the words of queued block j (32 at
 // a time), reloads its four logits, keys the tokens over the filter cut and
@@ -851,11 +878,142 @@ __device__ __noinline__ bool iid_fast(const RaceArgs& a, int64_t r, float lk, in
     return true;
 }
 
+// Exact finish of a row whose list could not prove itself complete: tokens
+// crowd its k-th key tau within the error bounds and the 32-entry list has no
+// room left to hold them (always the case for k = 32 on a full list).  One
+// more pass over the row collects every token whose list key is at most
+// filter_slack(tau) (plus the block error) into shared memory, up to
+// kRescanCap of them; the k smallest by their fp64 keys, in order, go to
+// lanes 0..: (dk, li).  Every token whose exact key is at most the row's
+// exact k-th key has a list key within that cut.  Returns false when more
+// tokens than the buffer holds crowd the cut.  `scratch` holds
+// 1 + 2 kRescanCap words.
+constexpr int kRescanCap = 96;
+
+template <int DT, bool BLK>
+__device__ __noinline__ bool rescan_row(const RaceArgs& a, int64_t r, float tau, int kr, int lane, Blk bk,
+                                        uint32_t* scratch, double& dk, int& li, int& nvalid) {
+    constexpr int VW = DT == 1 ? 8 : 4;
+    const uint64_t key = a.key[r], ctx = a.ctx[r];
+    const uint32_t pos = a.pos[r];
+    const char* row = reinterpret_cast<const char*>(a.logits) + (size_t)r * (size_t)a.stride * (DT == 1 ? 2 : 4);
+    const float c = a.c;
+    const float cut = filter_slack(tau) + (BLK ? 4.0f * kBlkErr : 0.f);
+    const float tz = filter_tz(cut + (BLK ? bk.shift() : 0.f));
+    int* cnt = reinterpret_cast<int*>(scratch);
+    float* ck = reinterpret_cast<float*>(scratch + 1);
+    int* ci = reinterpret_cast<int*>(scratch + 1 + kRescanCap);
+    if (lane == 0) *cnt = 0;
+    __syncwarp();
+    RowPhilox rp;
+    rp.init(key, ctx, pos);
+    for (int64_t v0 = 0; v0 < a.nv; v0 += 32) {
+        const int64_t v = v0 + lane;
+        if (v < a.nv) {
+            const uint4 dv = load_scalar<DT>(row, v, a.V);
+            const uint4 d[2] = {dv, dv};
+#pragma unroll
+            for (int h = 0; h < (DT == 1 ? 2 : 1); ++h) {
+                float l[4];
+                block_logits<DT>(d, h, l);
+                const uint32_t cb = DT == 1 ? (uint32_t)(2 * v + h) : (uint32_t)v;
+                const uint4 q = rp.block(cb);
+                const uint32_t wq[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int64_t i = (int64_t)4 * cb + e;
+                    if (i < a.V && v * VW + 4 * h + e < a.V && filter_pass(wq[e], l[e], c, tz)) {
+                        float k;
+                        if constexpr (BLK)
+                            k = block_key_of(key, ctx, pos, i, wq[e], l[e], c, bk.b, bk.B, bk.invB());
+                        else
+                            k = key32(wq[e], l[e], c);
+                        if (k <= cut) {
+                            const int slot = atomicAdd(cnt, 1);
+                            if (slot < kRescanCap) {
+                                ck[slot] = k;
+                                ci[slot] = (int)i;
+                            }
+                        }
+                    }
+                }
+            }
+        }
+    }
+    __syncwarp();
+    const int n = *cnt;
+    if (n > kRescanCap) return false;
+    // fp64 keys of the candidates (lane m holds candidates m, m + 32, m + 64)
+    double d[3];
+    int id[3];
+#pragma unroll
+    for (int t = 0; t < 3; ++t) {
+        const int m = lane + 32 * t;
+        d[t] = (double)INFINITY;
+        id[t] = INT_MAX;
+        if (m < n) {
+            id[t] = ci[m];
+            const uint32_t w = word_of(key, ctx, pos, id[t], 1);
+            const float l = logit_at<DT>(a, r, id[t]);
+            if constexpr (BLK) {
+                uint32_t wf;
+                const int J = block_words(key, ctx, pos, id[t], bk.b, bk.B, wf);
+                d[t] = block_key64(w, J, wf, bk.b, bk.B, l, a.T);
+            } else {
+                d[t] = key64(w, l, a.T);
+            }
+        }
+    }
+    // the min(n, 32) smallest in order: lane m receives the m-th
+    dk = (double)INFINITY;
+    li = INT_MAX;
+    const int take = min(n, 32);
+    for (int m = 0; m < take; ++m) {
+        double bd = d[0];
+        int bi = id[0], bt = 0;
+#pragma unroll
+        for (int t = 1; t < 3; ++t)
+            if (lex_less_d(d[t], id[t], bd, bi)) {
+                bd = d[t];
+                bi = id[t];
+                bt = t;
+            }
+        double wd = bd;
+        int wi = bi, wl = lane;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            const double od = __shfl_xor_sync(FULL, wd, off);
+            const int oi = __shfl_xor_sync(FULL, wi, off);
+            const int ol = __shfl_xor_sync(FULL, wl, off);
+            if (lex_less_d(od, oi, wd, wi)) {
+                wd = od;
+                wi = oi;
+                wl = ol;
+            }
+        }
+        if (lane == m) {
+            dk = wd;
+            li = wi;
+        }
+        if (lane == wl) {
+#pragma unroll
+            for (int t = 0; t < 3; ++t)
+                if (t == bt) {
+                    d[t] = (double)INFINITY;
+                    id[t] = INT_MAX;
+                }
+        }
+    }
+    nvalid = take;
+    (void)kr;
+    return true;
+}
+
 // Warp 0 finishes row r from its complete list (lk, li) and the drop bound.
 // BLK: the near-tie keys are those of the row's block arrivals.
 template <int DT, bool VERIFY, bool BLK = false>
 __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk, int li, float theta_drop, int kr,
-                                          int kp, int lane, Blk bk = Blk{}) {
+                                          int kp, int lane, Blk bk = Blk{}, uint32_t* scratch = nullptr) {
     const int nvalid = __popc(__ballot_sync(FULL, lane < kp && lk < kInf));
     const float tau = nvalid >= kr ? __shfl_sync(FULL, lk, kr - 1) : kInf;
     // list-key error bound (block rows: widened by kBlkErr)
@@ -867,6 +1025,16 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
         complete = true;
     else
         complete = theta_drop == kInf || theta_drop > tau + err(tau) + err(theta_drop);
+    if (!complete && nvalid >= kr && scratch != nullptr) {
+        // the boundary is crowded: finish the row exactly with one more pass
+        double dkr;
+        int lir, nvr;
+        if (rescan_row<DT, BLK>(a, r, tau, kr, lane, bk, scratch, dkr, lir, nvr)) {
+            if (lane == 0 && a.status && tau > -kInf && fabsf(tau) > 65536.0f) atomicOr(a.status, PPS_FLAG_LOGIT_RANGE);
+            emit_row<DT, VERIFY>(a, r, dkr, (float)dkr, lir, nvr, kr, lane, a.key[r], a.ctx[r], a.pos[r]);
+            return;
+        }
+    }
     if (lane == 0 && a.status) {
         unsigned f = complete ? 0u : PPS_FLAG_GUARD;
         if (nvalid >= kr && tau > -kInf && fabsf(tau) > 65536.0f) f |= PPS_FLAG_LOGIT_RANGE;
@@ -1023,13 +1191,13 @@ __device__ __noinline__ void sequence_ticket(const RaceArgs& a, int64_t r, int l
 
 template <int DT, bool VERIFY, bool BLK>
 __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_t gw, int64_t NW, int64_t v0,
-                                            int64_t v1, const WarpList L, int kr, int kp, Blk bk) {
+                                            int64_t v1, const WarpList L, int kr, int kp, Blk bk, uint32_t* scratch) {
     const int lane = threadIdx.x & 31;
     const int64_t nv = a.nv;
     float lk = L.lk;
     int li = L.li;
     // every token of the segment left out of the list has a key >= theta_drop
-    float theta_drop = fminf(L.th, L.tf);
+    float theta_drop = L.drop();
     bool final_here = v0 == 0 && v1 == nv;
     if (!final_here) {
         // publish this segment's list; the last warp of the row merges all segments
@@ -1064,7 +1232,7 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
         }
     }
     if (final_here) {
-        finalize_row<DT, VERIFY, BLK>(a, r, lk, li, theta_drop, kr, kp, lane, bk);
+        finalize_row<DT, VERIFY, BLK>(a, r, lk, li, theta_drop, kr, kp, lane, bk, scratch);
         if constexpr (VERIFY) sequence_ticket(a, r, lane);
     }
 }
@@ -1114,7 +1282,7 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
         stream_segment<DT, VEC, BLK, VERIFY || DT == 0, VERIFY ? PPS_UNITS_VERIFY : PPS_UNITS>(
             L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk, slot);
 
-        finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk);
+        finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk, s_queue);
     }
 }
 

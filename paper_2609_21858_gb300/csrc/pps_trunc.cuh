@@ -698,7 +698,7 @@ __device__ __forceinline__ void merge_low_f(float& xk, int& xi, float yk, int yi
 }
 template <int DT, bool VERIFY, bool BLK>
 __device__ __noinline__ void finalize_trunc(const RaceArgs& a, int64_t r, const TopList& L, int kr, int kp,
-                                            float* s_val, Blk bk) {
+                                            float* s_val, Blk bk, uint32_t* scratch) {
     const int lane = threadIdx.x & 31;
     const int k = a.top_k;
     const float lk = L.entry(k - 1);  // l_(k); -inf when the row has fewer than k usable tokens
@@ -722,7 +722,7 @@ __device__ __noinline__ void finalize_trunc(const RaceArgs& a, int64_t r, const 
         W.reset(kp, kr);
         SlowState st{W};
         st = tail_loop<DT, BLK>(st, row, a.V, 0, a.nv, a.c, key, ctx, pos, lk, bk);
-        finalize_row<DT, VERIFY, BLK>(a, r, st.L.lk, st.L.li, fminf(st.L.th, st.L.tf), kr, kp, lane, bk);
+        finalize_row<DT, VERIFY, BLK>(a, r, st.L.lk, st.L.li, st.L.drop(), kr, kp, lane, bk, scratch);
         return;
     }
     // S = the list's entries with logit >= keep: the race's fp32 keys, the 32
@@ -748,7 +748,8 @@ __device__ __noinline__ void finalize_trunc(const RaceArgs& a, int64_t r, const 
 
 template <int DT, bool VERIFY, bool BLK>
 __device__ __noinline__ void finish_trunc_segment(const RaceArgs& a, int64_t r, int64_t gw, int64_t NW, int64_t v0,
-                                                  int64_t v1, TopList L, int kr, int kp, float* s_val, Blk bk) {
+                                                  int64_t v1, TopList L, int kr, int kp, float* s_val, Blk bk,
+                                                  uint32_t* scratch) {
     const int lane = threadIdx.x & 31;
     const int64_t nv = a.nv;
     bool final_here = v0 == 0 && v1 == nv;
@@ -783,7 +784,7 @@ __device__ __noinline__ void finish_trunc_segment(const RaceArgs& a, int64_t r, 
         }
     }
     if (final_here) {
-        finalize_trunc<DT, VERIFY, BLK>(a, r, L, kr, kp, s_val, bk);
+        finalize_trunc<DT, VERIFY, BLK>(a, r, L, kr, kp, s_val, bk, scratch);
         if constexpr (VERIFY) sequence_ticket(a, r, lane);
     }
 }
@@ -820,6 +821,7 @@ __global__ void __launch_bounds__(kThreads, PPS_TRUNC_MIN_BLOCKS) trunc_kernel(c
             bk.b = __ldg(a.row_block + r);
             bk.B = a.n_blocks;
         }
-        finish_trunc_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, s_val, bk);
+        finish_trunc_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, s_val, bk,
+                                              reinterpret_cast<uint32_t*>(s_ci));
     }
 }
