@@ -239,6 +239,48 @@ def test_iid_multi_arrival_near_ties_are_resolved_exactly():
                 assert list(got[r]) == list(want[r]), (name, r, got[r], want[r])
 
 
+@pytest.mark.parametrize("mode", [pps.DISTINCT, pps.IID])
+def test_k32_full_vocab_lists_complete(mode):
+    # k = 32 fills the 32-entry list: the left-out-key drop bound must prove every row complete
+    wl = synth.make_workload("ksweep", K_sweep=32, n_seq=2)
+    gd, gv, status = run_gpu(wl, mode)
+    assert status == 0
+    t = wl.tree
+    roots = np.nonzero(t.row_k == 32)[0]
+    sel = torch.as_tensor(roots)
+    od = oracle.draft_rows(wl.q_logits[sel].float().numpy(), synth.u64(wl.draft_key[sel]),
+                           synth.u64(wl.draft_ctx[sel]), synth.u32(wl.draft_pos[sel]), 32, mode=mode)
+    sub = {k: (x[roots] if x is not None and x.ndim >= 1 and x.shape[0] == t.n_draft else x) for k, x in gd.items()}
+    compare_draft(sub, od, rows=roots)
+
+
+def test_crowded_k32_boundary_is_rescanned_exactly():
+    # the 32nd and 33rd race keys tie within ~1e-7: the list cannot prove itself complete and the
+    # row is finished by the exact second pass
+    n, V, K = 24, 600, 32
+    key, ctx, pos = _rand_ids(n, 81)
+    rng = np.random.default_rng(82)
+    logits = rng.normal(0, 1.0, (n, V)).astype(np.float32)
+    for r in range(n):
+        w = oracle.words(key[r:r + 1], ctx[r:r + 1], pos[r:r + 1], V)[0]
+        x = np.array([math.log(oracle.exp1(int(v))) for v in w])
+        s = x - logits[r]
+        order = np.argsort(s)
+        a, b = order[31], order[32 + r % 3]
+        logits[r, b] = np.float32(x[b] - s[a] + (1e-7 if r % 2 else -1e-7))
+    L = torch.as_tensor(logits).cuda()
+    ids = dev_ids(key, ctx, pos)
+    d_o = oracle.draft_rows(logits, key, ctx, pos, K, mode=oracle.DISTINCT)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    d = pps.draft_list(L, *ids, K, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    got = d["tok"].cpu().numpy()
+    for r in range(n):
+        if d_o["min_gap"][r] > 1e-12:
+            assert list(got[r]) == list(d_o["tok"][r]), (r, got[r], d_o["tok"][r])
+
+
 def test_workspace_reuse_is_deterministic():
     wl = synth.make_workload("chain4x4", n_seq=4, vocab=9000, seed=71)
     a = run_gpu(wl)
