@@ -14,19 +14,19 @@ namespace pps {
 // over the 32 consecutive tokens of an iteration, with the open segment
 // carried to the next iteration, so a warp issues one fp64 atomic per
 // segment end it sees (plus one at the end of its chunk).
-constexpr int kScoreChunk = 32 * 64;
+constexpr int kScoreAhead = 4;  // iterations whose inputs a warp loads together
 
 __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict__ tokens,
                                                        const uint64_t* __restrict__ key,
                                                        const uint64_t* __restrict__ ctx,
                                                        const uint32_t* __restrict__ pos, int64_t n, int32_t n_seg,
                                                        const int64_t* __restrict__ seg_off, ScoreParams P,
-                                                       float* out_score, double* out_sum) {
+                                                       float* out_score, double* out_sum, int64_t chunk) {
     const int lane = threadIdx.x & 31;
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t c0 = gw * kScoreChunk;
+    const int64_t c0 = gw * chunk;
     if (c0 >= n) return;
-    const int64_t c1 = min(n, c0 + (int64_t)kScoreChunk);
+    const int64_t c1 = min(n, c0 + chunk);
     // segment of the chunk's first token (binary search, lane 0)
     int seg = 0;
     if (out_sum && seg_off) {
@@ -44,20 +44,40 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
         seg = __shfl_sync(FULL, seg, 0);
     }
     double carry = 0.0;  // running sum of the open segment `seg` (warp-uniform)
-    for (int64_t base = c0; base < c1; base += 32) {
+    for (int64_t grp = c0; grp < c1; grp += 32 * kScoreAhead) {
+        // the group's inputs first: more loads in flight per warp
+        int32_t tk[kScoreAhead];
+        uint64_t kk[kScoreAhead], cx[kScoreAhead];
+        uint32_t ps[kScoreAhead];
+#pragma unroll
+        for (int u = 0; u < kScoreAhead; ++u) {
+            const int64_t t = grp + 32 * u + lane;
+            if (t < c1) {
+                tk[u] = tokens[t];
+                kk[u] = key[t];
+                cx[u] = ctx[t];
+                ps[u] = pos[t];
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kScoreAhead; ++u) {
+        const int64_t base = grp + 32 * u;
+        if (base >= c1) break;
         const int64_t t = base + lane;
         float A = 0.0f;
         if (t < c1) {
-            int64_t tok = tokens[t];
-            A = score_kind32(word_of(key[t], ctx[t], pos[t], tok, 1), P);
+            A = score_kind32(word_of(kk[u], cx[u], ps[u], (int64_t)tk[u], 1), P);
             if (out_score) out_score[t] = A;
         }
         if (!out_sum) continue;
+        // within an iteration the sums run over at most 32 fp32 scores in fp32
+        // (relative error <= 32 * 2^-24); across iterations and segments in fp64
+        // (FP64 runs at a small fraction of the FP32 rate on this part)
         if (!seg_off) {
-            double v = A;
+            float v = A;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
-            carry += v;
+            carry += (double)v;
             continue;
         }
         // segment of my token, advanced from the warp's open segment (segments are contiguous)
@@ -67,11 +87,11 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
             while (my + 1 < n_seg && seg_off[my + 1] <= t) ++my;
         }
         // segmented inclusive scan over the lanes of each segment run
-        double v = A;
+        float v = A;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            double ov = __shfl_up_sync(FULL, v, o);
-            int os = __shfl_up_sync(FULL, my, o);
+            const float ov = __shfl_up_sync(FULL, v, o);
+            const int os = __shfl_up_sync(FULL, my, o);
             if (lane >= o && os == my) v += ov;
         }
         // the carried segment ended before this iteration's first run: flush it
@@ -85,15 +105,16 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
         const bool more = base + 32 < c1;
         if (t < c1 && (lane == 31 || nxt != my)) {
             const bool open = lane == 31 && more;  // may continue into the next iteration
-            if (!open) atomicAdd(out_sum + my, v + (my == seg ? carry : 0.0));
+            if (!open) atomicAdd(out_sum + my, (double)v + (my == seg ? carry : 0.0));
         }
         if (more) {
-            const double v31 = __shfl_sync(FULL, v, 31);
+            const float v31 = __shfl_sync(FULL, v, 31);
             const int s31 = __shfl_sync(FULL, my, 31);
-            carry = v31 + (s31 == seg ? carry : 0.0);
+            carry = (double)v31 + (s31 == seg ? carry : 0.0);
             seg = s31;
         } else {
             carry = 0.0;
+        }
         }
     }
     if (out_sum && !seg_off && lane == 0) atomicAdd(out_sum, carry);
@@ -140,8 +161,9 @@ __device__ double gamma_tail_logp(int64_t M, double S) {
             wsum = fmaf((float)m, r, wsum);
             if (r < 1e-12f * sum) break;
         }
+        // tot in [1, ~1e2]: its logarithm in fp32 errs by ~1e-7 absolute
         const double tot = (double)sum + d * (double)wsum;
-        return -S + (double)(M - 1) * ls - lgamma_stirling((double)M) + log(tot);
+        return -S + (double)(M - 1) * ls - lgamma_stirling((double)M) + (double)logf((float)tot);
     }
     const double d = (S - (double)Sf) / (double)Sf;
     float r = 1.0f, sum = 1.0f, comp = 0.0f, wsum = 0.0f;
@@ -155,9 +177,11 @@ __device__ double gamma_tail_logp(int64_t M, double S) {
         wsum = fmaf((float)m, r, wsum);
         if (r < 1e-12f * sum) break;
     }
+    // S < M: P(N >= M) <= ~1/2, so ln(1 - P(N >= M)) in fp32 errs by ~1e-7 absolute; the
+    // leading term's exponent (a difference of terms ~M ln M) stays in fp64
     const double tot = (double)sum + d * (double)wsum;
     const double lead = -S + (double)M * ls - lgamma_stirling((double)M + 1.0);
-    return log1p(-exp(lead) * tot);
+    return (double)log1pf(-expf((float)lead) * (float)tot);
 }
 
 // Chernoff bound on ln P(U_1 + ... + U_M >= S): the exponent
@@ -443,10 +467,24 @@ cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const ui
         if (e != cudaSuccess) return e;
     }
     if (n > 0) {
-        int64_t warps = (n + kScoreChunk - 1) / kScoreChunk;
-        int64_t blocks = (warps * 32 + 255) / 256;
+        // one wave: as many warps as the GPU holds at once, each a contiguous chunk
+        // (a multiple of the 128 tokens of one load group)
+        static int sms = 0, occ = 0;
+        if (sms == 0) {
+            int dev = 0;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, wm_score_kernel, 256, 0);
+            if (sms <= 0) sms = 1;
+            if (occ <= 0) occ = 1;
+        }
+        const int64_t resident = (int64_t)sms * occ * (256 / 32);
+        const int64_t group = 32 * kScoreAhead;
+        const int64_t chunk = ((n + resident - 1) / resident + group - 1) / group * group;
+        const int64_t warps = (n + chunk - 1) / chunk;
+        const int64_t blocks = (warps * 32 + 255) / 256;
         wm_score_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, key, ctx, pos, n, n_seg, seg_off, P, out_score,
-                                                              out_sum);
+                                                              out_sum, chunk);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
