@@ -187,6 +187,14 @@ def cpu_model() -> str:
     return platform.machine()
 
 
+def race_workload_name(args, wl) -> str:
+    """The config's workload string of a race workload (both arms print the same one)."""
+    t = wl.tree
+    trunc = f", top-k {args.top_k}, top-p {args.top_p}" if args.top_k > 0 else ""
+    return (f"{args.workload}: B={t.n_seq}, V={wl.vocab}, K={t.K}, gamma={t.gamma}, "
+            f"{t.n_nodes} target rows + {t.n_draft} draft rows per step{trunc}")
+
+
 def oracle_sample(wl, n_draft_rows: int, n_target_rows: int, seed: int = 0, top_k: int = 0, top_p: float = 1.0):
     """Host copies of a bounded sample of the workload's rows and a timer over them."""
     import oracle
@@ -436,15 +444,13 @@ def main():
                "single_thread_value": reps1 * (nd + nn) / tot1, "cpu_model": cpu_model(),
                "nproc": os.cpu_count()}
 
-    trunc = f", top-k {args.top_k}, top-p {args.top_p}" if args.top_k > 0 else ""
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": args.steps,
             "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if wl.dtype == torch.bfloat16 else "f32",
             "data": "synthetic (seeded Zipf-rank logits; no model, no dataset)",
-            "config": {"workload": f"{args.workload}: B={t.n_seq}, V={wl.vocab}, K={t.K}, gamma={t.gamma}, "
-                                   f"{t.n_nodes} target rows + {t.n_draft} draft rows per step{trunc}",
+            "config": {"workload": race_workload_name(args, wl),
                        "rows_per_step": rows_per_step, "l2": l2_note,
                        "parallelism": f"replicas x{world}"},
             "gb_per_s": ach_all, "emitted_tokens_per_s": emitted * world / (ms_step / 1e3),
@@ -747,7 +753,7 @@ def run_reference(args, world):
     wl = synth.make_workload(args.workload, device="cuda" if torch.cuda.is_available() else "cpu",
                              K_sweep=args.k if args.workload == "ksweep" else None)
     t = wl.tree
-    run, nd, nn, cores = oracle_sample(wl, 4, 4)
+    run, nd, nn, cores = oracle_sample(wl, 4, 4, top_k=args.top_k, top_p=args.top_p)
     for _ in range(max(1, min(args.warmup, 2))):
         run()
     times = [run() for _ in range(args.steps)]
@@ -757,8 +763,8 @@ def run_reference(args, world):
         "impl": "reference", "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": f"{args.workload}: B={t.n_seq}, V={wl.vocab}, K={t.K}, gamma={t.gamma}",
-                   "rows_per_step": nd + nn},
+        "config": {"workload": race_workload_name(args, wl), "rows_per_step": nd + nn,
+                   "parallelism": f"replicas x{world}"},
         "cpu_baseline": {"value": value, "unit": "rows/s", "cores": cores, "kind": "oracle",
                          "sample": f"{nd} draft + {nn} target rows per step", "cpu_model": cpu_model(),
                          "nproc": os.cpu_count()},
