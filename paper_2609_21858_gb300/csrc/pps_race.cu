@@ -32,7 +32,7 @@
 #define PPS_UNITS 3  // 8-token units per lane per fast-loop iteration (2 Philox blocks each), draft rows
 #endif
 #ifndef PPS_UNITS_VERIFY
-#define PPS_UNITS_VERIFY 4  // the same for verify rows
+#define PPS_UNITS_VERIFY 3  // the same for verify rows and one-token draft rows
 #endif
 #ifndef PPS_PREFETCH
 #define PPS_PREFETCH 0  // 1: load the next iteration's vectors one iteration ahead (costs registers)
@@ -50,7 +50,7 @@
 #define PPS_PACKED 0  // 1: pairs of filter sums with packed fp32x2 fma/add
 #endif
 #ifndef PPS_RACE_MIN_BLOCKS
-#define PPS_RACE_MIN_BLOCKS 12  // one-warp CTAs resident per SM (register budget 168, no spills)
+#define PPS_RACE_MIN_BLOCKS 16  // one-warp CTAs resident per SM (register budget 128, no spills)
 #endif
 #ifndef PPS_BLOCK_MIN_BLOCKS
 #define PPS_BLOCK_MIN_BLOCKS 12  // the same for proposal rows of the augmented race (16 spills)
@@ -1274,13 +1274,19 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
         }
         WarpList L;
         L.reset(kp, kr);
-        // a row cut between warps shares its filter bound (verify and proposal rows: on K-list
-        // draft rows the extra registers cost more occupancy than the shared bound saves)
+        // A one-token draft list is a target race: such rows stream like verify rows (one filter
+        // test per vector).  A row cut between warps shares its filter bound (verify, one-token
+        // draft and proposal rows: on K-list draft rows the shared bound saves too little).
+        const bool one = VERIFY || (!BLK && kr == 1);
         uint32_t* slot = nullptr;
-        if constexpr (PPS_ROWBOUND && (VERIFY || BLK))
-            if (a.row_bound && (v0 > 0 || v1 < nv)) slot = a.row_bound + r;
-        stream_segment<DT, VEC, BLK, VERIFY || DT == 0, VERIFY ? PPS_UNITS_VERIFY : PPS_UNITS>(
-            L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk, slot);
+        if constexpr (PPS_ROWBOUND)
+            if ((one || BLK) && a.row_bound && (v0 > 0 || v1 < nv)) slot = a.row_bound + r;
+        if (!VERIFY && !BLK && one)
+            stream_segment<DT, VEC, false, true, PPS_UNITS_VERIFY>(L, row, a.V, v0, v1, c, key, ctx, pos, s_queue,
+                                                                 bk, slot);
+        else
+            stream_segment<DT, VEC, BLK, VERIFY || DT == 0, VERIFY ? PPS_UNITS_VERIFY : PPS_UNITS>(
+                L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk, slot);
 
         finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk, s_queue);
     }
