@@ -10,11 +10,24 @@ namespace pps {
 #define FULL 0xffffffffu
 
 // Detector (App. E): every warp takes a contiguous chunk of tokens; lane t of
-// an iteration scores token base + t.  Segment sums: a segmented warp scan
-// over the 32 consecutive tokens of an iteration, with the open segment
-// carried to the next iteration, so a warp issues one fp64 atomic per
-// segment end it sees (plus one at the end of its chunk).
+// an iteration scores token base + t, and a warp loads and scores the tokens
+// of kScoreAhead iterations (a group of 128) together.  Segment sums: when a
+// group lies inside the open segment (segments of a text are usually longer
+// than a group), each lane adds its four scores and one warp reduction adds
+// the group to the segment's running sum; a group that holds a segment
+// boundary takes a segmented warp scan per iteration.  The running sum is a
+// float-float pair (an exact fp32 two-sum per addition, FP64 being slow on this
+// part) and goes to the segment's fp64 slot with one atomic per segment end the
+// warp sees (plus one at the end of its chunk).
 constexpr int kScoreAhead = 4;  // iterations whose inputs a warp loads together
+
+// hi + lo += v, with the rounding error of hi + v kept in lo (two-sum)
+__device__ __forceinline__ void ff_add(float& hi, float& lo, float v) {
+    const float s = hi + v;
+    const float bp = s - hi;
+    lo += (hi - (s - bp)) + (v - bp);
+    hi = s;
+}
 
 __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict__ tokens,
                                                        const uint64_t* __restrict__ key,
@@ -27,9 +40,11 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
     const int64_t c0 = gw * chunk;
     if (c0 >= n) return;
     const int64_t c1 = min(n, c0 + chunk);
-    // segment of the chunk's first token (binary search, lane 0)
+    const bool segs = out_sum != nullptr && seg_off != nullptr;
+    // the open segment (warp-uniform): the segment of the chunk's first token (binary search, lane 0)
     int seg = 0;
-    if (out_sum && seg_off) {
+    int64_t seg_end = LLONG_MAX;
+    if (segs) {
         if (lane == 0) {
             int lo = 0, hi = n_seg;  // seg_off[lo] <= c0 < seg_off[hi]
             while (hi - lo > 1) {
@@ -42,8 +57,9 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
             seg = lo;
         }
         seg = __shfl_sync(FULL, seg, 0);
+        seg_end = seg + 1 < n_seg ? seg_off[seg + 1] : LLONG_MAX;
     }
-    double carry = 0.0;  // running sum of the open segment `seg` (warp-uniform)
+    float chi = 0.0f, clo = 0.0f;  // running sum of the open segment
     for (int64_t grp = c0; grp < c1; grp += 32 * kScoreAhead) {
         // the group's inputs first: more loads in flight per warp
         int32_t tk[kScoreAhead];
@@ -59,65 +75,89 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
                 ps[u] = pos[t];
             }
         }
+        float A[kScoreAhead];
 #pragma unroll
         for (int u = 0; u < kScoreAhead; ++u) {
-        const int64_t base = grp + 32 * u;
-        if (base >= c1) break;
-        const int64_t t = base + lane;
-        float A = 0.0f;
-        if (t < c1) {
-            A = score_kind32(word_of(kk[u], cx[u], ps[u], (int64_t)tk[u], 1), P);
-            if (out_score) out_score[t] = A;
+            const int64_t t = grp + 32 * u + lane;
+            A[u] = 0.0f;
+            if (t < c1) {
+                A[u] = score_kind32(word_of(kk[u], cx[u], ps[u], (int64_t)tk[u], 1), P);
+                if (out_score) out_score[t] = A[u];
+            }
         }
         if (!out_sum) continue;
-        // within an iteration the sums run over at most 32 fp32 scores in fp32
-        // (relative error <= 32 * 2^-24); across iterations and segments in fp64
-        // (FP64 runs at a small fraction of the FP32 rate on this part)
-        if (!seg_off) {
-            float v = A;
+        const int64_t gend = min(grp + 32 * kScoreAhead, c1);
+        if (segs && grp >= seg_end) {
+            // the open segment ended before this group: flush it, move to the group's first segment
+            if (lane == 0 && (chi != 0.0f || clo != 0.0f)) atomicAdd(out_sum + seg, (double)chi + (double)clo);
+            chi = clo = 0.0f;
+            do {
+                ++seg;
+            } while (seg + 1 < n_seg && seg_off[seg + 1] <= grp);
+            seg_end = seg + 1 < n_seg ? seg_off[seg + 1] : LLONG_MAX;
+        }
+        if (gend <= seg_end) {
+            // the whole group lies in the open segment (or there is one segment)
+            float v = A[0];
+#pragma unroll
+            for (int u = 1; u < kScoreAhead; ++u) v += A[u];
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
-            carry += (double)v;
+            ff_add(chi, clo, v);
             continue;
         }
-        // segment of my token, advanced from the warp's open segment (segments are contiguous)
-        int my = INT_MAX;
-        if (t < c1) {
-            my = seg;
-            while (my + 1 < n_seg && seg_off[my + 1] <= t) ++my;
-        }
-        // segmented inclusive scan over the lanes of each segment run
-        float v = A;
+        // a segment boundary inside the group: a segmented scan per iteration
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const float ov = __shfl_up_sync(FULL, v, o);
-            const int os = __shfl_up_sync(FULL, my, o);
-            if (lane >= o && os == my) v += ov;
+        for (int u = 0; u < kScoreAhead; ++u) {
+            const int64_t base = grp + 32 * u;
+            if (base >= c1) break;
+            const int64_t t = base + lane;
+            // segment of my token, advanced from the warp's open segment (segments are contiguous)
+            int my = INT_MAX;
+            if (t < c1) {
+                my = seg;
+                while (my + 1 < n_seg && seg_off[my + 1] <= t) ++my;
+            }
+            // segmented inclusive scan over the lanes of each segment run
+            float v = A[u];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const float ov = __shfl_up_sync(FULL, v, o);
+                const int os = __shfl_up_sync(FULL, my, o);
+                if (lane >= o && os == my) v += ov;
+            }
+            // the open segment ended before this iteration's first run: flush it
+            const int s0 = __shfl_sync(FULL, my, 0);
+            if (s0 != seg) {
+                if (lane == 0 && (chi != 0.0f || clo != 0.0f)) atomicAdd(out_sum + seg, (double)chi + (double)clo);
+                chi = clo = 0.0f;
+                seg = s0;
+            }
+            const int nxt = __shfl_down_sync(FULL, my, 1);
+            const bool more = base + 32 < c1;
+            if (t < c1 && (lane == 31 || nxt != my)) {
+                const bool open = lane == 31 && more;  // may continue into the next iteration
+                if (!open) atomicAdd(out_sum + my, (double)v + (my == seg ? (double)chi + (double)clo : 0.0));
+            }
+            if (more) {
+                const float v31 = __shfl_sync(FULL, v, 31);
+                const int s31 = __shfl_sync(FULL, my, 31);
+                if (s31 == seg) {
+                    ff_add(chi, clo, v31);
+                } else {
+                    chi = v31;
+                    clo = 0.0f;
+                }
+                seg = s31;
+            } else {
+                chi = clo = 0.0f;
+            }
         }
-        // the carried segment ended before this iteration's first run: flush it
-        const int s0 = __shfl_sync(FULL, my, 0);
-        if (s0 != seg) {
-            if (lane == 0 && carry != 0.0) atomicAdd(out_sum + seg, carry);
-            carry = 0.0;
-            seg = s0;
-        }
-        const int nxt = __shfl_down_sync(FULL, my, 1);
-        const bool more = base + 32 < c1;
-        if (t < c1 && (lane == 31 || nxt != my)) {
-            const bool open = lane == 31 && more;  // may continue into the next iteration
-            if (!open) atomicAdd(out_sum + my, (double)v + (my == seg ? carry : 0.0));
-        }
-        if (more) {
-            const float v31 = __shfl_sync(FULL, v, 31);
-            const int s31 = __shfl_sync(FULL, my, 31);
-            carry = (double)v31 + (s31 == seg ? carry : 0.0);
-            seg = s31;
-        } else {
-            carry = 0.0;
-        }
-        }
+        seg_end = seg + 1 < n_seg ? seg_off[seg + 1] : LLONG_MAX;
     }
-    if (out_sum && !seg_off && lane == 0) atomicAdd(out_sum, carry);
+    // the chunk's open sum (the scan path flushes its own at the chunk's end)
+    if (out_sum && lane == 0 && (chi != 0.0f || clo != 0.0f))
+        atomicAdd(out_sum + (segs ? seg : 0), (double)chi + (double)clo);
 }
 
 // ln Gamma(x) for x >= 16 by Stirling's asymptotic series (truncation error
@@ -133,23 +173,53 @@ __device__ double lgamma_stirling(double x) {
     return shift + (x - 0.5) * log(x) - x + 0.91893853320467274178 + series;
 }
 
+// Stirling's series of ln Gamma(M) - (M - 1/2) ln M + M - ln sqrt(2 pi) for M >= 16
+// (1/(12M) and its next three terms; below 1e-3 there, so fp32 suffices)
+__device__ __forceinline__ float stirling_tail(float M) {
+    const float r = 1.0f / M, r2 = r * r;
+    return r * (1.0f / 12.0f - r2 * (1.0f / 360.0f - r2 * (1.0f / 1260.0f - r2 * (1.0f / 1680.0f))));
+}
+
+// ln of the Poisson term e^-S S^k / k! for k = M - 1 (top = false) or k = M (top = true).
+// For M >= 16, with y = S/M - 1 and Stirling's formula for ln Gamma(M) (ln M! = ln Gamma(M)
+// + ln M), both are k log1p(y) - (S - M) - ln sqrt(2 pi M) - stirling_tail(M): the large
+// parts S and k ln S cancel against M and k ln M inside log1p, so one fp64 log1p is the
+// only fp64 transcendental, and the M-only terms (below ~12) are fp32 (errors < 1e-6).
+// Smaller M take ln Gamma from lgamma_stirling.
+__device__ double poisson_lead(int64_t M, double S, bool top) {
+    if (M < 16) {
+        const double ls = log(S);
+        return top ? -S + (double)M * ls - lgamma_stirling((double)M + 1.0)
+                   : -S + (double)(M - 1) * ls - lgamma_stirling((double)M);
+    }
+    const double Md = (double)M;
+    double rM = (double)(1.0f / (float)M);
+    rM = rM * (2.0 - Md * rM);  // one Newton step: relative error ~1e-14
+    const double y = (S - Md) * rM;
+    const float Mf = (float)M;
+    const float c = 0.5f * logf(6.28318530717958648f * Mf) + stirling_tail(Mf);
+    return (top ? Md : Md - 1.0) * log1p(y) - (S - Md) - (double)c;
+}
+
 // ln P(Gamma(M,1) >= S) for integer M >= 1, as the Poisson probability
 // P(N <= M-1), N ~ Poisson(S).  The leading term e^-S S^j / j! at j = M-1
-// (S >= M) or j = M (S < M) is taken in fp64; the sum of the ratios of the
-// other terms to it, all <= 1 and summed away from the mode until they stop
-// mattering, in compensated fp32 (FP64 throughput is low on this part): for
-// S >= M downward from M-1 (ratios j/S), below as 1 - P(N >= M) upward from M
-// (ratios S/j).  Relative error of the sum ~1e-7, i.e. ~1e-7 absolute in ln p.
+// (S >= M) or j = M (S < M) is taken in fp64 (poisson_lead); the sum of the
+// ratios of the other terms to it, all <= 1 and summed away from the mode
+// until they stop mattering, in compensated fp32 (FP64 throughput is low on
+// this part): for S >= M downward from M-1 (ratios j/S), below as
+// 1 - P(N >= M) upward from M (ratios S/j).  Relative error of the sum ~1e-7,
+// i.e. ~1e-7 absolute in ln p.
 __device__ double gamma_tail_logp(int64_t M, double S) {
     if (!(S > 0.0)) return 0.0;
-    const double ls = log(S);
     const float Sf = (float)S;
     // compensated (Kahan) fp32 sums; stop once a term is below 1e-12 of the sum.
     // The m-th term carries the fp32 image of S (or 1/S) m times: with its
     // relative error d, the exact sum is sum + d * sum_m m r_m to first order.
     if (S >= (double)M) {
         const float inv = 1.0f / Sf;
-        const double d = 1.0 / (S * (double)inv) - 1.0;  // (1/S) / inv - 1
+        // d = (1/S) / inv - 1 = e / (1 - e) with e = 1 - S inv (|e| < 1e-7): e + e^2
+        const double e = 1.0 - S * (double)inv;
+        const double d = fma(e, e, e);
         float r = 1.0f, sum = 1.0f, comp = 0.0f, wsum = 0.0f;
         int m = 0;
         for (int64_t j = M - 1; j > 0; --j) {
@@ -163,9 +233,9 @@ __device__ double gamma_tail_logp(int64_t M, double S) {
         }
         // tot in [1, ~1e2]: its logarithm in fp32 errs by ~1e-7 absolute
         const double tot = (double)sum + d * (double)wsum;
-        return -S + (double)(M - 1) * ls - lgamma_stirling((double)M) + (double)logf((float)tot);
+        return poisson_lead(M, S, false) + (double)logf((float)tot);
     }
-    const double d = (S - (double)Sf) / (double)Sf;
+    const double d = (S - (double)Sf) * (double)(1.0f / Sf);  // relative error of Sf (its own error ~1e-14)
     float r = 1.0f, sum = 1.0f, comp = 0.0f, wsum = 0.0f;
     int m = 0;
     for (int64_t j = M + 1;; ++j) {
@@ -177,10 +247,9 @@ __device__ double gamma_tail_logp(int64_t M, double S) {
         wsum = fmaf((float)m, r, wsum);
         if (r < 1e-12f * sum) break;
     }
-    // S < M: P(N >= M) <= ~1/2, so ln(1 - P(N >= M)) in fp32 errs by ~1e-7 absolute; the
-    // leading term's exponent (a difference of terms ~M ln M) stays in fp64
+    // S < M: P(N >= M) <= ~1/2, so ln(1 - P(N >= M)) in fp32 errs by ~1e-7 absolute
     const double tot = (double)sum + d * (double)wsum;
-    const double lead = -S + (double)M * ls - lgamma_stirling((double)M + 1.0);
+    const double lead = poisson_lead(M, S, true);
     return (double)log1pf(-expf((float)lead) * (float)tot);
 }
 
