@@ -21,6 +21,7 @@ namespace pps {
 // warp sees (plus one at the end of its chunk).
 constexpr int kScoreAhead = 4;  // iterations whose inputs a warp loads together
 
+
 // hi + lo += v, with the rounding error of hi + v kept in lo (two-sum)
 __device__ __forceinline__ void ff_add(float& hi, float& lo, float v) {
     const float s = hi + v;
@@ -60,29 +61,39 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
         seg_end = seg + 1 < n_seg ? seg_off[seg + 1] : LLONG_MAX;
     }
     float chi = 0.0f, clo = 0.0f;  // running sum of the open segment
-    for (int64_t grp = c0; grp < c1; grp += 32 * kScoreAhead) {
-        // the group's inputs first: more loads in flight per warp
+    // per-lane input pointers, advanced a group at a time (constant offsets inside a group)
+    constexpr int G = 32 * kScoreAhead;
+    const int32_t* tp = tokens + c0 + lane;
+    const uint64_t* kp = key + c0 + lane;
+    const uint64_t* xp = ctx + c0 + lane;
+    const uint32_t* pp = pos + c0 + lane;
+    for (int64_t grp = c0; grp < c1; grp += G) {
+        // the group's inputs first, more loads in flight per warp (lim: the group's tokens from
+        // this lane's first one on)
+        const int lim = (int)min((int64_t)G, c1 - grp) - lane;
         int32_t tk[kScoreAhead];
         uint64_t kk[kScoreAhead], cx[kScoreAhead];
         uint32_t ps[kScoreAhead];
 #pragma unroll
         for (int u = 0; u < kScoreAhead; ++u) {
-            const int64_t t = grp + 32 * u + lane;
-            if (t < c1) {
-                tk[u] = tokens[t];
-                kk[u] = key[t];
-                cx[u] = ctx[t];
-                ps[u] = pos[t];
+            if (32 * u < lim) {
+                tk[u] = tp[32 * u];
+                kk[u] = kp[32 * u];
+                cx[u] = xp[32 * u];
+                ps[u] = pp[32 * u];
             }
         }
+        tp += G;
+        kp += G;
+        xp += G;
+        pp += G;
         float A[kScoreAhead];
 #pragma unroll
         for (int u = 0; u < kScoreAhead; ++u) {
-            const int64_t t = grp + 32 * u + lane;
             A[u] = 0.0f;
-            if (t < c1) {
+            if (32 * u < lim) {
                 A[u] = score_kind32(word_of(kk[u], cx[u], ps[u], (int64_t)tk[u], 1), P);
-                if (out_score) out_score[t] = A[u];
+                if (out_score) out_score[grp + 32 * u + lane] = A[u];
             }
         }
         if (!out_sum) continue;
