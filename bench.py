@@ -506,12 +506,16 @@ def run_detector(args, rank, world, dev):
         sc, sums, logp = pps.wm_detect(tok, key, ctx, pos, seg, want_scores=False, stream=stream)
     torch.cuda.synchronize(dev)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk = Clocks(dev.index or 0)
     barrier(world)
+    clk.start()
+    time.sleep(0.3)
     e0.record(stream)
     for _ in range(args.steps):
         sc, sums, logp = pps.wm_detect(tok, key, ctx, pos, seg, want_scores=False, stream=stream)
     e1.record(stream)
     torch.cuda.synchronize(dev)
+    clocks = clk.stop()
     ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     # the score kernel alone (scores and segment sums, no p-values): the pass's dominant kernel
     barrier(world)
@@ -548,7 +552,7 @@ def run_detector(args, rank, world, dev):
             "detection": {"tpr_at_1pct_fpr": float(np.mean(wm <= alpha)), "fpr_null": float(np.mean(null <= alpha)),
                           "anlppt_watermarked": float(np.mean(-wm / 128.0)),
                           "anlppt_null": float(np.mean(-null / 128.0)), "segments": int(n_seg)},
-            "gpu_launches": 2 * args.steps,
+            "gpu_launches": 2 * args.steps, "clocks": clocks,
         }))
 
 
