@@ -212,52 +212,80 @@ __device__ double poisson_lead(int64_t M, double S, bool top) {
     return (top ? Md : Md - 1.0) * log1p(y) - (S - Md) - (double)c;
 }
 
+// The ratios r_m (r_0 = 1) of the Poisson terms to the leading one, summed in
+// compensated (Kahan) fp32 until a term drops below 1e-12 of the sum: downward
+// (S >= M: r_m = r_{m-1} (M - m) / S, s = 1/S in fp32) or upward (S < M:
+// r_m = r_{m-1} S / (M + m), s = S in fp32).  Also returns sum_m m r_m, the
+// first-order sensitivity to the relative error of s.  For M < kSeriesF64Min,
+// where the counters are exact in fp32 (int64 -> fp32 conversions in the loop
+// cost a quarter of the kernel).
+template <bool DOWN>
+__device__ __forceinline__ void poisson_ratios(int64_t M, float s, float& sum, float& wsum) {
+    float r = 1.0f, comp = 0.0f, m = 0.0f;
+    sum = 1.0f;
+    wsum = 0.0f;
+    for (float j = (float)(DOWN ? M - 1 : M + 1); !DOWN || j > 0.0f; j += DOWN ? -1.0f : 1.0f) {
+        r *= DOWN ? j * s : s / j;
+        m += 1.0f;
+        const float y = r - comp, t = sum + y;
+        comp = (t - sum) - y;
+        sum = t;
+        wsum = fmaf(m, r, wsum);
+        if (r < 1e-12f * sum) break;
+    }
+}
+
+// From this segment length on the series runs in fp64: with S near M, successive
+// ratios j/S differ by ~1/M, below the fp32 spacing near 1 for M ~ 2^24, so their
+// rounding errors stop averaging out and the fp32 product drifts (measured on the
+// host: 7e-7 in ln p at M = 2^16, 1.3e-5 at 2^24).  Such segments are rare; their
+// ~6 sqrt(M) fp64 steps cost microseconds.
+constexpr int64_t kSeriesF64Min = 1 << 18;
+
 // ln P(Gamma(M,1) >= S) for integer M >= 1, as the Poisson probability
 // P(N <= M-1), N ~ Poisson(S).  The leading term e^-S S^j / j! at j = M-1
 // (S >= M) or j = M (S < M) is taken in fp64 (poisson_lead); the sum of the
 // ratios of the other terms to it, all <= 1 and summed away from the mode
-// until they stop mattering, in compensated fp32 (FP64 throughput is low on
-// this part): for S >= M downward from M-1 (ratios j/S), below as
-// 1 - P(N >= M) upward from M (ratios S/j).  Relative error of the sum ~1e-7,
-// i.e. ~1e-7 absolute in ln p.
+// until they stop mattering: for S >= M downward from M-1 (ratios j/S), below
+// as 1 - P(N >= M) upward from M (ratios S/j).  Below kSeriesF64Min tokens in
+// compensated fp32 (poisson_ratios; FP64 throughput is low on this part) with a
+// first-order correction for the fp32 image of S (the m-th term carries it m
+// times: with its relative error d, the exact sum is sum + d * sum_m m r_m);
+// error below 1e-6 absolute in ln p.  From kSeriesF64Min on in fp64.
 __device__ double gamma_tail_logp(int64_t M, double S) {
     if (!(S > 0.0)) return 0.0;
+    if (M >= kSeriesF64Min) {
+        double r = 1.0, sum = 1.0;
+        if (S >= (double)M) {
+            const double inv = 1.0 / S;
+            for (int64_t j = M - 1; j > 0; --j) {
+                r *= (double)j * inv;
+                sum += r;
+                if (r < 1e-17 * sum) break;
+            }
+            return poisson_lead(M, S, false) + log(sum);
+        }
+        for (int64_t j = M + 1;; ++j) {
+            r *= S / (double)j;
+            sum += r;
+            if (r < 1e-17 * sum) break;
+        }
+        return log1p(-exp(poisson_lead(M, S, true)) * sum);
+    }
     const float Sf = (float)S;
-    // compensated (Kahan) fp32 sums; stop once a term is below 1e-12 of the sum.
-    // The m-th term carries the fp32 image of S (or 1/S) m times: with its
-    // relative error d, the exact sum is sum + d * sum_m m r_m to first order.
+    float sum, wsum;
     if (S >= (double)M) {
         const float inv = 1.0f / Sf;
         // d = (1/S) / inv - 1 = e / (1 - e) with e = 1 - S inv (|e| < 1e-7): e + e^2
         const double e = 1.0 - S * (double)inv;
         const double d = fma(e, e, e);
-        float r = 1.0f, sum = 1.0f, comp = 0.0f, wsum = 0.0f;
-        int m = 0;
-        for (int64_t j = M - 1; j > 0; --j) {
-            r *= (float)j * inv;
-            ++m;
-            const float y = r - comp, t = sum + y;
-            comp = (t - sum) - y;
-            sum = t;
-            wsum = fmaf((float)m, r, wsum);
-            if (r < 1e-12f * sum) break;
-        }
-        // tot in [1, ~1e2]: its logarithm in fp32 errs by ~1e-7 absolute
+        poisson_ratios<true>(M, inv, sum, wsum);
+        // tot in [1, ~1e3]: its logarithm in fp32 errs by ~1e-7 absolute
         const double tot = (double)sum + d * (double)wsum;
         return poisson_lead(M, S, false) + (double)logf((float)tot);
     }
     const double d = (S - (double)Sf) * (double)(1.0f / Sf);  // relative error of Sf (its own error ~1e-14)
-    float r = 1.0f, sum = 1.0f, comp = 0.0f, wsum = 0.0f;
-    int m = 0;
-    for (int64_t j = M + 1;; ++j) {
-        r *= Sf / (float)j;
-        ++m;
-        const float y = r - comp, t = sum + y;
-        comp = (t - sum) - y;
-        sum = t;
-        wsum = fmaf((float)m, r, wsum);
-        if (r < 1e-12f * sum) break;
-    }
+    poisson_ratios<false>(M, Sf, sum, wsum);
     // S < M: P(N >= M) <= ~1/2, so ln(1 - P(N >= M)) in fp32 errs by ~1e-7 absolute
     const double tot = (double)sum + d * (double)wsum;
     const double lead = poisson_lead(M, S, true);

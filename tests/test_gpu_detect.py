@@ -95,7 +95,9 @@ def test_p_values_in_watermarked_tails_and_single_segment():
     assert logp.item() < math.log(1e-3)
 
 
-@pytest.mark.parametrize("M", [1, 2, 7, 128, 1000, 4096, 20000])
+# 2^18 - 1 and 2^18: the longest segment whose Poisson series runs in fp32 and the shortest in
+# fp64; 2^24 + 5: a segment where an fp32 series would have drifted by ~1e-5
+@pytest.mark.parametrize("M", [1, 2, 7, 128, 1000, 4096, 20000, (1 << 18) - 1, 1 << 18, (1 << 24) + 5])
 def test_gamma_and_chernoff_for_one_segment_of_m_tokens(M):
     # seg_off = NULL: one segment of all M tokens; null tokens, so S is near M (Aaronson) or M/2 (U)
     tok, key, ctx, pos = _tuples(M, M)
