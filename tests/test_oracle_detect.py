@@ -42,6 +42,20 @@ def test_gamma_tail_matches_the_regularised_upper_incomplete_gamma(M, ratio):
     assert oracle.gamma_tail_logp(M, S) == pytest.approx(want, rel=1e-11, abs=1e-12)
 
 
+@pytest.mark.parametrize("M", [1 << 18, 1 << 20, (1 << 24) + 5])
+@pytest.mark.parametrize("c", [-1.5, 0.0, 3.0])
+def test_gamma_tail_of_long_segments_matches_scipy(M, c):
+    # segments of 2^18 .. 2^24 tokens, S within a few standard deviations of M, against scipy's
+    # regularised upper incomplete gamma (which agrees with mpmath to 1e-13 where mpmath
+    # converges).  The oracle's running log-term is compensated; what remains is its
+    # log-sum-exp accumulator, rescaled at each of the ~S rising terms with one rounding each:
+    # ~1e-8 at 2^24 tokens, far inside the GPU parity tolerance of 2e-6
+    sp = pytest.importorskip("scipy.special")
+    S = M + c * math.sqrt(M) + 0.31
+    want = math.log(sp.gammaincc(M, S))
+    assert oracle.gamma_tail_logp(M, S) == pytest.approx(want, rel=1e-10, abs=5e-8)
+
+
 def test_gamma_tail_p_values_are_uniform_under_the_null():
     # S_A of M independent Exp(1) scores: the p-value is U(0,1) (App. D.2)
     rng = np.random.default_rng(1)
