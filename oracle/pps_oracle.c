@@ -17,7 +17,7 @@
  *                      published multipliers and Weyl key increments.  The
  *                      paper only asks for a keyed pseudorandom function
  *                      F_{ctx,k} (Sec. 3.1, Eq. 1) / keyed source G(k,c)
- *                      (Alg. 3); Philox is this build's reading.
+ *                      (Alg. 3); Philox is the reading taken here.
  *   orc_word           the keyed source Pi_k(c): counter (token>>2, pos,
  *                      ctx_lo, ctx_hi), key (key_lo ^ (j-1)*0x9E3779B9, key_hi)
  *                      for arrival j, output lane token&3.
