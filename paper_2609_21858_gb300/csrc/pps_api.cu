@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 
 #include "pps.h"
@@ -79,6 +80,31 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratch
 constexpr int kMaxDevices = 64;
 static std::mutex g_noalloc_mu;
 static void* g_noalloc_ptr[kMaxDevices];
+
+int device_sm_count() {
+    static std::atomic<int> cache[kMaxDevices];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    int v = dev >= 0 && dev < kMaxDevices ? cache[dev].load(std::memory_order_relaxed) : 0;
+    if (v == 0) {
+        if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) v = 1;
+        if (dev >= 0 && dev < kMaxDevices) cache[dev].store(v, std::memory_order_relaxed);
+    }
+    return v;
+}
+
+int resident_ctas(int slot, const void* fn, int threads) {
+    static std::atomic<int> cache[kMaxDevices][kOccSlots];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    const bool cached = dev >= 0 && dev < kMaxDevices && slot >= 0 && slot < kOccSlots;
+    int v = cached ? cache[dev][slot].load(std::memory_order_relaxed) : 0;
+    if (v == 0) {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, fn, threads, 0) != cudaSuccess || v <= 0) v = 1;
+        if (cached) cache[dev][slot].store(v, std::memory_order_relaxed);
+    }
+    return v;
+}
 
 // Device address of the scratch on the current device (set up on first use).
 static pps_status noalloc_scratch(void** out) {

@@ -89,6 +89,17 @@ void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials
                      uint32_t** seq_cnt);
 
 // launchers (pps_race.cu)
+// Launch limits of the current device, cached per device on first use (relaxed
+// atomics: concurrent first calls from several host threads store the same value).
+// resident_ctas: CTAs of `threads` threads of kernel `fn` resident per SM; `slot`
+// (< kOccSlots) names the kernel in the cache.
+constexpr int kOccSlots = 32;
+constexpr int kOccRace = 0;    // 12 slots: dtype x (draft, verify, block) x vec
+constexpr int kOccTrunc = 12;  // 12 slots, the same
+constexpr int kOccScore = 24;
+int device_sm_count();
+int resident_ctas(int slot, const void* fn, int threads);
+
 cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
 int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk = false);
 cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);

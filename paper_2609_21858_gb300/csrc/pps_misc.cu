@@ -577,16 +577,8 @@ cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const ui
     if (n > 0) {
         // one wave: as many warps as the GPU holds at once, each a contiguous chunk
         // (a multiple of the 128 tokens of one load group)
-        static int sms = 0, occ = 0;
-        if (sms == 0) {
-            int dev = 0;
-            cudaGetDevice(&dev);
-            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, wm_score_kernel, 256, 0);
-            if (sms <= 0) sms = 1;
-            if (occ <= 0) occ = 1;
-        }
-        const int64_t resident = (int64_t)sms * occ * (256 / 32);
+        const int64_t resident =
+            (int64_t)device_sm_count() * resident_ctas(kOccScore, (const void*)wm_score_kernel, 256) * (256 / 32);
         const int64_t group = 32 * kScoreAhead;
         const int64_t chunk = ((n + resident - 1) / resident + group - 1) / group * group;
         const int64_t warps = (n + chunk - 1) / chunk;

@@ -1308,19 +1308,10 @@ static const void* race_fn(int dtype, bool verify, bool blk, bool vec) {
 }
 
 int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk) {
-    static int sms = 0, occ[2][3][2] = {};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (sms == 0) {
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (sms <= 0) sms = 1;
-    }
-    int& o = occ[dtype][verify ? 1 : (blk ? 2 : 0)][vec];
-    if (o == 0) {
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, race_fn(dtype, verify, blk && !verify, vec), kThreads, 0);
-        if (o <= 0) o = 1;
-    }
-    int64_t g = (int64_t)sms * o;
+    const int kind = verify ? 1 : (blk ? 2 : 0);
+    const int o = resident_ctas(kOccRace + (dtype * 3 + kind) * 2 + (vec ? 1 : 0),
+                                race_fn(dtype, verify, blk && !verify, vec), kThreads);
+    int64_t g = (int64_t)device_sm_count() * o;
     int64_t by_size = (total + kMinVecsPerWarp - 1) / kMinVecsPerWarp;
     if (by_size < g) g = by_size;
     if (g > kGridMax) g = kGridMax;
@@ -1373,19 +1364,10 @@ static const void* trunc_fn(int dtype, bool verify, bool blk, bool vec) {
 }
 
 int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec, bool blk) {
-    static int sms = 0, occ[2][3][2] = {};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (sms == 0) {
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (sms <= 0) sms = 1;
-    }
-    int& o = occ[dtype][verify ? 1 : (blk ? 2 : 0)][vec];
-    if (o == 0) {
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, trunc_fn(dtype, verify, blk && !verify, vec), kThreads, 0);
-        if (o <= 0) o = 1;
-    }
-    int64_t g = (int64_t)sms * o;
+    const int kind = verify ? 1 : (blk ? 2 : 0);
+    const int o = resident_ctas(kOccTrunc + (dtype * 3 + kind) * 2 + (vec ? 1 : 0),
+                                trunc_fn(dtype, verify, blk && !verify, vec), kThreads);
+    int64_t g = (int64_t)device_sm_count() * o;
     int64_t by_size = (total + kMinVecsPerWarp - 1) / kMinVecsPerWarp;
     if (by_size < g) g = by_size;
     if (n_rows > 0 && n_rows <= g) g = n_rows * (g / n_rows);
