@@ -117,9 +117,29 @@ def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
-def _stream(stream):
-    s = stream if stream is not None else torch.cuda.current_stream()
-    return ctypes.c_void_p(s.cuda_stream)
+def _stream(stream, dev=None):
+    """The stream's handle; with no stream, the current stream of `dev` (the tensors' device)."""
+    if stream is None:
+        stream = torch.cuda.current_stream(dev)
+    elif dev is not None and stream.device != dev:
+        raise ValueError(f"stream is on {stream.device}, the tensors on {dev}")
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _need(name, t, dev, dtype, numel=0, contiguous=True):
+    """Raise unless tensor `t` (skipped when None) is on `dev` with `dtype` and holds at least
+    `numel` elements: the library writes and reads through plain pointers, so a short or
+    misplaced buffer must be refused here, before anything is launched."""
+    if t is None:
+        return
+    if not isinstance(t, torch.Tensor) or not t.is_cuda or t.device != dev:
+        raise TypeError(f"{name} must be a CUDA tensor on {dev}")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if contiguous and not t.is_contiguous():
+        raise TypeError(f"{name} must be contiguous")
+    if t.numel() < numel:
+        raise ValueError(f"{name} holds {t.numel()} elements; the call needs {numel}")
 
 
 def _dtype_code(t: torch.Tensor) -> int:
@@ -130,11 +150,18 @@ def _dtype_code(t: torch.Tensor) -> int:
     raise TypeError(f"logits must be bfloat16 or float32, got {t.dtype}")
 
 
-def _ids(key, ctx, pos):
+def _ids(key, ctx, pos, n=0, dev=None):
+    """Row ids (bit patterns of the unsigned key, context label and position), n of each."""
     for name, t, dt in (("key", key, torch.int64), ("ctx", ctx, torch.int64), ("pos", pos, torch.int32)):
         if not t.is_cuda or t.dtype != dt or not t.is_contiguous():
             raise TypeError(f"{name} must be a contiguous CUDA {dt} tensor (bit pattern of the unsigned id)")
+        _need(name, t, dev if dev is not None else t.device, dt, n)
     return RowIds(key.data_ptr(), ctx.data_ptr(), pos.data_ptr())
+
+
+def _need_out(out: dict, spec, dev):
+    for name, dt, numel in spec:
+        _need(name, out.get(name), dev, dt, numel)
 
 
 def _rows(logits):
@@ -154,7 +181,19 @@ def workspace(n_rows: int, n_seq: int = 0, device=None) -> torch.Tensor:
 
 
 def workspace_clear(ws: torch.Tensor, stream=None):
-    _check("pps_workspace_clear", lib().pps_workspace_clear(_ptr(ws), ws.numel(), _stream(stream)))
+    _need("ws", ws, ws.device, torch.uint8)
+    with torch.cuda.device(ws.device):
+        _check("pps_workspace_clear", lib().pps_workspace_clear(_ptr(ws), ws.numel(), _stream(stream, ws.device)))
+
+
+def _need_draft(out, n, K, row_k, status, dev):
+    _need_out(out, [("tok", torch.int32, n * K), ("key", torch.float32, n * K), ("mult", torch.int32, n * K),
+                    ("ndist", torch.int32, n), ("samples", torch.int32, n * K)], dev)
+    for name in ("tok", "mult", "ndist"):
+        if out.get(name) is None:
+            raise TypeError(f"out[{name!r}] is required")
+    _need("row_k", row_k, dev, torch.int32, n)
+    _need("status", status, dev, torch.int32, 1)
 
 
 def draft_list(q_logits, key, ctx, pos, K: int, row_k=None, mode: int = DISTINCT, temperature: float = 1.0,
@@ -171,20 +210,22 @@ def draft_list(q_logits, key, ctx, pos, K: int, row_k=None, mode: int = DISTINCT
                    samples=torch.empty(n, K, dtype=torch.int32, device=dev) if samples else None)
     if ws is None:
         ws = workspace(n, 0, dev)
-    if row_k is not None and (row_k.dtype != torch.int32 or not row_k.is_cuda):
-        raise TypeError("row_k must be a CUDA int32 tensor")
-    if top_k > 0:
-        code = lib().pps_draft_list_trunc(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
-                                          float(temperature), int(top_k), float(top_p), int(K), _ptr(row_k),
-                                          int(mode), _ptr(out["tok"]), _ptr(out.get("key")), _ptr(out["mult"]),
-                                          _ptr(out["ndist"]), _ptr(out.get("samples")), _ptr(status), _ptr(ws),
-                                          ws.numel(), _stream(stream))
-        _check("pps_draft_list_trunc", code)
-        return out
-    code = lib().pps_draft_list(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
-                                float(temperature), int(K), _ptr(row_k), int(mode), _ptr(out["tok"]),
-                                _ptr(out.get("key")), _ptr(out["mult"]), _ptr(out["ndist"]), _ptr(out.get("samples")),
-                                _ptr(status), _ptr(ws), ws.numel(), _stream(stream))
+    _need_draft(out, n, K, row_k, status, dev)
+    _need("ws", ws, dev, torch.uint8)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        if top_k > 0:
+            code = lib().pps_draft_list_trunc(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, ids,
+                                              float(temperature), int(top_k), float(top_p), int(K), _ptr(row_k),
+                                              int(mode), _ptr(out["tok"]), _ptr(out.get("key")), _ptr(out["mult"]),
+                                              _ptr(out["ndist"]), _ptr(out.get("samples")), _ptr(status), _ptr(ws),
+                                              ws.numel(), _stream(stream, dev))
+            _check("pps_draft_list_trunc", code)
+            return out
+        code = lib().pps_draft_list(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, ids, float(temperature),
+                                    int(K), _ptr(row_k), int(mode), _ptr(out["tok"]), _ptr(out.get("key")),
+                                    _ptr(out["mult"]), _ptr(out["ndist"]), _ptr(out.get("samples")), _ptr(status),
+                                    _ptr(ws), ws.numel(), _stream(stream, dev))
     _check("pps_draft_list", code)
     return out
 
@@ -202,12 +243,13 @@ def draft_list_noalloc(q_logits, key, ctx, pos, K: int, row_k=None, mode: int = 
                    mult=torch.empty(n, K, dtype=torch.int32, device=dev),
                    ndist=torch.empty(n, dtype=torch.int32, device=dev),
                    samples=torch.empty(n, K, dtype=torch.int32, device=dev) if samples else None)
-    if row_k is not None and (row_k.dtype != torch.int32 or not row_k.is_cuda):
-        raise TypeError("row_k must be a CUDA int32 tensor")
-    code = lib().pps_draft_list_noalloc(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
-                                        float(temperature), int(K), _ptr(row_k), int(mode), _ptr(out["tok"]),
-                                        _ptr(out.get("key")), _ptr(out["mult"]), _ptr(out["ndist"]),
-                                        _ptr(out.get("samples")), _ptr(status), _stream(stream))
+    _need_draft(out, n, K, row_k, status, dev)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        code = lib().pps_draft_list_noalloc(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, ids,
+                                            float(temperature), int(K), _ptr(row_k), int(mode), _ptr(out["tok"]),
+                                            _ptr(out.get("key")), _ptr(out["mult"]), _ptr(out["ndist"]),
+                                            _ptr(out.get("samples")), _ptr(status), _stream(stream, dev))
     _check("pps_draft_list_noalloc", code)
     return out
 
@@ -232,28 +274,46 @@ def verify_tree(p_logits, key, ctx, pos, gamma: int, seq_off, node_draft_row, dr
                    score_sum=torch.empty(n_seq, dtype=torch.float64, device=dev))
     if ws is None:
         ws = workspace(n, n_seq, dev)
-    for name, t in (("seq_off", seq_off), ("node_draft_row", node_draft_row), ("draft_tok", draft_tok),
-                    ("draft_ndist", draft_ndist), ("child_node", child_node)):
-        if not t.is_cuda or t.dtype != torch.int32 or not t.is_contiguous():
-            raise TypeError(f"{name} must be a contiguous CUDA int32 tensor")
-    if top_k > 0:
-        code = lib().pps_verify_tree_trunc(_ptr(p_logits), _dtype_code(p_logits), n, V, stride, _ids(key, ctx, pos),
-                                           float(temperature), int(top_k), float(top_p), n_seq, int(gamma),
-                                           _ptr(seq_off), _ptr(node_draft_row), draft_tok.shape[0], _ptr(draft_tok),
-                                           _ptr(draft_ndist), int(K), _ptr(child_node), _ptr(out["winner"]),
-                                           _ptr(out["word"]), _ptr(out["accept_len"]), _ptr(out["n_emitted"]),
-                                           _ptr(out["emitted"]), _ptr(out["score"]), _ptr(out["score_sum"]),
-                                           _ptr(status), _ptr(ws), ws.numel(), _stream(stream))
-        _check("pps_verify_tree_trunc", code)
-        return out
-    code = lib().pps_verify_tree(_ptr(p_logits), _dtype_code(p_logits), n, V, stride, _ids(key, ctx, pos),
-                                 float(temperature), n_seq, int(gamma), _ptr(seq_off), _ptr(node_draft_row),
-                                 draft_tok.shape[0], _ptr(draft_tok), _ptr(draft_ndist), int(K), _ptr(child_node), _ptr(out["winner"]),
-                                 _ptr(out["word"]), _ptr(out["accept_len"]), _ptr(out["n_emitted"]),
-                                 _ptr(out["emitted"]), _ptr(out["score"]), _ptr(out["score_sum"]), _ptr(status),
-                                 _ptr(ws), ws.numel(), _stream(stream))
+    n_draft = draft_tok.shape[0]
+    for name, t, numel in (("seq_off", seq_off, n_seq + 1), ("node_draft_row", node_draft_row, n),
+                           ("draft_tok", draft_tok, n_draft * K), ("draft_ndist", draft_ndist, n_draft),
+                           ("child_node", child_node, n_draft * K)):
+        _need(name, t, dev, torch.int32, numel)
+    _need_out(out, [("winner", torch.int32, n), ("word", torch.int32, n), ("accept_len", torch.int32, n_seq),
+                    ("n_emitted", torch.int32, n_seq), ("emitted", torch.int32, n_seq * W),
+                    ("score", torch.float32, n_seq * W), ("score_sum", torch.float64, n_seq)], dev)
+    _need("status", status, dev, torch.int32, 1)
+    _need("ws", ws, dev, torch.uint8)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        if top_k > 0:
+            code = lib().pps_verify_tree_trunc(_ptr(p_logits), _dtype_code(p_logits), n, V, stride, ids,
+                                               float(temperature), int(top_k), float(top_p), n_seq, int(gamma),
+                                               _ptr(seq_off), _ptr(node_draft_row), n_draft, _ptr(draft_tok),
+                                               _ptr(draft_ndist), int(K), _ptr(child_node), _ptr(out["winner"]),
+                                               _ptr(out["word"]), _ptr(out["accept_len"]), _ptr(out["n_emitted"]),
+                                               _ptr(out["emitted"]), _ptr(out["score"]), _ptr(out["score_sum"]),
+                                               _ptr(status), _ptr(ws), ws.numel(), _stream(stream, dev))
+            _check("pps_verify_tree_trunc", code)
+            return out
+        code = lib().pps_verify_tree(_ptr(p_logits), _dtype_code(p_logits), n, V, stride, ids, float(temperature),
+                                     n_seq, int(gamma), _ptr(seq_off), _ptr(node_draft_row), n_draft,
+                                     _ptr(draft_tok), _ptr(draft_ndist), int(K), _ptr(child_node),
+                                     _ptr(out["winner"]), _ptr(out["word"]), _ptr(out["accept_len"]),
+                                     _ptr(out["n_emitted"]), _ptr(out["emitted"]), _ptr(out["score"]),
+                                     _ptr(out["score_sum"]), _ptr(status), _ptr(ws), ws.numel(),
+                                     _stream(stream, dev))
     _check("pps_verify_tree", code)
     return out
+
+
+def _need_detector(tokens, seg_off, n, n_seg, dev):
+    if not isinstance(tokens, torch.Tensor) or tokens.dtype != torch.int32 or not tokens.is_cuda:
+        raise TypeError("tokens must be a CUDA int32 tensor")
+    _need("tokens", tokens, dev, torch.int32, n)
+    if seg_off is not None and (seg_off.dtype != torch.int64 or not seg_off.is_cuda):
+        raise TypeError("seg_off must be a CUDA int64 tensor")
+    _need("seg_off", seg_off, dev, torch.int64, n_seg + 1)
 
 
 def wm_score(tokens, key, ctx, pos, seg_off=None, out_score=None, out_sum=None, want_scores=True, stream=None):
@@ -265,12 +325,13 @@ def wm_score(tokens, key, ctx, pos, seg_off=None, out_score=None, out_sum=None, 
         out_score = torch.empty(n, dtype=torch.float32, device=dev)
     if out_sum is None:
         out_sum = torch.empty(n_seg, dtype=torch.float64, device=dev)
-    if tokens.dtype != torch.int32 or not tokens.is_cuda:
-        raise TypeError("tokens must be a CUDA int32 tensor")
-    if seg_off is not None and (seg_off.dtype != torch.int64 or not seg_off.is_cuda):
-        raise TypeError("seg_off must be a CUDA int64 tensor")
-    code = lib().pps_wm_score(_ptr(tokens), _ids(key, ctx, pos), n, n_seg, _ptr(seg_off), _ptr(out_score),
-                              _ptr(out_sum), _stream(stream))
+    _need_detector(tokens, seg_off, n, n_seg, dev)
+    _need("out_score", out_score, dev, torch.float32, n)
+    _need("out_sum", out_sum, dev, torch.float64, n_seg)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        code = lib().pps_wm_score(_ptr(tokens), ids, n, n_seg, _ptr(seg_off), _ptr(out_score), _ptr(out_sum),
+                                  _stream(stream, dev))
     _check("pps_wm_score", code)
     return out_score, out_sum
 
@@ -281,11 +342,13 @@ def tree_expand(K: int, gamma: int, depth: int, draft, rows_key, rows_ctx, rows_
     pps_draft_list (IID) outputs of those rows; writes nxt = dict(key, ctx, pos, k) of the next
     depth's rows, child_node and nodes = dict(key, ctx, pos) in place."""
     n_seq = nxt["k"].numel() // K
-    code = lib().pps_tree_expand(n_seq, int(K), int(gamma), int(depth), _ptr(draft["tok"]), _ptr(draft["mult"]),
-                                 _ptr(draft["ndist"]), _ids(rows_key, rows_ctx, rows_pos), _ptr(row_k),
-                                 _ptr(nxt["key"]), _ptr(nxt["ctx"]), _ptr(nxt["pos"]), _ptr(nxt["k"]),
-                                 _ptr(child_node), _ptr(nodes["key"]), _ptr(nodes["ctx"]), _ptr(nodes["pos"]),
-                                 _stream(stream))
+    dev = nxt["k"].device
+    ids = _ids(rows_key, rows_ctx, rows_pos, 0, dev)
+    with torch.cuda.device(dev):
+        code = lib().pps_tree_expand(n_seq, int(K), int(gamma), int(depth), _ptr(draft["tok"]), _ptr(draft["mult"]),
+                                     _ptr(draft["ndist"]), ids, _ptr(row_k), _ptr(nxt["key"]), _ptr(nxt["ctx"]),
+                                     _ptr(nxt["pos"]), _ptr(nxt["k"]), _ptr(child_node), _ptr(nodes["key"]),
+                                     _ptr(nodes["ctx"]), _ptr(nodes["pos"]), _stream(stream, dev))
     _check("pps_tree_expand", code)
 
 
@@ -302,16 +365,23 @@ def draft_hetero(q_logits, key, ctx, pos, row_block, n_blocks: int, temperature:
         ws = workspace(n, 0, dev)
     if row_block.dtype != torch.int32 or not row_block.is_cuda or not row_block.is_contiguous():
         raise TypeError("row_block must be a contiguous CUDA int32 tensor")
-    if top_k > 0:
-        code = lib().pps_draft_hetero_trunc(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
-                                            float(temperature), int(top_k), float(top_p), _ptr(row_block),
-                                            int(n_blocks), _ptr(out_tok), _ptr(out_key), _ptr(status), _ptr(ws),
-                                            ws.numel(), _stream(stream))
-        _check("pps_draft_hetero_trunc", code)
-        return out_tok
-    code = lib().pps_draft_hetero(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, _ids(key, ctx, pos),
-                                  float(temperature), _ptr(row_block), int(n_blocks), _ptr(out_tok), _ptr(out_key),
-                                  _ptr(status), _ptr(ws), ws.numel(), _stream(stream))
+    _need("row_block", row_block, dev, torch.int32, n)
+    _need("out_tok", out_tok, dev, torch.int32, n)
+    _need("out_key", out_key, dev, torch.float32, n)
+    _need("status", status, dev, torch.int32, 1)
+    _need("ws", ws, dev, torch.uint8)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        if top_k > 0:
+            code = lib().pps_draft_hetero_trunc(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, ids,
+                                                float(temperature), int(top_k), float(top_p), _ptr(row_block),
+                                                int(n_blocks), _ptr(out_tok), _ptr(out_key), _ptr(status), _ptr(ws),
+                                                ws.numel(), _stream(stream, dev))
+            _check("pps_draft_hetero_trunc", code)
+            return out_tok
+        code = lib().pps_draft_hetero(_ptr(q_logits), _dtype_code(q_logits), n, V, stride, ids, float(temperature),
+                                      _ptr(row_block), int(n_blocks), _ptr(out_tok), _ptr(out_key), _ptr(status),
+                                      _ptr(ws), ws.numel(), _stream(stream, dev))
     _check("pps_draft_hetero", code)
     return out_tok
 
@@ -324,20 +394,28 @@ def hetero_expand(n_blocks: int, gamma: int, depth: int, draft_tok, rows_key, ro
     proposal rows (None at the last depth) in place."""
     n_seq = row_owner.numel() // n_blocks
     nx = nxt or {}
-    code = lib().pps_hetero_expand(n_seq, int(n_blocks), int(gamma), int(depth), _ptr(draft_tok),
-                                   _ids(rows_key, rows_ctx, rows_pos), _ptr(row_owner), _ptr(nx.get("key")),
-                                   _ptr(nx.get("ctx")), _ptr(nx.get("pos")), _ptr(nx.get("owner")),
-                                   _ptr(lists["tok"]), _ptr(lists["ndist"]), _ptr(lists["child"]),
-                                   _ptr(nodes["key"]), _ptr(nodes["ctx"]), _ptr(nodes["pos"]), _stream(stream))
+    dev = row_owner.device
+    ids = _ids(rows_key, rows_ctx, rows_pos, 0, dev)
+    with torch.cuda.device(dev):
+        code = lib().pps_hetero_expand(n_seq, int(n_blocks), int(gamma), int(depth), _ptr(draft_tok), ids,
+                                       _ptr(row_owner), _ptr(nx.get("key")), _ptr(nx.get("ctx")), _ptr(nx.get("pos")),
+                                       _ptr(nx.get("owner")), _ptr(lists["tok"]), _ptr(lists["ndist"]),
+                                       _ptr(lists["child"]), _ptr(nodes["key"]), _ptr(nodes["ctx"]),
+                                       _ptr(nodes["pos"]), _stream(stream, dev))
     _check("pps_hetero_expand", code)
 
 
 def hetero_block(tokens, key, ctx, pos, n_blocks: int, out=None, stream=None):
     """pps_hetero_block: the block J of the target's augmented point for each token."""
     n = tokens.numel()
+    dev = tokens.device
     if out is None:
-        out = torch.empty(n, dtype=torch.int32, device=tokens.device)
-    code = lib().pps_hetero_block(_ptr(tokens), _ids(key, ctx, pos), n, int(n_blocks), _ptr(out), _stream(stream))
+        out = torch.empty(n, dtype=torch.int32, device=dev)
+    _need_detector(tokens, None, n, 0, dev)
+    _need("out", out, dev, torch.int32, n)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        code = lib().pps_hetero_block(_ptr(tokens), ids, n, int(n_blocks), _ptr(out), _stream(stream, dev))
     _check("pps_hetero_block", code)
     return out
 
@@ -354,21 +432,22 @@ def wm_detect(tokens, key, ctx, pos, seg_off=None, kind: int = SCORE_AARONSON, p
     out_score = torch.empty(n, dtype=torch.float32, device=dev) if want_scores else None
     out_sum = torch.empty(n_seg, dtype=torch.float64, device=dev)
     out_logp = torch.empty(n_seg, dtype=torch.float64, device=dev) if want_logp else None
-    if tokens.dtype != torch.int32 or not tokens.is_cuda:
-        raise TypeError("tokens must be a CUDA int32 tensor")
-    if seg_off is not None and (seg_off.dtype != torch.int64 or not seg_off.is_cuda):
-        raise TypeError("seg_off must be a CUDA int64 tensor")
-    code = lib().pps_wm_detect(_ptr(tokens), _ids(key, ctx, pos), n, n_seg, _ptr(seg_off), int(kind), float(param),
-                               _ptr(out_score), _ptr(out_sum), _ptr(out_logp), _stream(stream))
+    _need_detector(tokens, seg_off, n, n_seg, dev)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        code = lib().pps_wm_detect(_ptr(tokens), ids, n, n_seg, _ptr(seg_off), int(kind), float(param),
+                                   _ptr(out_score), _ptr(out_sum), _ptr(out_logp), _stream(stream, dev))
     _check("pps_wm_detect", code)
     return out_score, out_sum, out_logp
 
 
 def philox_words(key, ctx, pos, vocab: int, arrival: int = 1, stream=None):
     n = key.numel()
-    out = torch.empty(n, vocab, dtype=torch.int32, device=key.device)
-    _check("pps_philox_words", lib().pps_philox_words(_ids(key, ctx, pos), n, vocab, arrival, _ptr(out),
-                                                      _stream(stream)))
+    dev = key.device
+    out = torch.empty(n, vocab, dtype=torch.int32, device=dev)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        _check("pps_philox_words", lib().pps_philox_words(ids, n, vocab, arrival, _ptr(out), _stream(stream, dev)))
     return out
 
 
