@@ -332,8 +332,10 @@ pps_status pps_hetero_block(const int32_t* tokens, pps_row_ids ids, int64_t n, i
  * n_seg, seg_off  nullable seg_off [n_seg+1]: segment g = tokens
  *              seg_off[g] .. seg_off[g+1]-1 (non-decreasing, seg_off[0] = 0,
  *              seg_off[n_seg] = n); NULL = one segment of all n tokens
- * out_score    nullable [n] A_t (fp32)
- * out_sum      nullable [n_seg] (or [1]) S_A per segment (fp64); zeroed by the call
+ * out_score    nullable [n] A_t (fp32; relative error below 2.2e-6, absolute below 2e-7)
+ * out_sum      nullable [n_seg] (or [1]) S_A per segment (fp64; the fp32 scores summed with
+ *              fp32 warp reductions into a compensated float-float running sum); zeroed by
+ *              the call
  */
 pps_status pps_wm_score(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,
                         float* out_score, double* out_sum, pps_stream_t stream);
