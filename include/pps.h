@@ -70,6 +70,7 @@ typedef struct {
 /* bits OR-ed into *status */
 #define PPS_FLAG_GUARD 1u       /* fp32 streaming filter could not prove a row's candidate set complete */
 #define PPS_FLAG_LOGIT_RANGE 2u /* |logit / T| too large for the fp32 filter's error bound (> 2^16)      */
+#define PPS_FLAG_TREE 4u        /* a sequence's root row (seq_off[s]) lies outside the node rows: nothing emitted */
 
 #define PPS_MAX_K 32
 
@@ -399,6 +400,9 @@ pps_status pps_wm_detect(const int32_t* tokens, pps_row_ids ids, int64_t n, int3
  */
 #define PPS_NOALLOC_MAX_ROWS 4096
 #define PPS_NOALLOC_MAX_WARPS 2432
+/* bytes of the array: a 272-byte partial list per (row + warp) slot, then two
+ * 32-bit counters per row: 272 * (4096 + 2432) + 8 * 4096 */
+#define PPS_NOALLOC_SCRATCH_BYTES 1808384
 pps_status pps_draft_list_noalloc(const void* q_logits, pps_dtype dtype, int64_t n_rows, int64_t vocab,
                                   int64_t row_stride, pps_row_ids ids, float temperature, int32_t K,
                                   const int32_t* row_k, pps_draft_mode mode, int32_t* out_tok, float* out_key,

@@ -16,6 +16,13 @@ small vocabularies (O(V^2) loops are fine here):
 * ``accept_distinct`` the same conditioning for the K smallest first arrivals:
                       token j lands ahead of i with probability
                       1 - exp(-e (q_j/q_i - p_j/p_i)_+), a Poisson-binomial count.
+* ``alpha_sorted``    the same alpha for a full vocabulary in O(V log V): the
+                      term (q_j/q_i - p_j/p_i)_+ is positive exactly when
+                      q_j/p_j > q_i/p_i, so with the tokens ordered by
+                      rho = q/p, alpha_i = (p_i/q_i) Q_i - P_i where Q_i and P_i
+                      sum q and p over the tokens of strictly larger rho.
+* ``accept_iid_full`` ``accept_iid`` through ``alpha_sorted`` (depth-0 acceptance
+                      of the benchmark trees at V = 128256).
 * ``bound_thm41``     1 - sum_i p_i (p_i / (p_i + q_i))^K              (Thm 4.1, Eq. 5).
 * ``bound_lml``       sum_i p_i K / (K + alpha_i)                      (App. B.3 rewrite).
 * ``bound_no_comm``   (1 - TV) / (1 + TV) (Eq. 3): the worst-case value of a
@@ -63,6 +70,40 @@ def alpha(p, q):
             s += max(q[j] / q[i] - p[j] / p[i], 0.0)
         a[i] = p[i] * s
     return a
+
+
+def alpha_sorted(p, q):
+    """alpha_i = p_i sum_j (q_j/q_i - p_j/p_i)_+ for tokens with p_i, q_i > 0, in
+    O(V log V) (tokens with p_i = 0 get alpha 0; they carry no target mass)."""
+    p = np.asarray(p, np.float64)
+    q = np.asarray(q, np.float64)
+    a = np.zeros_like(p)
+    live = (p > 0) & (q > 0)
+    pl, ql = p[live], q[live]
+    rho = ql / pl
+    order = np.argsort(rho, kind="stable")
+    rs, ps, qs = rho[order], pl[order], ql[order]
+    # suffix sums over strictly larger rho: sum over positions after the last tie of each value
+    cq = np.concatenate([np.cumsum(qs[::-1])[::-1], [0.0]])
+    cp = np.concatenate([np.cumsum(ps[::-1])[::-1], [0.0]])
+    after = np.searchsorted(rs, rs, side="right")
+    al = np.maximum(ps / qs * cq[after] - cp[after], 0.0)
+    # tokens with q_j > 0 = p_j also come ahead of every live i (rho_j = inf)
+    inf_q = float(q[(p <= 0) & (q > 0)].sum())
+    al = al + ps / qs * inf_q
+    out = np.zeros(order.size)
+    out[order] = al
+    a[live] = out
+    # tokens with p_i > 0 = q_i can never be drafted: alpha = inf (never accepted)
+    a[(p > 0) & (q <= 0)] = np.inf
+    return a
+
+
+def accept_iid_full(p, q, K: int) -> float:
+    p = np.asarray(p, np.float64)
+    a = alpha_sorted(p, q)
+    frac = np.where(np.isinf(a), 1.0, a / (1.0 + np.where(np.isinf(a), 0.0, a)))
+    return float(1.0 - np.sum(p * frac ** K))
 
 
 def accept_iid(p, q, K: int) -> float:

@@ -75,6 +75,7 @@ static RaceArgs base_args(const void* logits, pps_dtype dtype, int64_t n_rows, i
 constexpr size_t kNoAllocPartialBytes = sizeof(Partial) * (size_t)(PPS_NOALLOC_MAX_ROWS + PPS_NOALLOC_MAX_WARPS);
 constexpr size_t kNoAllocCounterBytes = sizeof(uint32_t) * 2 * (size_t)PPS_NOALLOC_MAX_ROWS;
 constexpr size_t kNoAllocScratchBytes = kNoAllocPartialBytes + kNoAllocCounterBytes;
+static_assert(kNoAllocScratchBytes == PPS_NOALLOC_SCRATCH_BYTES, "pps.h states the no-alloc scratch size");
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 constexpr int kMaxDevices = 64;

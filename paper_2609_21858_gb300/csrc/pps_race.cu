@@ -1094,7 +1094,20 @@ __device__ __forceinline__ int seq_of_node(const int32_t* seq_off, int n_seq, in
 __device__ __noinline__ void walk_sequence(const RaceArgs& a, int s, int lane) {
     const int W = a.gamma + 1;
     int c = __ldg(a.seq_off + s);
-    if (c < 0 || c >= a.n_rows) return;
+    if (c < 0 || c >= a.n_rows) {
+        // no root row: nothing emitted, and the caller learns of it through the status word
+        for (int t = lane; t < W; t += 32) {
+            a.out_em[(size_t)s * W + t] = -1;
+            a.out_sc[(size_t)s * W + t] = 0.0f;
+        }
+        if (lane == 0) {
+            a.out_acc[s] = 0;
+            a.out_ne[s] = 0;
+            a.out_ss[s] = 0.0;
+            if (a.status) atomicOr(a.status, PPS_FLAG_TREE);
+        }
+        return;
+    }
     int acc = 0, ne = 0;
     int y_[3] = {-1, -1, -1};
     uint32_t w_[3] = {0u, 0u, 0u};

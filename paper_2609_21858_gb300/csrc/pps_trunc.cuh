@@ -24,8 +24,11 @@
 // tie group: the row is then finished by a counting pass (for top-p) and, when
 // the tie group stays in S, by the exact fp32 race of pps_race.cu over the
 // tokens with logit >= l_(k).  Otherwise the finishing warp keys the <= 64
-// surviving tokens in fp64 (s = ln E - l/T, no filter and no error bound
-// needed), sorts them and emits the row exactly like the untruncated race.
+// surviving tokens with the race's fp32 key, keeps the 32 smallest and hands
+// them to finalize_row with a drop bound of +inf (S is complete, nothing was
+// dropped); finalize_row re-keys in fp64 (s = ln E - l/T) every pair closer
+// than the fp32 error bounds, so the row is emitted exactly like the
+// untruncated race.
 
 #ifndef PPS_TRUNC_UNITS
 #define PPS_TRUNC_UNITS 8  // 16-byte vectors per lane per iteration of the top-k scan (even)

@@ -15,10 +15,10 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", "libpps.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_SIZE = 0, 1, 2, 3, 4, 5
-NOALLOC_MAX_ROWS = 4096
+NOALLOC_MAX_ROWS = 4096  # PPS_NOALLOC_MAX_ROWS of include/pps.h (tests/test_abi.py checks the two agree)
 F32, BF16 = 0, 1
 DISTINCT, IID = 0, 1
-FLAG_GUARD, FLAG_LOGIT_RANGE = 1, 2
+FLAG_GUARD, FLAG_LOGIT_RANGE, FLAG_TREE = 1, 2, 4
 MAX_K = 32
 MAX_TOP_K = 64
 MAX_BLOCKS = 32

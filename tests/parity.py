@@ -15,6 +15,8 @@ import oracle
 from paper_2609_21858_gb300 import pps, synth
 
 FLIP_MARGIN = 1e-6
+# one dict per full-size comparison (flip counts, accept lengths); printed at the end of the session
+REPORT: list = []
 TOP_P_MARGIN = 1e-12  # top-p decisions closer than this to 1 - top_p may differ (exp and summation rounding)
 
 
@@ -26,6 +28,25 @@ def dev_ids(key, ctx, pos, device="cuda"):
 
 def score_rtol(dtype) -> float:
     return 1e-5 if dtype == torch.float32 else 1e-3
+
+
+# Detector p-values.  A segment is declared watermarked when ln p <= ln alpha.  The per-token scores
+# may err by SCORE_REL = 1e-5 relative (the fp32 tolerance above), which moves a segment's sum S by
+# up to 1e-5 S and its ln p by 1e-5 S |d ln p / dS|.  Evaluating ln p at the kernel's own S must add
+# no more than a tenth of that, and in any case no more than LOGP_FLOOR = 2e-6 (a relative change of
+# 2e-6 in p, which no decision at a significance level resolves).
+SCORE_REL = 1e-5
+LOGP_FLOOR = 2e-6
+
+
+def logp_tol_gamma(M: int, S: float, lnq: float) -> float:
+    """Tolerance on ln p of the Aaronson sum S of M tokens (p = Q(M, S), the regularised upper
+    incomplete gamma; d ln Q / dS = -S^(M-1) e^-S / (Gamma(M) Q))."""
+    import math
+    if M <= 0 or not (S > 0) or not math.isfinite(lnq):
+        return LOGP_FLOOR
+    dlog = math.exp(min(700.0, (M - 1) * math.log(S) - S - math.lgamma(M) - lnq))
+    return LOGP_FLOOR + 0.1 * SCORE_REL * S * dlog
 
 
 def compare_draft(g, o, rows=None, loose=None):

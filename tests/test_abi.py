@@ -186,3 +186,46 @@ def test_hetero_entry_points_validate_arguments():
     for kw in (dict(B=0), dict(B=33), dict(n=-1), dict(tok=None), dict(out=None)):
         assert block(**kw) == pps.ERR_INVALID_ARG, kw
     assert block(n=0) == pps.OK
+
+
+def _header_defines():
+    txt = open(os.path.join(ROOT, "include", "pps.h")).read()
+    return {m.group(1): int(m.group(2)) for m in re.finditer(r"#define\s+(PPS_[A-Z0-9_]+)\s+(\d+)u?\b", txt)}
+
+
+def test_binding_constants_match_the_header():
+    d = _header_defines()
+    assert d["PPS_NOALLOC_MAX_ROWS"] == pps.NOALLOC_MAX_ROWS
+    assert d["PPS_MAX_K"] == pps.MAX_K and d["PPS_MAX_TOP_K"] == pps.MAX_TOP_K and d["PPS_MAX_BLOCKS"] == pps.MAX_BLOCKS
+    assert (d["PPS_FLAG_GUARD"], d["PPS_FLAG_LOGIT_RANGE"], d["PPS_FLAG_TREE"]) == (
+        pps.FLAG_GUARD, pps.FLAG_LOGIT_RANGE, pps.FLAG_TREE)
+    # the stated scratch size: a 272-byte partial list per (row + warp) slot and two counters per row
+    assert d["PPS_NOALLOC_SCRATCH_BYTES"] == 272 * (d["PPS_NOALLOC_MAX_ROWS"] + d["PPS_NOALLOC_MAX_WARPS"]) + \
+        8 * d["PPS_NOALLOC_MAX_ROWS"]
+
+
+def test_noalloc_entry_point_rejects_bad_arguments_without_a_gpu():
+    # every refusal below returns before the scratch address is looked up (no CUDA call)
+    L = pps.lib()
+    fake = ctypes.c_void_p(256)
+    ids = pps.RowIds(256, 256, 256)
+
+    def draft(**kw):
+        a = dict(logits=fake, dtype=pps.BF16, n=4, V=100, stride=100, ids=ids, T=1.0, K=4, mode=pps.DISTINCT,
+                 tok=fake, mult=fake, nd=fake)
+        a.update(kw)
+        return L.pps_draft_list_noalloc(a["logits"], a["dtype"], a["n"], a["V"], a["stride"], a["ids"], a["T"],
+                                        a["K"], None, a["mode"], a["tok"], None, a["mult"], a["nd"], None, None, None)
+
+    assert draft(K=0) == pps.ERR_INVALID_ARG
+    assert draft(K=pps.MAX_K + 1) == pps.ERR_INVALID_ARG
+    assert draft(K=8, V=5, stride=5) == pps.ERR_INVALID_ARG
+    assert draft(stride=99) == pps.ERR_INVALID_ARG
+    assert draft(T=0.0) == pps.ERR_INVALID_ARG
+    assert draft(dtype=7) == pps.ERR_UNSUPPORTED
+    assert draft(mode=5) == pps.ERR_UNSUPPORTED
+    assert draft(ids=_ids0()) == pps.ERR_INVALID_ARG
+    for name in ("tok", "mult", "nd"):
+        assert draft(**{name: None}) == pps.ERR_INVALID_ARG, name
+    assert draft(n=pps.NOALLOC_MAX_ROWS + 1) == pps.ERR_SIZE
+    assert draft(n=0) == pps.OK

@@ -1,6 +1,6 @@
 """GPU parity: libpps (through its C ABI) against the CPU oracle on the same
 seeded inputs.  Sizes span several CTAs, rows split across CTAs and ragged
-tails; the last test runs the full benchmark workload and checks sampled rows."""
+tails; tests/test_gpu_fullsize.py runs the named configurations at full size."""
 import math
 import os
 
@@ -339,48 +339,3 @@ def test_drafter_invariance_on_gpu():
     wl.q_logits = (wl.q_logits.float() + torch.randn(wl.q_logits.shape) * 3.0).to(wl.dtype)
     _, v2, _ = run_gpu(wl)
     assert np.array_equal(v1["winner"], v2["winner"]) and np.array_equal(v1["word"], v2["word"])
-
-
-# ------------------------------------------------------------------ full size, sampled
-
-# The named configurations at their full sizes, launched as bench.py launches them: the
-# 2624 + 2112 bf16 rows of the K = 8 tree, the 65,792 + 41,216 fp32 rows of V = 152,064 of the
-# static (16, 3, 2, 1) tree (65 GB), and the K sweep's end points (K = 1, and K = 32 with
-# multi-arrival lists).  Rows are sampled for the oracle; the root rows (the longest lists) are
-# always among them.
-@pytest.mark.parametrize("name,kw,mode", [
-    ("zipf_k8", {}, pps.DISTINCT),
-    ("branch16", {}, pps.DISTINCT),
-    ("ksweep", {"K_sweep": 1}, pps.DISTINCT),
-    ("ksweep", {"K_sweep": 32}, pps.IID),
-])
-def test_full_size_sampled_rows(name, kw, mode):
-    wl = synth.make_workload(name, device="cuda", **kw)
-    t = wl.tree
-    gd, gv, status = run_gpu(wl, mode)
-    assert status == 0
-    rng = np.random.default_rng(7)
-    roots = np.nonzero(t.row_k == t.K)[0]
-    dr = np.union1d(rng.choice(roots, min(4, roots.size), replace=False),
-                    rng.choice(t.n_draft, 20, replace=False))
-    nr = np.sort(rng.choice(t.n_nodes, 24, replace=False))
-    dsel = torch.as_tensor(dr, device="cuda")
-    nsel = torch.as_tensor(nr, device="cuda")
-    od = oracle.draft_rows(wl.q_logits[dsel].float().cpu().numpy(), synth.u64(wl.draft_key[dsel]),
-                           synth.u64(wl.draft_ctx[dsel]), synth.u32(wl.draft_pos[dsel]), t.K, row_k=t.row_k[dr],
-                           mode=mode, T=float(np.float32(wl.temperature)))
-    sub = {k: (x[dr] if x is not None and x.ndim >= 1 and x.shape[0] == t.n_draft else x) for k, x in gd.items()}
-    compare_draft(sub, od, rows=dr)
-    win, wd, _, mg = oracle.target_rows(wl.p_logits[nsel].float().cpu().numpy(), synth.u64(wl.node_key[nsel]),
-                                        synth.u64(wl.node_ctx[nsel]), synth.u32(wl.node_pos[nsel]),
-                                        T=float(np.float32(wl.temperature)))
-    compare_winners(gv["winner"][nr], gv["word"][nr], win, wd, mg)
-    ow = oracle.walk(t.gamma, t.seq_off, t.node_draft_row, gd["tok"], gd["ndist"], t.child_node, gv["winner"],
-                     gv["word"])
-    assert np.array_equal(gv["accept_len"], ow["accept_len"]) and np.array_equal(gv["emitted"], ow["emitted"])
-    np.testing.assert_allclose(gv["score_sum"], ow["score_sum"], rtol=score_rtol(wl.dtype))
-    # acceptance at the root against the exact DISTINCT acceptance is checked statistically elsewhere;
-    # here the accept lengths must at least be in range
-    assert gv["accept_len"].min() >= 0 and gv["accept_len"].max() <= t.gamma
-    del wl, gd, gv
-    torch.cuda.empty_cache()

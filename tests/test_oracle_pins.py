@@ -287,6 +287,39 @@ def test_closed_forms_agree_with_each_other():
     assert cf.accept_distinct(np.array([.5, .5, 0, 0]) + 1e-300, np.array([0, 0, .5, .5]) + 1e-300, 1) < 1e-6
 
 
+def test_sorted_alpha_matches_the_pairwise_definition():
+    # alpha_sorted (suffix sums over tokens ordered by q/p) against the pairwise sum of Thm B.2,
+    # on random pairs, pairs with many equal ratios (q = p on half the tokens: those terms are 0),
+    # and pairs with masked tokens (p_j = 0 < q_j adds q_j/q_i; p_i > 0 = q_i is never drafted)
+    rng = np.random.default_rng(44)
+    for t in range(30):
+        V = int(rng.integers(2, 50))
+        lp = rng.normal(0, 2, V)
+        lq = lp + rng.normal(0, 1, V)
+        if t % 3 == 0:
+            lq[: V // 2] = lp[: V // 2]
+        p, q = cf.softmax(lp), cf.softmax(lq)
+        if t % 3 == 1 and V > 4:
+            p[0], q[1] = 0.0, 0.0
+            p, q = p / p.sum(), q / q.sum()
+        a = cf.alpha_sorted(p, q)
+        for i in range(V):
+            if p[i] <= 0:
+                continue
+            if q[i] <= 0:
+                assert a[i] == np.inf
+                continue
+            want = p[i] * sum(max(q[j] / q[i] - p[j] / p[i], 0.0) for j in range(V))
+            assert a[i] == pytest.approx(want, rel=1e-10, abs=1e-15), (t, i)
+        live = (p > 0) & (q > 0)
+        if live.all():
+            for K in (1, 4, 9):
+                assert cf.accept_iid_full(p, q, K) == pytest.approx(cf.accept_iid(p, q, K), rel=1e-12, abs=1e-15)
+    # P = Q: every ratio equal, alpha = 0, acceptance 1
+    p = cf.softmax(rng.normal(0, 1, 1000))
+    assert np.all(cf.alpha_sorted(p, p) == 0.0) and cf.accept_iid_full(p, p, 3) == pytest.approx(1.0)
+
+
 def _mc_accept(lp, lq, K, mode, n, seed):
     key, ctx, pos = _ids(n, seed)
     win, _, _, _ = oracle.target_rows(np.tile(lp, (n, 1)), key, ctx, pos)
