@@ -196,7 +196,7 @@ static pps_status draft_list(const void* q_logits, pps_dtype dtype, int64_t n_ro
         a.G = trunc_grid(a.total, a.n_rows, dt, false, vec);
         e = launch_trunc(a, dt, false, vec, (cudaStream_t)stream);
     } else {
-        a.G = race_grid(a.total, dt, false, vec);
+        a.G = race_grid(a.total, dt, false, vec, false, a.n_rows);
         e = launch_race(a, dt, false, vec, (cudaStream_t)stream);
     }
     return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
@@ -269,7 +269,7 @@ static pps_status verify_tree(const void* p_logits, pps_dtype dtype, int64_t n_n
         a.G = trunc_grid(a.total, a.n_rows, dt, true, vec);
         e = launch_trunc(a, dt, true, vec, (cudaStream_t)stream);
     } else {
-        a.G = race_grid(a.total, dt, true, vec);
+        a.G = race_grid(a.total, dt, true, vec, false, a.n_rows);
         e = launch_race(a, dt, true, vec, (cudaStream_t)stream);
     }
     return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
@@ -340,7 +340,7 @@ pps_status pps_draft_list_noalloc(const void* q_logits, pps_dtype dtype, int64_t
     a.seq_cnt = nullptr;
     const int dt = dtype == PPS_BF16 ? 1 : 0;
     const bool vec = vec_ok(q_logits, dtype, row_stride);
-    a.G = race_grid(a.total, dt, false, vec);
+    a.G = race_grid(a.total, dt, false, vec, false, a.n_rows);
     if (a.G > PPS_NOALLOC_MAX_WARPS) a.G = PPS_NOALLOC_MAX_WARPS;
     return launch_race(a, dt, false, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
 }
@@ -436,7 +436,7 @@ static pps_status draft_hetero(const void* q_logits, pps_dtype dtype, int64_t n_
         a.G = trunc_grid(a.total, a.n_rows, dt, false, vec, n_blocks > 1);
         e = launch_trunc(a, dt, false, vec, (cudaStream_t)stream);
     } else {
-        a.G = race_grid(a.total, dt, false, vec, n_blocks > 1);
+        a.G = race_grid(a.total, dt, false, vec, n_blocks > 1, a.n_rows);
         e = launch_race(a, dt, false, vec, (cudaStream_t)stream);
     }
     return e == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;

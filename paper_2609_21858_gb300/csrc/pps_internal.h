@@ -101,7 +101,7 @@ int device_sm_count();
 int resident_ctas(int slot, const void* fn, int threads);
 
 cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
-int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk = false);
+int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk = false, int64_t n_rows = 0);
 cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
 int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec, bool blk = false);
 

@@ -55,6 +55,9 @@
 #ifndef PPS_BLOCK_MIN_BLOCKS
 #define PPS_BLOCK_MIN_BLOCKS 12  // the same for proposal rows of the augmented race (16 spills)
 #endif
+#ifndef PPS_SEG_CAP
+#define PPS_SEG_CAP 30  // at most this many warp segments per row (small launches; keeps <= 32 partial lists)
+#endif
 
 namespace pps {
 
@@ -1202,9 +1205,119 @@ __device__ __noinline__ void sequence_ticket(const RaceArgs& a, int64_t r, int l
     __syncwarp();
 }
 
+// Merge the partial lists of warps first_w..last_w of row r into (lk, li) and
+// lower theta_drop to a bound on every key the merged list leaves out.  The
+// partials were written by warps all over the GPU (L2 round trips of a
+// microsecond or so), so they are loaded kMergeBatch at a time, all loads of a
+// batch in flight together, and a batch is merged as a tree (independent pairs
+// first), so that a small launch with many warps per row does not pay one
+// round trip and one dependent merge per partial.  Merging two sorted lists
+// keeps the kp smallest of their union and reports the smallest key it drops,
+// so every key left out of the result is >= the minimum of both lists' drop
+// bounds and the dropped keys.
+constexpr int kMergeBatch = 8;
+
+__device__ __forceinline__ void merge_partials(const RaceArgs& a, int64_t r, int64_t first_w, int64_t last_w, int kp,
+                                               int lane, float& lk, int& li, float& theta_drop) {
+    for (int64_t w0 = first_w; w0 <= last_w; w0 += kMergeBatch) {
+        const int nb = (int)min((int64_t)kMergeBatch, last_w - w0 + 1);  // warp-uniform
+        float pk[kMergeBatch], pd[kMergeBatch];
+        int pi[kMergeBatch];
+#pragma unroll
+        for (int b = 0; b < kMergeBatch; ++b) {
+            pk[b] = kInf;
+            pi[b] = INT_MAX;
+            pd[b] = kInf;
+            if (b < nb) {
+                const Partial* Q = a.partials + (w0 + b + r);
+                pk[b] = __ldcg(Q->key + lane);
+                pi[b] = __ldcg(Q->idx + lane);
+                pd[b] = __ldcg(&Q->theta_drop);
+            }
+        }
+        // tree: (0,1) (2,3) (4,5) (6,7), then (0,2) (4,6), then (0,4); empty lists are skipped
+#pragma unroll
+        for (int s = 1; s < kMergeBatch; s <<= 1) {
+#pragma unroll
+            for (int b = 0; b + s < kMergeBatch; b += 2 * s) {
+                if (b + s < nb) {
+                    const float dk = warp_merge<true>(pk[b], pi[b], pk[b + s], pi[b + s], kp, lane);
+                    pd[b] = fminf(fminf(pd[b], pd[b + s]), dk);
+                }
+            }
+        }
+        const float dk = warp_merge<true>(lk, li, pk[0], pi[0], kp, lane);
+        theta_drop = fminf(theta_drop, fminf(pd[0], dk));
+    }
+}
+
+// Merge by selection rounds, for at most 32 partial lists: list j is staged in
+// column j of s_k / s_i (entry e at [e * 32 + j], e < kp; one 16-byte load
+// per four entries, all lanes at once), lane j holds the head of list j, and
+// each of kp rounds moves the warp's smallest head (key, token) to entry m of
+// the merged list and advances its lane.  One warp argmin per output entry
+// replaces one dependent bitonic merge per list.  Tokens are unique across the
+// lists (disjoint segments of one row), so only the owner's head matches the
+// winner.  The smallest head left over is the smallest listed key dropped.
+__device__ __noinline__ void merge_rounds(const RaceArgs& a, int64_t r, int64_t first_w, int P, int kp, int lane,
+                                          float* s_k, int* s_i, float& lk, int& li, float& theta_drop) {
+    float th = kInf;
+    if (lane < P) {
+        const Partial* Q = a.partials + (first_w + lane + r);
+        th = __ldcg(&Q->theta_drop);
+        for (int e = 0; e < kp; e += 4) {
+            const float4 k4 = __ldcg(reinterpret_cast<const float4*>(Q->key + e));
+            const int4 i4 = __ldcg(reinterpret_cast<const int4*>(Q->idx + e));
+            s_k[(e + 0) * 32 + lane] = k4.x;
+            s_k[(e + 1) * 32 + lane] = k4.y;
+            s_k[(e + 2) * 32 + lane] = k4.z;
+            s_k[(e + 3) * 32 + lane] = k4.w;
+            s_i[(e + 0) * 32 + lane] = i4.x;
+            s_i[(e + 1) * 32 + lane] = i4.y;
+            s_i[(e + 2) * 32 + lane] = i4.z;
+            s_i[(e + 3) * 32 + lane] = i4.w;
+        }
+    }
+    __syncwarp();
+    int h = 0;
+    float hk = lane < P ? s_k[lane] : kInf;
+    int hi = lane < P ? s_i[lane] : INT_MAX;
+    lk = kInf;
+    li = INT_MAX;
+    for (int m = 0; m < kp; ++m) {
+        float bk = hk;
+        int bi = hi;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float ok = __shfl_xor_sync(FULL, bk, o);
+            const int oi = __shfl_xor_sync(FULL, bi, o);
+            if (lex_less(ok, oi, bk, bi)) {
+                bk = ok;
+                bi = oi;
+            }
+        }
+        if (bi == INT_MAX) break;  // fewer listed entries than kp (warp-uniform)
+        if (lane == m) {
+            lk = bk;
+            li = bi;
+        }
+        if (hi == bi) {
+            ++h;
+            hk = h < kp ? s_k[h * 32 + lane] : kInf;
+            hi = h < kp ? s_i[h * 32 + lane] : INT_MAX;
+        }
+    }
+    float d = fminf(hk, th);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) d = fminf(d, __shfl_xor_sync(FULL, d, o));
+    theta_drop = fminf(theta_drop, d);
+    __syncwarp();
+}
+
 template <int DT, bool VERIFY, bool BLK>
 __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_t gw, int64_t NW, int64_t v0,
-                                            int64_t v1, const WarpList L, int kr, int kp, Blk bk, uint32_t* scratch) {
+                                            int64_t v1, const WarpList L, int kr, int kp, Blk bk, uint32_t* scratch,
+                                            float* s_mk, int* s_mi) {
     const int lane = threadIdx.x & 31;
     const int64_t nv = a.nv;
     float lk = L.lk;
@@ -1237,11 +1350,10 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
             lk = kInf;
             li = INT_MAX;
             theta_drop = kInf;
-            for (int64_t ww = first_w; ww <= last_w; ++ww) {
-                const Partial* Q = a.partials + (ww + r);
-                float dk = warp_merge<true>(lk, li, __ldcg(Q->key + lane), __ldcg(Q->idx + lane), kp, lane);
-                theta_drop = fminf(theta_drop, fminf(__ldcg(&Q->theta_drop), dk));
-            }
+            if (last_w - first_w < 32)
+                merge_rounds(a, r, first_w, (int)(last_w - first_w + 1), kp, lane, s_mk, s_mi, lk, li, theta_drop);
+            else
+                merge_partials(a, r, first_w, last_w, kp, lane, lk, li, theta_drop);
         }
     }
     if (final_here) {
@@ -1261,6 +1373,8 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
 template <int DT, bool VERIFY, bool VEC, bool BLK>
 __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RACE_MIN_BLOCKS) race_kernel(const RaceArgs a) {
     __shared__ uint32_t s_queue[kQueueCap];
+    __shared__ float s_mk[32 * 32];  // staging of the partial lists merged by merge_rounds
+    __shared__ int s_mi[32 * 32];
     const int64_t NW = a.G;
     const int64_t gw = blockIdx.x;
     const int64_t g0 = gw * a.total / NW, g1 = (gw + 1) * a.total / NW;
@@ -1301,7 +1415,7 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
             stream_segment<DT, VEC, BLK, VERIFY || DT == 0, VERIFY ? PPS_UNITS_VERIFY : PPS_UNITS>(
                 L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk, slot);
 
-        finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk, s_queue);
+        finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk, s_queue, s_mk, s_mi);
     }
 }
 
@@ -1320,13 +1434,14 @@ static const void* race_fn(int dtype, bool verify, bool blk, bool vec) {
     return vec ? (const void*)race_kernel<0, false, true, false> : (const void*)race_kernel<0, false, false, false>;
 }
 
-int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk) {
+int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk, int64_t n_rows) {
     const int kind = verify ? 1 : (blk ? 2 : 0);
     const int o = resident_ctas(kOccRace + (dtype * 3 + kind) * 2 + (vec ? 1 : 0),
                                 race_fn(dtype, verify, blk && !verify, vec), kThreads);
     int64_t g = (int64_t)device_sm_count() * o;
     int64_t by_size = (total + kMinVecsPerWarp - 1) / kMinVecsPerWarp;
     if (by_size < g) g = by_size;
+    if (PPS_SEG_CAP > 0 && n_rows > 0 && n_rows * PPS_SEG_CAP < g) g = n_rows * PPS_SEG_CAP;
     if (g > kGridMax) g = kGridMax;
     if (g < 1) g = 1;
     return (int)g;
