@@ -71,6 +71,7 @@ typedef struct {
 #define PPS_FLAG_GUARD 1u       /* fp32 streaming filter could not prove a row's candidate set complete */
 #define PPS_FLAG_LOGIT_RANGE 2u /* |logit / T| too large for the fp32 filter's error bound (> 2^16)      */
 #define PPS_FLAG_TREE 4u        /* a sequence's root row (seq_off[s]) lies outside the node rows: nothing emitted */
+#define PPS_FLAG_TIMEOUT 8u     /* an LM-head kernel gave up waiting on its pipeline and returned early         */
 
 #define PPS_MAX_K 32
 
@@ -374,6 +375,59 @@ typedef enum {
 pps_status pps_wm_detect(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,
                          pps_score_kind kind, double param, float* out_score, double* out_sum, double* out_logp,
                          pps_stream_t stream);
+
+/*
+ * LM head with the race fused into it (App. B: the batched-target algorithm
+ * evaluates the target model once for every context of a draft block; the
+ * race of Alg. 2 is then the only consumer of those logits).
+ *
+ *   logits[r, i] = sum_j hidden[r, j] * weight[i, j]
+ *
+ * hidden   [n_rows, d] bf16, row stride ld_hidden elements: the last hidden
+ *          state of each context (node row or draft row)
+ * weight   [vocab, d] bf16, row stride ld_weight elements: the LM-head matrix,
+ *          one row per token
+ * The product is formed on the tensor cores (tcgen05.mma, bf16 operands, fp32
+ * accumulation) in 128 x 256 tiles with a fixed reduction order; the fp32
+ * accumulators are the logits.  Both bases must be 16-byte aligned, both row
+ * strides multiples of 8 elements (16 bytes), ld >= d; PPS_ERR_INVALID_ARG
+ * otherwise.
+ *
+ * pps_lmhead_logits writes those logits to out_logits [n_rows, ld_out] fp32
+ * (ld_out >= vocab): the unfused path, whose output the streaming entry points
+ * (pps_draft_list, pps_verify_tree with PPS_F32) take.
+ *
+ * pps_lmhead_draft_list and pps_lmhead_verify_tree compute the same outputs
+ * as pps_draft_list / pps_verify_tree would on those fp32 logits, bit for bit
+ * (tokens, words, multiplicities, accept lengths, scores), without writing the
+ * logits anywhere: the race runs on each accumulator tile in the GEMM's
+ * epilogue, and a second small kernel merges each row's partial lists and
+ * finishes the row (near-tie re-keying, IID epilogue, tree walk).  Draft lists
+ * are limited to K <= PPS_LMHEAD_MAX_K.  A row whose kept candidates cannot
+ * prove its list complete (more than one near tie at the k-th key) raises
+ * PPS_FLAG_GUARD; PPS_FLAG_TIMEOUT reports a pipeline that gave up waiting
+ * (outputs undefined).  The workspace holds the partial lists and the
+ * sequence tickets: pps_lmhead_workspace_size bytes, zeroed once before first
+ * use (pps_workspace_clear); the calls leave it ready for the next call.
+ */
+#define PPS_LMHEAD_MAX_K 8
+size_t pps_lmhead_workspace_size(int64_t n_rows, int32_t n_seq);
+pps_status pps_lmhead_logits(const void* hidden, int64_t ld_hidden, const void* weight, int64_t ld_weight,
+                             int64_t n_rows, int64_t vocab, int64_t d, float* out_logits, int64_t ld_out,
+                             pps_stream_t stream);
+pps_status pps_lmhead_draft_list(const void* hidden, int64_t ld_hidden, const void* weight, int64_t ld_weight,
+                                 int64_t n_rows, int64_t vocab, int64_t d, pps_row_ids ids, float temperature,
+                                 int32_t K, const int32_t* row_k, pps_draft_mode mode, int32_t* out_tok,
+                                 float* out_key, int32_t* out_mult, int32_t* out_ndistinct, int32_t* out_samples,
+                                 uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream);
+pps_status pps_lmhead_verify_tree(const void* hidden, int64_t ld_hidden, const void* weight, int64_t ld_weight,
+                                  int64_t n_nodes, int64_t vocab, int64_t d, pps_row_ids ids, float temperature,
+                                  int32_t n_seq, int32_t gamma, const int32_t* seq_off, const int32_t* node_draft_row,
+                                  int64_t n_draft, const int32_t* draft_tok, const int32_t* draft_ndistinct,
+                                  int32_t K, const int32_t* child_node, int32_t* out_winner, uint32_t* out_word,
+                                  int32_t* out_accept_len, int32_t* out_n_emitted, int32_t* out_emitted,
+                                  float* out_score, double* out_score_sum, uint32_t* status, void* ws,
+                                  size_t ws_bytes, pps_stream_t stream);
 
 /*
  * pps_draft_list_noalloc -- pps_draft_list for callers that must not

@@ -107,6 +107,8 @@ def lib():
             L.orc_hetero_rows.restype = None
             L.orc_truncate_rows.argtypes = [f32p, i64, i64, i64, f64, i32, f64, f32p, f64p]
             L.orc_truncate_rows.restype = None
+            L.orc_lmhead_logits.argtypes = [f32p, f32p, i64, i64, i64, f64p]
+            L.orc_lmhead_logits.restype = None
             L.orc_set_threads.argtypes = [ctypes.c_int]
             L.orc_set_threads.restype = ctypes.c_int
             _lib = L
@@ -374,3 +376,15 @@ def hetero_tree(n_seq, B, gamma):
     return dict(list_tok=np.full((nl, B), -1, np.int32), child_node=np.full((nl, B), -1, np.int32),
                 list_nd=np.zeros(nl, np.int32), node_key=np.zeros(n_seq * N1, np.uint64),
                 node_ctx=np.zeros(n_seq * N1, np.uint64), node_pos=np.zeros(n_seq * N1, np.uint32))
+
+
+def lmhead_logits(hidden, weight):
+    """logits = hidden . weight^T in fp64 (hidden [n, d], weight [V, d], fp32 images of bf16)."""
+    h = _c(hidden, np.float32)
+    w = _c(weight, np.float32)
+    n, d = h.shape
+    V = w.shape[0]
+    assert w.shape[1] == d
+    out = np.zeros((n, V), np.float64)
+    lib().orc_lmhead_logits(_ptr(h, ctypes.c_float), _ptr(w, ctypes.c_float), n, V, d, _ptr(out, ctypes.c_double))
+    return out

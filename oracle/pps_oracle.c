@@ -34,6 +34,8 @@
  *                      over every token u with Q(u) > 0 (direct finite-support
  *                      MPFR algorithm, App. B, Thm "exactness of direct
  *                      finite-support MPFR").
+ *   orc_lmhead_logits  logits = hidden . weight^T in fp64 (the LM head whose
+ *                      output the race consumes; App. B cost remark).
  *   orc_walk           follow the realised target path through the context
  *                      tree, accept while y(c*) is in D(c*), bonus token after
  *                      gamma acceptances (Alg. 4; batched algorithm, App. B).
@@ -794,6 +796,26 @@ void orc_hetero_expand(int32_t n_seq, int32_t B, int32_t gamma, int32_t depth, c
             }
         }
     }
+}
+
+/*
+ * The LM head (the last layer that produces the logits the race reads): the
+ * inner product of each context's hidden state with each token's row of the
+ * LM-head matrix, logits[r][i] = sum_j hidden[r][j] * weight[i][j], summed in
+ * fp64 in index order.  The operands are the fp32 images of bf16 values, so
+ * every product is exact in fp64; for operands whose partial sums are exactly
+ * representable (small dyadic values) the result is exact in any order.
+ */
+void orc_lmhead_logits(const float* hidden, const float* weight, int64_t n_rows, int64_t V, int64_t d,
+                       double* out)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t r = 0; r < n_rows; ++r)
+        for (int64_t i = 0; i < V; ++i) {
+            double acc = 0.0;
+            for (int64_t j = 0; j < d; ++j) acc += (double)hidden[r * d + j] * (double)weight[i * d + j];
+            out[r * V + i] = acc;
+        }
 }
 
 /* raw words of rows x vocab for a given arrival (bit-exact checks) */

@@ -1,6 +1,7 @@
 // pps_api.cu -- extern "C" entry points of libpps: argument validation,
 // workspace layout and launches.  Every entry point returns before launching
 // anything when an argument is invalid.
+#include <climits>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -343,6 +344,112 @@ pps_status pps_draft_list_noalloc(const void* q_logits, pps_dtype dtype, int64_t
     a.G = race_grid(a.total, dt, false, vec, false, a.n_rows);
     if (a.G > PPS_NOALLOC_MAX_WARPS) a.G = PPS_NOALLOC_MAX_WARPS;
     return launch_race(a, dt, false, vec, (cudaStream_t)stream) == cudaSuccess ? PPS_OK : PPS_ERR_CUDA;
+}
+
+// ---------------------------------------------------------------- LM head
+
+static pps_status check_lmhead(const void* hidden, int64_t ldh, const void* weight, int64_t ldw, int64_t n_rows,
+                               int64_t vocab, int64_t d) {
+    if (n_rows < 0 || n_rows > INT32_MAX || vocab < 1 || vocab > INT32_MAX || d < 1 || ldh < d || ldw < d)
+        return PPS_ERR_INVALID_ARG;
+    if (!weight || (n_rows > 0 && !hidden)) return PPS_ERR_INVALID_ARG;
+    // TMA: 16-byte aligned bases and 16-byte row strides
+    if (!aligned16(weight) || (hidden && !aligned16(hidden)) || ldh % 8 != 0 || ldw % 8 != 0) return PPS_ERR_INVALID_ARG;
+    return PPS_OK;
+}
+
+size_t pps_lmhead_workspace_size(int64_t n_rows, int32_t n_seq) {
+    return lmhead_workspace_bytes(n_rows < 0 ? 0 : n_rows, n_seq);
+}
+
+pps_status pps_lmhead_logits(const void* hidden, int64_t ld_hidden, const void* weight, int64_t ld_weight,
+                             int64_t n_rows, int64_t vocab, int64_t d, float* out_logits, int64_t ld_out,
+                             pps_stream_t stream) {
+    pps_status st = check_lmhead(hidden, ld_hidden, weight, ld_weight, n_rows, vocab, d);
+    if (st != PPS_OK) return st;
+    if (ld_out < vocab || (n_rows > 0 && !out_logits)) return PPS_ERR_INVALID_ARG;
+    if (n_rows == 0) return PPS_OK;
+    return launch_lmhead_logits(hidden, ld_hidden, weight, ld_weight, n_rows, vocab, d, out_logits, ld_out,
+                                (cudaStream_t)stream) == cudaSuccess
+               ? PPS_OK
+               : PPS_ERR_CUDA;
+}
+
+pps_status pps_lmhead_draft_list(const void* hidden, int64_t ld_hidden, const void* weight, int64_t ld_weight,
+                                 int64_t n_rows, int64_t vocab, int64_t d, pps_row_ids ids, float temperature,
+                                 int32_t K, const int32_t* row_k, pps_draft_mode mode, int32_t* out_tok,
+                                 float* out_key, int32_t* out_mult, int32_t* out_ndistinct, int32_t* out_samples,
+                                 uint32_t* status, void* ws, size_t ws_bytes, pps_stream_t stream) {
+    pps_status st = check_lmhead(hidden, ld_hidden, weight, ld_weight, n_rows, vocab, d);
+    if (st != PPS_OK) return st;
+    if (!(temperature > 0.0f) || !std::isfinite(temperature)) return PPS_ERR_INVALID_ARG;
+    if (n_rows > 0 && (!ids.key || !ids.ctx_hash || !ids.pos)) return PPS_ERR_INVALID_ARG;
+    if (mode != PPS_DRAFT_DISTINCT && mode != PPS_DRAFT_IID) return PPS_ERR_UNSUPPORTED;
+    if (K < 1 || K > PPS_LMHEAD_MAX_K || K > vocab) return PPS_ERR_INVALID_ARG;
+    if (n_rows == 0) return PPS_OK;
+    if (!out_tok || !out_mult || !out_ndistinct) return PPS_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < lmhead_workspace_bytes(n_rows, 0)) return PPS_ERR_WORKSPACE;
+    RaceArgs a = base_args(nullptr, PPS_F32, n_rows, vocab, vocab, ids, temperature);
+    a.K = K;
+    a.row_k = row_k;
+    a.iid = mode == PPS_DRAFT_IID;
+    a.out_tok = out_tok;
+    a.out_key = out_key;
+    a.out_mult = out_mult;
+    a.out_nd = out_ndistinct;
+    a.out_samples = out_samples;
+    a.status = status;
+    return launch_lmhead_race(hidden, ld_hidden, weight, ld_weight, d, a, false, ws, (cudaStream_t)stream) ==
+                   cudaSuccess
+               ? PPS_OK
+               : PPS_ERR_CUDA;
+}
+
+pps_status pps_lmhead_verify_tree(const void* hidden, int64_t ld_hidden, const void* weight, int64_t ld_weight,
+                                  int64_t n_nodes, int64_t vocab, int64_t d, pps_row_ids ids, float temperature,
+                                  int32_t n_seq, int32_t gamma, const int32_t* seq_off, const int32_t* node_draft_row,
+                                  int64_t n_draft, const int32_t* draft_tok, const int32_t* draft_ndistinct,
+                                  int32_t K, const int32_t* child_node, int32_t* out_winner, uint32_t* out_word,
+                                  int32_t* out_accept_len, int32_t* out_n_emitted, int32_t* out_emitted,
+                                  float* out_score, double* out_score_sum, uint32_t* status, void* ws,
+                                  size_t ws_bytes, pps_stream_t stream) {
+    pps_status st = check_lmhead(hidden, ld_hidden, weight, ld_weight, n_nodes, vocab, d);
+    if (st != PPS_OK) return st;
+    if (!(temperature > 0.0f) || !std::isfinite(temperature)) return PPS_ERR_INVALID_ARG;
+    if (n_seq < 0 || gamma < 1 || gamma > 64 || K < 1 || K > PPS_MAX_K || n_draft < 0) return PPS_ERR_INVALID_ARG;
+    if (n_nodes == 0 || n_seq == 0) return n_nodes == 0 && n_seq == 0 ? PPS_OK : PPS_ERR_INVALID_ARG;
+    if (n_nodes < n_seq) return PPS_ERR_INVALID_ARG;
+    if (!ids.key || !ids.ctx_hash || !ids.pos) return PPS_ERR_INVALID_ARG;
+    if (!seq_off || !node_draft_row || !draft_tok || !draft_ndistinct || !child_node || !out_winner || !out_word ||
+        !out_accept_len || !out_n_emitted || !out_emitted || !out_score || !out_score_sum)
+        return PPS_ERR_INVALID_ARG;
+    const size_t need = lmhead_workspace_bytes(n_nodes, n_seq);
+    if (!ws || ws_bytes < need) return PPS_ERR_WORKSPACE;
+    RaceArgs a = base_args(nullptr, PPS_F32, n_nodes, vocab, vocab, ids, temperature);
+    a.K = 1;
+    a.n_seq = n_seq;
+    a.gamma = gamma;
+    a.seq_off = seq_off;
+    a.node_draft_row = node_draft_row;
+    a.n_draft = n_draft;
+    a.draft_tok = draft_tok;
+    a.draft_nd = draft_ndistinct;
+    a.Kd = K;
+    a.child_node = child_node;
+    a.out_winner = out_winner;
+    a.out_word = out_word;
+    a.out_acc = out_accept_len;
+    a.out_ne = out_n_emitted;
+    a.out_em = out_emitted;
+    a.out_sc = out_score;
+    a.out_ss = out_score_sum;
+    a.status = status;
+    // the sequence tickets follow the partial lists
+    a.seq_cnt = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + lmhead_workspace_bytes(n_nodes, 0));
+    return launch_lmhead_race(hidden, ld_hidden, weight, ld_weight, d, a, true, ws, (cudaStream_t)stream) ==
+                   cudaSuccess
+               ? PPS_OK
+               : PPS_ERR_CUDA;
 }
 
 pps_status pps_wm_detect(const int32_t* tokens, pps_row_ids ids, int64_t n, int32_t n_seg, const int64_t* seg_off,

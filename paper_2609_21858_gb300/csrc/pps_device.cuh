@@ -106,6 +106,11 @@ struct RowPhilox {
         ctx = ((uint64_t)__reduce_or_sync(0xffffffffu, (uint32_t)(ctx >> 32)) << 32) |
               __reduce_or_sync(0xffffffffu, (uint32_t)ctx);
         pos = __reduce_or_sync(0xffffffffu, pos);
+        init_thread(key, ctx, pos);
+    }
+
+    // The same for a thread whose row is its own (the LM-head epilogue: one row per thread).
+    __device__ __forceinline__ void init_thread(uint64_t key, uint64_t ctx, uint32_t pos) {
         const uint32_t k0 = (uint32_t)key, k1 = (uint32_t)(key >> 32);
         const uint32_t c2 = (uint32_t)ctx, c3 = (uint32_t)(ctx >> 32);
         uint32_t hi1, lo1;

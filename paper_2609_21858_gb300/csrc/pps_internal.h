@@ -105,6 +105,14 @@ int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk = false,
 cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream);
 int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec, bool blk = false);
 
+// the LM-head GEMM with the race in its epilogue (pps_lmhead.cuh, in pps_race.cu).
+// hidden [n_rows, d] and weight [V, d] are bf16 with row strides ldh, ldw elements.
+size_t lmhead_workspace_bytes(int64_t n_rows, int32_t n_seq);
+cudaError_t launch_lmhead_logits(const void* hidden, int64_t ldh, const void* weight, int64_t ldw, int64_t n_rows,
+                                 int64_t V, int64_t d, float* out, int64_t ldo, cudaStream_t st);
+cudaError_t launch_lmhead_race(const void* hidden, int64_t ldh, const void* weight, int64_t ldw, int64_t d,
+                               const RaceArgs& ra, bool verify, void* ws, cudaStream_t st);
+
 // launchers (pps_misc.cu)
 // detection score kind and its constants (pps_device.cuh score_kind32)
 struct ScoreParams {

@@ -20,7 +20,11 @@
 // k-th key plus both error bounds) and re-orders near-ties with the fp64 key
 // s = ln E - l/T, so the selected tokens and their order are those of the
 // exact definition (Alg. 2, Eq. 4, App. B algorithms).
+#include <cuda.h>
+
+#include <atomic>
 #include <cfloat>
+#include <cstring>
 #include <climits>
 #include <cstdint>
 
@@ -727,15 +731,29 @@ __device__ __forceinline__ float logit_at(const RaceArgs& a, int64_t r, int64_t 
     return load_logit<DT>(base, i);
 }
 
+// Where the finishing steps read the logits of a row's listed tokens: the
+// dense row in HBM (the streaming kernels), or the table of the row's
+// candidates that the LM-head path keeps (its logits never reach HBM).
+template <int DT>
+struct DenseLogits {
+    static constexpr bool kDense = true;
+    const char* row;
+    __device__ __forceinline__ float operator()(int64_t i) const { return load_logit<DT>(row, i); }
+};
+template <int DT>
+__device__ __forceinline__ DenseLogits<DT> dense_logits(const RaceArgs& a, int64_t r) {
+    return DenseLogits<DT>{reinterpret_cast<const char*>(a.logits) + (size_t)r * (size_t)a.stride * (DT == 1 ? 2 : 4)};
+}
+
 __device__ void walk_sequence(const RaceArgs& a, int s, int lane);
 
 // Outputs of row r from its sorted entries: lane m holds the m-th smallest
 // (key, token) of the row's list (dk fp64 when exact, sk fp32), nvalid of them
 // usable.  Verify rows: the winner and its word.  Draft rows: the list, its
 // multiplicities and labels (IID: the kr smallest multi-arrival scores).
-template <int DT, bool VERIFY>
+template <int DT, bool VERIFY, class LP>
 __device__ __forceinline__ void emit_row(const RaceArgs& a, int64_t r, double dk, float sk, int li, int nvalid, int kr,
-                                         int lane, uint64_t key, uint64_t ctx, uint32_t pos) {
+                                         int lane, uint64_t key, uint64_t ctx, uint32_t pos, const LP& lp) {
     if (VERIFY) {
         int win = __shfl_sync(FULL, li, 0);
         if (nvalid == 0) win = -1;
@@ -756,7 +774,7 @@ __device__ __forceinline__ void emit_row(const RaceArgs& a, int64_t r, double dk
         // the kr smallest (ties by token, then arrival) are the samples
         mult = 0;
         sample = -1;
-        float lt = mine ? logit_at<DT>(a, r, li) : 0.0f;
+        float lt = mine ? lp(li) : 0.0f;
         double G = mine ? exp1_f64(word_of(key, ctx, pos, li, 1)) : 0.0;
         double h = mine ? dk : (double)INFINITY;
         int j = 1;
@@ -815,13 +833,13 @@ __device__ __forceinline__ void emit_row(const RaceArgs& a, int64_t r, double dk
 // bounds, the samples and their order are those of the exact scores and the
 // row is written here; otherwise it returns false and the caller re-keys the
 // row in fp64 (emit_row).
-template <int DT>
+template <int DT, class LP>
 __device__ __noinline__ bool iid_fast(const RaceArgs& a, int64_t r, float lk, int li, int nvalid, int kr, int lane,
-                                      uint64_t key, uint64_t ctx, uint32_t pos) {
+                                      uint64_t key, uint64_t ctx, uint32_t pos, const LP lp) {
     const int nuse = min(nvalid, kr);
     const bool mine = lane < nuse;
     const int tok = mine ? li : -1;
-    const float lt = mine ? logit_at<DT>(a, r, li) : 0.0f;
+    const float lt = mine ? lp(li) : 0.0f;
     float y = mine ? neg_log2_u(word_of(key, ctx, pos, li, 1)) : 0.0f;
     float h = mine ? lk : kInf;  // arrival 1's score is the list key itself
     int j = 1, mult = 0, sample = -1, nsel = 0;
@@ -1014,9 +1032,9 @@ __device__ __noinline__ bool rescan_row(const RaceArgs& a, int64_t r, float tau,
 
 // Warp 0 finishes row r from its complete list (lk, li) and the drop bound.
 // BLK: the near-tie keys are those of the row's block arrivals.
-template <int DT, bool VERIFY, bool BLK = false>
-__device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk, int li, float theta_drop, int kr,
-                                          int kp, int lane, Blk bk = Blk{}, uint32_t* scratch = nullptr) {
+template <int DT, bool VERIFY, bool BLK, class LP>
+__device__ __forceinline__ void finalize_row_lp(const RaceArgs& a, int64_t r, float lk, int li, float theta_drop,
+                                                int kr, int kp, int lane, const LP& lp, Blk bk, uint32_t* scratch) {
     const int nvalid = __popc(__ballot_sync(FULL, lane < kp && lk < kInf));
     const float tau = nvalid >= kr ? __shfl_sync(FULL, lk, kr - 1) : kInf;
     // list-key error bound (block rows: widened by kBlkErr)
@@ -1028,13 +1046,13 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
         complete = true;
     else
         complete = theta_drop == kInf || theta_drop > tau + err(tau) + err(theta_drop);
-    if (!complete && nvalid >= kr && scratch != nullptr) {
+    if (LP::kDense && !complete && nvalid >= kr && scratch != nullptr) {
         // the boundary is crowded: finish the row exactly with one more pass
         double dkr;
         int lir, nvr;
         if (rescan_row<DT, BLK>(a, r, tau, kr, lane, bk, scratch, dkr, lir, nvr)) {
             if (lane == 0 && a.status && tau > -kInf && fabsf(tau) > 65536.0f) atomicOr(a.status, PPS_FLAG_LOGIT_RANGE);
-            emit_row<DT, VERIFY>(a, r, dkr, (float)dkr, lir, nvr, kr, lane, a.key[r], a.ctx[r], a.pos[r]);
+            emit_row<DT, VERIFY>(a, r, dkr, (float)dkr, lir, nvr, kr, lane, a.key[r], a.ctx[r], a.pos[r], lp);
             return;
         }
     }
@@ -1051,7 +1069,7 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
     const uint64_t key = a.key[r], ctx = a.ctx[r];
     const uint32_t pos = a.pos[r];
     if constexpr (!VERIFY && !BLK) {
-        if (a.iid && !any_close && PPS_IID_FAST && iid_fast<DT>(a, r, lk, li, nvalid, kr, lane, key, ctx, pos))
+        if (a.iid && !any_close && PPS_IID_FAST && iid_fast<DT>(a, r, lk, li, nvalid, kr, lane, key, ctx, pos, lp))
             return;
     }
     const bool need_exact = any_close || (!VERIFY && a.iid);
@@ -1063,14 +1081,21 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
             if constexpr (BLK) {
                 uint32_t wf;
                 const int J = block_words(key, ctx, pos, li, bk.b, bk.B, wf);
-                dk = block_key64(w, J, wf, bk.b, bk.B, logit_at<DT>(a, r, li), a.T);
+                dk = block_key64(w, J, wf, bk.b, bk.B, lp(li), a.T);
             } else
-                dk = key64(w, logit_at<DT>(a, r, li), a.T);
+                dk = key64(w, lp(li), a.T);
         }
         warp_sort_d(dk, li, lane);
         sk = (float)dk;
     }
-    emit_row<DT, VERIFY>(a, r, dk, sk, li, nvalid, kr, lane, key, ctx, pos);
+    emit_row<DT, VERIFY>(a, r, dk, sk, li, nvalid, kr, lane, key, ctx, pos, lp);
+}
+
+// Warp 0 finishes row r of a streamed logits matrix from its complete list.
+template <int DT, bool VERIFY, bool BLK = false>
+__device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk, int li, float theta_drop, int kr,
+                                          int kp, int lane, Blk bk = Blk{}, uint32_t* scratch = nullptr) {
+    finalize_row_lp<DT, VERIFY, BLK>(a, r, lk, li, theta_drop, kr, kp, lane, dense_logits<DT>(a, r), bk, scratch);
 }
 
 __device__ __forceinline__ int64_t warp_of(int64_t g, int64_t total, int64_t NW) {
@@ -1421,6 +1446,7 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
 
 
 #include "pps_trunc.cuh"
+#include "pps_lmhead.cuh"
 
 // the race kernel instance: dtype x (verify | block draft | draft) x vec
 static const void* race_fn(int dtype, bool verify, bool blk, bool vec) {

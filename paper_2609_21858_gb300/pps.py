@@ -18,10 +18,11 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_SIZE = 0, 1, 
 NOALLOC_MAX_ROWS = 4096  # PPS_NOALLOC_MAX_ROWS of include/pps.h (tests/test_abi.py checks the two agree)
 F32, BF16 = 0, 1
 DISTINCT, IID = 0, 1
-FLAG_GUARD, FLAG_LOGIT_RANGE, FLAG_TREE = 1, 2, 4
+FLAG_GUARD, FLAG_LOGIT_RANGE, FLAG_TREE, FLAG_TIMEOUT = 1, 2, 4, 8
 MAX_K = 32
 MAX_TOP_K = 64
 MAX_BLOCKS = 32
+LMHEAD_MAX_K = 8
 
 _lock = threading.Lock()
 _lib = None
@@ -88,6 +89,16 @@ def lib():
             L.pps_hetero_expand.restype = ctypes.c_int
             L.pps_hetero_block.argtypes = [vp, RowIds, i64, i32, vp, vp]
             L.pps_hetero_block.restype = ctypes.c_int
+            L.pps_lmhead_workspace_size.argtypes = [i64, i32]
+            L.pps_lmhead_workspace_size.restype = sz
+            L.pps_lmhead_logits.argtypes = [vp, i64, vp, i64, i64, i64, i64, vp, i64, vp]
+            L.pps_lmhead_logits.restype = ctypes.c_int
+            L.pps_lmhead_draft_list.argtypes = [vp, i64, vp, i64, i64, i64, i64, RowIds, f32, i32, vp, ctypes.c_int,
+                                                vp, vp, vp, vp, vp, vp, vp, sz, vp]
+            L.pps_lmhead_draft_list.restype = ctypes.c_int
+            L.pps_lmhead_verify_tree.argtypes = [vp, i64, vp, i64, i64, i64, i64, RowIds, f32, i32, i32, vp, vp, i64,
+                                                 vp, vp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+            L.pps_lmhead_verify_tree.restype = ctypes.c_int
             L.pps_philox_words.argtypes = [RowIds, i64, i64, i32, vp, vp]
             L.pps_philox_words.restype = ctypes.c_int
             L.pps_selftest_philox_rate.argtypes = [u64, vp, i32, vp]
@@ -469,4 +480,110 @@ def selftest_philox_rate(n_blocks: int, out_len: int, stream=None):
     """Launch the Philox-only throughput kernel (returns the folded words)."""
     out = torch.empty(out_len, dtype=torch.int32, device="cuda")
     _check("pps_selftest_philox_rate", lib().pps_selftest_philox_rate(n_blocks, _ptr(out), out_len, _stream(stream)))
+    return out
+
+
+# ---------------------------------------------------------------- LM head (the race fused into the GEMM)
+
+def _lm_operands(hidden, weight):
+    """Shapes and strides of the bf16 hidden states [n, d] and LM-head matrix [V, d]."""
+    for name, t in (("hidden", hidden), ("weight", weight)):
+        if not isinstance(t, torch.Tensor) or not t.is_cuda or t.dim() != 2 or t.stride(1) != 1:
+            raise TypeError(f"{name} must be a 2-D CUDA tensor with unit stride along d")
+        if t.dtype != torch.bfloat16:
+            raise TypeError(f"{name} must be bfloat16, got {t.dtype}")
+    if hidden.device != weight.device:
+        raise ValueError("hidden and weight must be on the same device")
+    if hidden.shape[1] != weight.shape[1]:
+        raise ValueError(f"hidden has d={hidden.shape[1]}, weight d={weight.shape[1]}")
+    return hidden.shape[0], weight.shape[0], hidden.shape[1], hidden.stride(0), weight.stride(0)
+
+
+def lmhead_workspace(n_rows: int, n_seq: int = 0, device=None) -> torch.Tensor:
+    """A zeroed workspace for the fused LM-head calls."""
+    nb = int(lib().pps_lmhead_workspace_size(n_rows, n_seq))
+    return torch.zeros(nb, dtype=torch.uint8, device=device or "cuda")
+
+
+def lmhead_logits(hidden, weight, out=None, stream=None):
+    """pps_lmhead_logits: fp32 logits = hidden @ weight^T on the tensor cores (the unfused path)."""
+    n, V, d, ldh, ldw = _lm_operands(hidden, weight)
+    dev = hidden.device
+    if out is None:
+        out = torch.empty(n, V, dtype=torch.float32, device=dev)
+    if out.dtype != torch.float32 or out.device != dev or out.dim() != 2 or out.stride(1) != 1 or \
+            out.shape[0] < n or out.shape[1] < V:
+        raise TypeError("out must be a float32 [n_rows, >= vocab] tensor on the operands' device")
+    with torch.cuda.device(dev):
+        code = lib().pps_lmhead_logits(_ptr(hidden), ldh, _ptr(weight), ldw, n, V, d, _ptr(out), out.stride(0),
+                                       _stream(stream, dev))
+    _check("pps_lmhead_logits", code)
+    return out
+
+
+def lmhead_draft_list(hidden, weight, key, ctx, pos, K: int, row_k=None, mode: int = DISTINCT,
+                      temperature: float = 1.0, ws=None, status=None, out=None, keys: bool = True,
+                      samples: bool = True, stream=None):
+    """pps_lmhead_draft_list: the draft lists of pps_draft_list, computed in the LM-head GEMM's epilogue."""
+    n, V, d, ldh, ldw = _lm_operands(hidden, weight)
+    dev = hidden.device
+    if out is None:
+        out = dict(tok=torch.empty(n, K, dtype=torch.int32, device=dev),
+                   key=torch.empty(n, K, dtype=torch.float32, device=dev) if keys else None,
+                   mult=torch.empty(n, K, dtype=torch.int32, device=dev),
+                   ndist=torch.empty(n, dtype=torch.int32, device=dev),
+                   samples=torch.empty(n, K, dtype=torch.int32, device=dev) if samples else None)
+    if ws is None:
+        ws = lmhead_workspace(n, 0, dev)
+    _need_draft(out, n, K, row_k, status, dev)
+    _need("ws", ws, dev, torch.uint8)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        code = lib().pps_lmhead_draft_list(_ptr(hidden), ldh, _ptr(weight), ldw, n, V, d, ids, float(temperature),
+                                           int(K), _ptr(row_k), int(mode), _ptr(out["tok"]), _ptr(out.get("key")),
+                                           _ptr(out["mult"]), _ptr(out["ndist"]), _ptr(out.get("samples")),
+                                           _ptr(status), _ptr(ws), ws.numel(), _stream(stream, dev))
+    _check("pps_lmhead_draft_list", code)
+    return out
+
+
+def lmhead_verify_tree(hidden, weight, key, ctx, pos, gamma: int, seq_off, node_draft_row, draft_tok, draft_ndist,
+                       child_node, temperature: float = 1.0, ws=None, status=None, out=None, stream=None):
+    """pps_lmhead_verify_tree: the target race of every node, the tree walk and the scores of
+    pps_verify_tree, computed in the LM-head GEMM's epilogue."""
+    n, V, d, ldh, ldw = _lm_operands(hidden, weight)
+    dev = hidden.device
+    n_seq = seq_off.numel() - 1
+    K = draft_tok.shape[1]
+    W = gamma + 1
+    if out is None:
+        out = dict(winner=torch.empty(n, dtype=torch.int32, device=dev),
+                   word=torch.empty(n, dtype=torch.int32, device=dev),
+                   accept_len=torch.empty(n_seq, dtype=torch.int32, device=dev),
+                   n_emitted=torch.empty(n_seq, dtype=torch.int32, device=dev),
+                   emitted=torch.empty(n_seq, W, dtype=torch.int32, device=dev),
+                   score=torch.empty(n_seq, W, dtype=torch.float32, device=dev),
+                   score_sum=torch.empty(n_seq, dtype=torch.float64, device=dev))
+    if ws is None:
+        ws = lmhead_workspace(n, n_seq, dev)
+    n_draft = draft_tok.shape[0]
+    for name, t, numel in (("seq_off", seq_off, n_seq + 1), ("node_draft_row", node_draft_row, n),
+                           ("draft_tok", draft_tok, n_draft * K), ("draft_ndist", draft_ndist, n_draft),
+                           ("child_node", child_node, n_draft * K)):
+        _need(name, t, dev, torch.int32, numel)
+    _need_out(out, [("winner", torch.int32, n), ("word", torch.int32, n), ("accept_len", torch.int32, n_seq),
+                    ("n_emitted", torch.int32, n_seq), ("emitted", torch.int32, n_seq * W),
+                    ("score", torch.float32, n_seq * W), ("score_sum", torch.float64, n_seq)], dev)
+    _need("status", status, dev, torch.int32, 1)
+    _need("ws", ws, dev, torch.uint8)
+    ids = _ids(key, ctx, pos, n, dev)
+    with torch.cuda.device(dev):
+        code = lib().pps_lmhead_verify_tree(_ptr(hidden), ldh, _ptr(weight), ldw, n, V, d, ids, float(temperature),
+                                            n_seq, int(gamma), _ptr(seq_off), _ptr(node_draft_row), n_draft,
+                                            _ptr(draft_tok), _ptr(draft_ndist), int(K), _ptr(child_node),
+                                            _ptr(out["winner"]), _ptr(out["word"]), _ptr(out["accept_len"]),
+                                            _ptr(out["n_emitted"]), _ptr(out["emitted"]), _ptr(out["score"]),
+                                            _ptr(out["score_sum"]), _ptr(status), _ptr(ws), ws.numel(),
+                                            _stream(stream, dev))
+    _check("pps_lmhead_verify_tree", code)
     return out

@@ -296,3 +296,61 @@ def label_logits(labels, V: int, seed: int = 0, zipf: float = 1.0, noise: float 
     rank = np.empty_like(perm)
     np.put_along_axis(rank, perm, np.arange(1, V + 1).reshape(1, -1).repeat(lab.shape[0], 0), axis=1)
     return (-zipf * np.log(rank) + noise * g).astype(np.float32)
+
+
+# --- LM-head operands (the fused race takes hidden states and weights, not logits) ----------
+
+@dataclass
+class LmHeadWorkload:
+    tree: Tree
+    vocab: int
+    hp: torch.Tensor        # [n_nodes, d_target] bf16 hidden states of the target model, one per node
+    wp: torch.Tensor        # [V, d_target] bf16 target LM-head matrix
+    hq: torch.Tensor        # [n_draft, d_draft] bf16 hidden states of the draft model, one per draft row
+    wq: torch.Tensor        # [V, d_draft] bf16 draft LM-head matrix
+    node_key: torch.Tensor
+    node_ctx: torch.Tensor
+    node_pos: torch.Tensor
+    draft_key: torch.Tensor
+    draft_ctx: torch.Tensor
+    draft_pos: torch.Tensor
+    temperature: float = 1.0
+    recipe: str = ""
+
+
+def lmhead_workload(n_seq: int = 64, branching=(8, 1, 1, 1, 1), vocab: int = 128256, d_target: int = 4096,
+                    d_draft: int = 2048, seed: int = 5, device="cpu") -> LmHeadWorkload:
+    """Operands whose products are Zipf-shaped logits, like the zipf_k8 workload but produced by
+    an LM head: column 0 of every hidden state is 1 and column 0 of weight row i is -ln(rank_i)
+    (one random permutation of the ranks: the model's token frequencies); the other columns are
+    N(0, 1) (hidden) and N(0, 1/(d-1)) (weights), so target logits are -ln(rank) + N(0, 1).  The
+    draft model reads the first d_draft columns of the same hidden states with its weight columns
+    1..d_draft-1 equal to the target's, scaled to unit variance: draft logits = -ln(rank) + a noise
+    correlated ~sqrt((d_draft-1)/(d_target-1)) with the target's."""
+    assert 2 <= d_draft <= d_target
+    tree = make_tree(tuple(branching), n_seq)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    V = vocab
+    rank = torch.argsort(torch.rand(V, generator=gen, device=device)).float() + 1.0
+    wp = torch.randn(V, d_target, generator=gen, device=device) / math.sqrt(d_target - 1)
+    wp[:, 0] = -torch.log(rank)
+    wq = wp[:, :d_draft] * math.sqrt((d_target - 1) / (d_draft - 1))
+    wq[:, 0] = wp[:, 0]
+    hp = torch.randn(tree.n_nodes, d_target, generator=gen, device=device)
+    hp[:, 0] = 1.0
+    dn = torch.as_tensor(tree.draft_node, device=device, dtype=torch.long)
+    hq = hp[dn, :d_draft]
+    ids = splitmix64_stream(seed * 0x100000001 + 99, n_seq + tree.n_nodes + n_seq)
+    keys = ids[:n_seq]
+    ctx = ids[n_seq:n_seq + tree.n_nodes]
+    base_pos = (ids[n_seq + tree.n_nodes:] % np.uint64(4096)).astype(np.int64) + 16
+    seq_of_node = np.repeat(np.arange(n_seq), tree.nodes_per_seq)
+    t_key = torch.from_numpy(keys[seq_of_node].view(np.int64).copy()).to(device)
+    t_ctx = torch.from_numpy(ctx.view(np.int64).copy()).to(device)
+    t_pos = torch.from_numpy((base_pos[seq_of_node] + tree.node_depth).astype(np.uint32).view(np.int32).copy()).to(device)
+    return LmHeadWorkload(tree=tree, vocab=V, hp=hp.to(torch.bfloat16), wp=wp.to(torch.bfloat16),
+                          hq=hq.to(torch.bfloat16), wq=wq.to(torch.bfloat16), node_key=t_key, node_ctx=t_ctx,
+                          node_pos=t_pos, draft_key=t_key[dn], draft_ctx=t_ctx[dn], draft_pos=t_pos[dn],
+                          recipe=f"LM head: V={V}, d={d_target} (target) / {d_draft} (draft), hidden column 0 = 1, "
+                                 f"weight column 0 = -ln(rank), other entries Gaussian")
