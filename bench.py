@@ -276,6 +276,9 @@ def main():
     if args.workload == "hetero":
         run_hetero(args, rank, world, dev)
         return
+    if args.workload == "lmhead":
+        run_lmhead(args, rank, world, dev)
+        return
     wl = synth.make_workload(args.workload, device=dev, n_seq=args.n_seq,
                              K_sweep=args.k if args.workload == "ksweep" else None)
     t = wl.tree
@@ -835,9 +838,194 @@ def run_hetero(args, rank, world, dev):
         }))
 
 
+def _peak_tflops():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops"]), float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), "measured"
+    except Exception:
+        return 1900.0, 1700.0, "fallback"
+
+
+def run_lmhead(args, rank, world, dev):
+    """The race fused into the LM head (pps_lmhead_draft_list + pps_lmhead_verify_tree): the
+    zipf_k8 tree of B=64 sequences (K=8, gamma=5), V=128256, target hidden size 4096 (2624 node
+    rows), draft hidden size 2048 (2112 draft rows), bf16 operands whose products are Zipf-shaped
+    logits (synth.lmhead_workload).  One step = the draft GEMM + race and the target GEMM + race +
+    tree walk; no logits reach HBM.  The unfused step (pps_lmhead_logits twice, then
+    pps_draft_list and pps_verify_tree on the fp32 logits) is timed beside it."""
+    from paper_2609_21858_gb300 import pps, synth
+    n_seq = args.n_seq or 64
+    wl = synth.lmhead_workload(n_seq=n_seq, device=dev)
+    t = wl.tree
+    g = lambda x: torch.as_tensor(np.asarray(x)).to(dev).contiguous()
+    rk, so, ndr, cn = g(t.row_k), g(t.seq_off), g(t.node_draft_row), g(t.child_node)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    wsd, wsv = pps.lmhead_workspace(t.n_draft, 0, dev), pps.lmhead_workspace(t.n_nodes, t.n_seq, dev)
+    stream = torch.cuda.current_stream(dev)
+    dout = pps.lmhead_draft_list(wl.hq, wl.wq, wl.draft_key, wl.draft_ctx, wl.draft_pos, t.K, row_k=rk, ws=wsd,
+                                 status=status, keys=False, samples=False)
+    vout = pps.lmhead_verify_tree(wl.hp, wl.wp, wl.node_key, wl.node_ctx, wl.node_pos, t.gamma, so, ndr,
+                                  dout["tok"], dout["ndist"], cn, ws=wsv, status=status)
+
+    def step(hq=wl.hq, hp=wl.hp, ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        pps.lmhead_draft_list(hq, wl.wq, wl.draft_key, wl.draft_ctx, wl.draft_pos, t.K, row_k=rk, ws=wsd,
+                              status=status, out=dout, stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+        pps.lmhead_verify_tree(hp, wl.wp, wl.node_key, wl.node_ctx, wl.node_pos, t.gamma, so, ndr, dout["tok"],
+                               dout["ndist"], cn, ws=wsv, status=status, out=vout, stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    assert int(status.item()) == 0, f"status flags {int(status.item())}"
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk = Clocks(dev.index or 0)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    clk.start()
+    time.sleep(0.3)
+    e0.record(stream)
+    for k in range(args.steps):
+        step(ev=evs[k])
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = clk.stop()
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
+    t_d = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    t_v = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    V, dt_, dd_ = wl.vocab, wl.hp.shape[1], wl.hq.shape[1]
+    fl_v, fl_d = 2.0 * t.n_nodes * V * dt_, 2.0 * t.n_draft * V * dd_
+    peak, peak_sus, peak_kind = _peak_tflops()
+    # the unfused step: the same GEMMs writing fp32 logits, then the streaming race
+    lq = torch.empty(t.n_draft, V, device=dev)
+    lp = torch.empty(t.n_nodes, V, device=dev)
+    ud = pps.draft_list(lq, wl.draft_key, wl.draft_ctx, wl.draft_pos, t.K, row_k=rk)
+    uv = pps.verify_tree(lp, wl.node_key, wl.node_ctx, wl.node_pos, t.gamma, so, ndr, ud["tok"], ud["ndist"], cn)
+
+    def unfused():
+        pps.lmhead_logits(wl.hq, wl.wq, out=lq, stream=stream)
+        pps.draft_list(lq, wl.draft_key, wl.draft_ctx, wl.draft_pos, t.K, row_k=rk, out=ud, stream=stream)
+        pps.lmhead_logits(wl.hp, wl.wp, out=lp, stream=stream)
+        pps.verify_tree(lp, wl.node_key, wl.node_ctx, wl.node_pos, t.gamma, so, ndr, ud["tok"], ud["ndist"], cn,
+                        out=uv, stream=stream)
+
+    for _ in range(2):
+        unfused()
+    ms_unfused, _ = timed_replays(unfused, max(3, args.steps // 2), dev)
+    same = bool(torch.equal(uv["emitted"], vout["emitted"]) and torch.equal(ud["tok"], dout["tok"]))
+    del lq, lp
+    # end to end: the step's hidden states come from pinned host memory (the LM-head weights stay
+    # resident, as a serving engine keeps them), its emitted tokens and score sums go back
+    e2e = None
+    if args.e2e_steps > 0:
+        hq_h = torch.empty(wl.hq.shape, dtype=wl.hq.dtype, pin_memory=True)
+        hp_h = torch.empty(wl.hp.shape, dtype=wl.hp.dtype, pin_memory=True)
+        hq_h.copy_(wl.hq)
+        hp_h.copy_(wl.hp)
+        hq_d, hp_d = torch.empty_like(wl.hq), torch.empty_like(wl.hp)
+        em_h = torch.empty(vout["emitted"].shape, dtype=torch.int32, pin_memory=True)
+        ss_h = torch.empty(t.n_seq, dtype=torch.float64, pin_memory=True)
+
+        def e2e_step():
+            hq_d.copy_(hq_h, non_blocking=True)
+            hp_d.copy_(hp_h, non_blocking=True)
+            step(hq_d, hp_d)
+            em_h.copy_(vout["emitted"], non_blocking=True)
+            ss_h.copy_(vout["score_sum"], non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize(dev)
+        e_ms, _ = timed_replays(e2e_step, args.e2e_steps, dev)
+        e_ms = max_over_ranks(e_ms, world)
+        rows = t.n_nodes + t.n_draft
+        e2e = {"value": rows * world / (e_ms / 1e3), "unit": "rows/s",
+               "h2d_bytes_per_step": int((hq_h.numel() + hp_h.numel()) * 2),
+               "d2h_bytes_per_step": int(em_h.numel() * 4 + ss_h.numel() * 8), "ms_per_step": e_ms}
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = lmhead_oracle_sample(wl, args.cpu_seconds)
+    if rank == 0:
+        rows = t.n_nodes + t.n_draft
+        ach = (fl_v + fl_d) / (ms / 1e3) / 1e12
+        print(json.dumps({
+            "metric": METRIC, "value": rows * world / (ms / 1e3), "unit": "rows/s", "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded hidden states and LM-head weights with Zipf-shaped products; no model)",
+            "config": {"workload": f"lmhead: B={t.n_seq}, V={V}, K={t.K}, gamma={t.gamma}, d={dt_} target / {dd_} "
+                                   f"draft, {t.n_nodes} node rows + {t.n_draft} draft rows per step, race fused "
+                                   f"into the LM-head GEMM",
+                       "rows_per_step": rows, "l2": f"weights ({(wl.wp.numel() + wl.wq.numel()) * 2 / 1e9:.2f} GB) "
+                                                   f"larger than L2, no flush",
+                       "parallelism": f"replicas x{world}"},
+            "roofline": {"bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s", "frac": ach / peak,
+                         "traffic": None, "peak_kind": f"{peak_kind} (MEASURED_PEAKS bf16_tflops, cuBLAS burst)",
+                         "kernel": "lmhead_kernel<RaceEpi> (both launches of the step, with their finishing kernels)",
+                         "ms": ms, "flops": fl_v + fl_d, "frac_of_sustained": ach / peak_sus},
+            "launches": {"draft_ms": t_d, "draft_tflops": fl_d / (t_d / 1e3) / 1e12,
+                         "verify_ms": t_v, "verify_tflops": fl_v / (t_v / 1e3) / 1e12},
+            "unfused": {"ms_per_step": ms_unfused, "speedup_of_fusion": ms_unfused / ms,
+                        "same_outputs": same,
+                        "logits_bytes_avoided": int((t.n_nodes + t.n_draft) * V * 4 * 2)},
+            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": 4 * args.steps, "clocks": clocks,
+            "mean_accept_len": float(vout["accept_len"].float().mean().item()),
+        }))
+
+
+def lmhead_oracle_sample(wl, seconds: float):
+    """The oracle (fp64 LM head, then its race) on a bounded sample of the step's rows."""
+    import oracle
+    t = wl.tree
+    cores = oracle.set_threads(0)
+    rng = np.random.default_rng(0)
+    nr = np.sort(rng.choice(t.n_nodes, 16, replace=False))
+    dr = np.sort(rng.choice(t.n_draft, 13, replace=False))
+    hp = wl.hp[torch.as_tensor(nr, device=wl.hp.device)].float().cpu().numpy()
+    hq = wl.hq[torch.as_tensor(dr, device=wl.hq.device)].float().cpu().numpy()
+    wp, wq = wl.wp.float().cpu().numpy(), wl.wq.float().cpu().numpy()
+    from paper_2609_21858_gb300 import synth
+    ids_n = (synth.u64(wl.node_key)[nr], synth.u64(wl.node_ctx)[nr], synth.u32(wl.node_pos)[nr])
+    ids_d = (synth.u64(wl.draft_key)[dr], synth.u64(wl.draft_ctx)[dr], synth.u32(wl.draft_pos)[dr])
+
+    def run():
+        t0 = time.perf_counter()
+        lq = oracle.lmhead_logits(hq, wq).astype(np.float32)
+        oracle.draft_rows(lq, *ids_d, t.K, row_k=t.row_k[dr])
+        lp = oracle.lmhead_logits(hp, wp).astype(np.float32)
+        oracle.target_rows(lp, *ids_n)
+        return time.perf_counter() - t0
+
+    dt = run()
+    reps = max(1, int(seconds / max(dt, 1e-3)))
+    tot = sum(run() for _ in range(reps))
+    return {"value": reps * (len(nr) + len(dr)) / tot, "unit": "rows/s", "cores": cores, "kind": "oracle",
+            "sample": f"{len(dr)} draft + {len(nr)} target rows (fp64 LM head + race), x{reps} after one untimed, "
+                      f"{tot:.1f} s on {cores} threads", "cpu_model": cpu_model(), "nproc": os.cpu_count()}
+
+
 def run_reference(args, world):
     """The CPU oracle on a bounded sample per step, on this host's cores."""
     from paper_2609_21858_gb300 import synth
+    if args.workload == "lmhead":
+        wl = synth.lmhead_workload(device="cuda" if torch.cuda.is_available() else "cpu")
+        cpu = lmhead_oracle_sample(wl, 2.0 * args.steps)
+        t = wl.tree
+        print(json.dumps({
+            "impl": "reference", "metric": METRIC, "value": cpu["value"], "unit": "rows/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"lmhead: B={t.n_seq}, V={wl.vocab}, K={t.K}, gamma={t.gamma}",
+                       "parallelism": f"replicas x{world}"},
+            "cpu_baseline": cpu,
+            "e2e": {"value": cpu["value"], "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))
+        return
     wl = synth.make_workload(args.workload, device="cuda" if torch.cuda.is_available() else "cpu",
                              K_sweep=args.k if args.workload == "ksweep" else None)
     t = wl.tree
