@@ -229,3 +229,44 @@ def test_noalloc_entry_point_rejects_bad_arguments_without_a_gpu():
         assert draft(**{name: None}) == pps.ERR_INVALID_ARG, name
     assert draft(n=pps.NOALLOC_MAX_ROWS + 1) == pps.ERR_SIZE
     assert draft(n=0) == pps.OK
+
+
+def test_lmhead_entry_points_validate_arguments():
+    L = pps.lib()
+    fake = ctypes.c_void_p(256)
+    odd = ctypes.c_void_p(258)  # not 16-byte aligned
+    ids = pps.RowIds(256, 256, 256)
+    ws = int(L.pps_lmhead_workspace_size(8, 4))
+    assert ws >= 8 * 32 * 128
+
+    def logits(hidden=fake, ldh=64, weight=fake, ldw=64, n=8, V=100, d=64, out=fake, ldo=100):
+        return L.pps_lmhead_logits(hidden, ldh, weight, ldw, n, V, d, out, ldo, None)
+
+    for kw in (dict(d=0), dict(V=0), dict(n=-1), dict(ldh=32), dict(ldw=60), dict(ldh=68), dict(ldo=99),
+               dict(weight=None), dict(hidden=None), dict(out=None), dict(hidden=odd), dict(weight=odd)):
+        assert logits(**kw) == pps.ERR_INVALID_ARG, kw
+    assert logits(n=0) == pps.OK
+
+    def draft(K=4, mode=pps.DISTINCT, T=1.0, tok=fake, wsb=ws, **kw):
+        a = dict(hidden=fake, ldh=64, weight=fake, ldw=64, n=8, V=100, d=64)
+        a.update(kw)
+        return L.pps_lmhead_draft_list(a["hidden"], a["ldh"], a["weight"], a["ldw"], a["n"], a["V"], a["d"], ids, T,
+                                       K, None, mode, tok, None, fake, fake, None, None, fake, wsb, None)
+
+    assert draft(K=0) == pps.ERR_INVALID_ARG
+    assert draft(K=pps.LMHEAD_MAX_K + 1) == pps.ERR_INVALID_ARG
+    assert draft(T=0.0) == pps.ERR_INVALID_ARG
+    assert draft(mode=3) == pps.ERR_UNSUPPORTED
+    assert draft(tok=None) == pps.ERR_INVALID_ARG
+    assert draft(ldw=12) == pps.ERR_INVALID_ARG
+    assert draft(wsb=16) == pps.ERR_WORKSPACE
+    assert draft(n=0) == pps.OK
+
+    def verify(gamma=2, n_seq=2, K=2, wsb=ws, seq=fake):
+        return L.pps_lmhead_verify_tree(fake, 64, fake, 64, 8, 100, 64, ids, 1.0, n_seq, gamma, seq, fake, 4, fake,
+                                        fake, K, fake, fake, fake, fake, fake, fake, fake, fake, None, fake, wsb, None)
+
+    for kw in (dict(gamma=0), dict(gamma=65), dict(n_seq=9), dict(K=0), dict(seq=None)):
+        assert verify(**kw) == pps.ERR_INVALID_ARG, kw
+    assert verify(wsb=0) == pps.ERR_WORKSPACE
+    assert _header_defines()["PPS_LMHEAD_MAX_K"] == pps.LMHEAD_MAX_K
