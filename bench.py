@@ -552,7 +552,8 @@ def step_parity(wl, keep, dout, vout):
 
 def run_detector(args, rank, world, dev):
     """Detector pass (pps_wm_detect: Aaronson scores, per-segment sums and exact Gamma-tail
-    log p-values) over n_tokens (token, key, label, position) tuples in segments of 128: the
+    log p-values) over n_tokens (token, key, label, position) tuples in segments (texts) of
+    128 with one watermark key per text: the
     first half watermarked (race winners of fresh contexts, drawn by pps_verify_tree over
     N(0, 3^2) logits of 256 tokens), the second half uniform-random tokens (the null)."""
     from paper_2609_21858_gb300 import pps
@@ -560,7 +561,8 @@ def run_detector(args, rank, world, dev):
     half = n // 2
     g = torch.Generator(device=dev)
     g.manual_seed(4)
-    key = torch.randint(-2 ** 62, 2 ** 62, (n,), generator=g, device=dev, dtype=torch.int64)
+    # one watermark key per text (segment of 128 tokens); labels and positions per token
+    key = torch.randint(-2 ** 62, 2 ** 62, (n // 128,), generator=g, device=dev, dtype=torch.int64).repeat_interleave(128)
     ctx = torch.randint(-2 ** 62, 2 ** 62, (n,), generator=g, device=dev, dtype=torch.int64)
     pos = torch.randint(0, 2 ** 30, (n,), generator=g, device=dev, dtype=torch.int32)
     tok = torch.randint(0, 128256, (n,), generator=g, device=dev, dtype=torch.int32)

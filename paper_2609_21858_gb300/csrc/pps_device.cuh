@@ -86,6 +86,14 @@ __device__ __forceinline__ uint32_t word_of(uint64_t key, uint64_t ctx, uint32_t
     return lane_of(b, (uint32_t)(i & 3));
 }
 
+// word of token i (first arrival) under a key (k0, k1) that every lane of the
+// warp holds: callers pass values known warp-uniform (e.g. from
+// __reduce_or_sync), so the compiler keeps the key schedule in uniform registers
+__device__ __forceinline__ uint32_t word_of_ukey(uint32_t k0, uint32_t k1, uint64_t ctx, uint32_t pos, int64_t i) {
+    const uint4 b = philox((uint32_t)((uint64_t)i >> 2), pos, (uint32_t)ctx, (uint32_t)(ctx >> 32), k0, k1);
+    return lane_of(b, (uint32_t)(i & 3));
+}
+
 // Row-specialised Philox for the streaming loop (first arrival, fixed row).
 // Only counter word 0 (token >> 2) varies along a row, so the products of
 // the constant words in rounds 1-2 are hoisted per row: round 1 needs one
@@ -172,16 +180,17 @@ __device__ __forceinline__ float lg2_approx(float x) {
     asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
+// The first two cases are the same expression, so both values are formed and
+// one is selected (no divergent branch inside a warp).
 __device__ __forceinline__ float neg_log2_u(uint32_t w) {
-    if (w < 0x80000000u) return -lg2_approx(fmaf((float)w, 0x1p-32f, 0x1p-33f));
+    const float y = -lg2_approx(fmaf((float)w, 0x1p-32f, 0x1p-33f));
     const float v = fmaf((float)(~w), 0x1p-32f, 0x1p-33f);
-    if (v >= 0.0625f) return -lg2_approx(fmaf((float)w, 0x1p-32f, 0x1p-33f));
     float p = fmaf(v, 1.0f / 6.0f, 0.2f);
     p = fmaf(v, p, 0.25f);
     p = fmaf(v, p, 1.0f / 3.0f);
     p = fmaf(v, p, 0.5f);
     p = fmaf(v, p, 1.0f);
-    return v * kLog2e * p;
+    return (w >= 0x80000000u && v < 0.0625f) ? v * kLog2e * p : y;
 }
 
 // x = log2(-log2 u), the word part of the fp32 key

@@ -9,13 +9,16 @@ namespace pps {
 
 #define FULL 0xffffffffu
 
-// Detector (App. E): every warp takes a contiguous chunk of tokens; lane t of
-// an iteration scores token base + t, and a warp loads and scores the tokens
-// of kScoreAhead iterations (a group of 128) together.  Segment sums: when a
+// Detector (App. E): every warp takes a contiguous chunk of tokens and works
+// through it a group of 128 at a time; lane l loads and scores tokens
+// 4l .. 4l+3 of the group (16-byte loads when the arrays are aligned).  When
+// the whole group has one key (the tokens of one text), the Philox key
+// schedule is warp-uniform and kept in uniform registers.  Segment sums: when a
 // group lies inside the open segment (segments of a text are usually longer
 // than a group), each lane adds its four scores and one warp reduction adds
 // the group to the segment's running sum; a group that holds a segment
-// boundary takes a segmented warp scan per iteration.  The running sum is a
+// boundary is rearranged to lane-major order (shuffles) and takes a segmented
+// warp scan per 32 tokens.  The running sum is a
 // float-float pair (an exact fp32 two-sum per addition, FP64 being slow on this
 // part) and goes to the segment's fp64 slot with one atomic per segment end the
 // warp sees (plus one at the end of its chunk).
@@ -30,6 +33,7 @@ __device__ __forceinline__ void ff_add(float& hi, float& lo, float v) {
     hi = s;
 }
 
+template <bool VEC>
 __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict__ tokens,
                                                        const uint64_t* __restrict__ key,
                                                        const uint64_t* __restrict__ ctx,
@@ -61,40 +65,62 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
         seg_end = seg + 1 < n_seg ? seg_off[seg + 1] : LLONG_MAX;
     }
     float chi = 0.0f, clo = 0.0f;  // running sum of the open segment
-    // per-lane input pointers, advanced a group at a time (constant offsets inside a group)
     constexpr int G = 32 * kScoreAhead;
-    const int32_t* tp = tokens + c0 + lane;
-    const uint64_t* kp = key + c0 + lane;
-    const uint64_t* xp = ctx + c0 + lane;
-    const uint32_t* pp = pos + c0 + lane;
+    static_assert(kScoreAhead == 4, "a lane holds four consecutive tuples of a group");
     for (int64_t grp = c0; grp < c1; grp += G) {
-        // the group's inputs first, more loads in flight per warp (lim: the group's tokens from
-        // this lane's first one on)
-        const int lim = (int)min((int64_t)G, c1 - grp) - lane;
-        int32_t tk[kScoreAhead];
-        uint64_t kk[kScoreAhead], cx[kScoreAhead];
-        uint32_t ps[kScoreAhead];
+        // lane l holds tuples grp + 4 l .. grp + 4 l + 3 (the first nloc of them exist), loaded
+        // with 16-byte loads when the arrays allow it
+        const int64_t t0 = grp + 4 * lane;
+        const int nloc = (int)max((int64_t)0, min((int64_t)4, c1 - t0));
+        int32_t tk[4] = {0, 0, 0, 0};
+        uint64_t kk[4] = {0, 0, 0, 0}, cx[4] = {0, 0, 0, 0};
+        uint32_t ps[4] = {0, 0, 0, 0};
+        if (VEC && nloc == 4) {
+            const int4 t4 = __ldg(reinterpret_cast<const int4*>(tokens + t0));
+            const uint4 p4 = __ldg(reinterpret_cast<const uint4*>(pos + t0));
+            const ulonglong2 ka = __ldg(reinterpret_cast<const ulonglong2*>(key + t0));
+            const ulonglong2 kb = __ldg(reinterpret_cast<const ulonglong2*>(key + t0 + 2));
+            const ulonglong2 xa = __ldg(reinterpret_cast<const ulonglong2*>(ctx + t0));
+            const ulonglong2 xb = __ldg(reinterpret_cast<const ulonglong2*>(ctx + t0 + 2));
+            tk[0] = t4.x; tk[1] = t4.y; tk[2] = t4.z; tk[3] = t4.w;
+            ps[0] = p4.x; ps[1] = p4.y; ps[2] = p4.z; ps[3] = p4.w;
+            kk[0] = ka.x; kk[1] = ka.y; kk[2] = kb.x; kk[3] = kb.y;
+            cx[0] = xa.x; cx[1] = xa.y; cx[2] = xb.x; cx[3] = xb.y;
+        } else {
 #pragma unroll
-        for (int u = 0; u < kScoreAhead; ++u) {
-            if (32 * u < lim) {
-                tk[u] = tp[32 * u];
-                kk[u] = kp[32 * u];
-                cx[u] = xp[32 * u];
-                ps[u] = pp[32 * u];
+            for (int u = 0; u < 4; ++u)
+                if (u < nloc) {
+                    tk[u] = tokens[t0 + u];
+                    ps[u] = pos[t0 + u];
+                    kk[u] = key[t0 + u];
+                    cx[u] = ctx[t0 + u];
+                }
+        }
+        // one key for the whole group (the tokens of one text): its schedule in uniform registers
+        bool same = true;
+#pragma unroll
+        for (int u = 1; u < 4; ++u) same &= u >= nloc || kk[u] == kk[0];
+        const uint64_t k_any = nloc > 0 ? kk[0] : 0ull;
+        const uint32_t klo = __reduce_or_sync(FULL, (uint32_t)k_any), khi = __reduce_or_sync(FULL, (uint32_t)(k_any >> 32));
+        same &= nloc == 0 || k_any == (((uint64_t)khi << 32) | klo);
+        const bool ukey = __all_sync(FULL, same);
+        float A[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            A[u] = 0.0f;
+            if (u < nloc) {
+                const uint32_t w = ukey ? word_of_ukey(klo, khi, cx[u], ps[u], (int64_t)tk[u])
+                                        : word_of(kk[u], cx[u], ps[u], (int64_t)tk[u], 1);
+                A[u] = score_kind32(w, P);
             }
         }
-        tp += G;
-        kp += G;
-        xp += G;
-        pp += G;
-        float A[kScoreAhead];
+        if (out_score) {
+            if (VEC && nloc == 4)
+                *reinterpret_cast<float4*>(out_score + t0) = make_float4(A[0], A[1], A[2], A[3]);
+            else
 #pragma unroll
-        for (int u = 0; u < kScoreAhead; ++u) {
-            A[u] = 0.0f;
-            if (32 * u < lim) {
-                A[u] = score_kind32(word_of(kk[u], cx[u], ps[u], (int64_t)tk[u], 1), P);
-                if (out_score) out_score[grp + 32 * u + lane] = A[u];
-            }
+                for (int u = 0; u < 4; ++u)
+                    if (u < nloc) out_score[t0 + u] = A[u];
         }
         if (!out_sum) continue;
         const int64_t gend = min(grp + 32 * kScoreAhead, c1);
@@ -117,7 +143,17 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
             ff_add(chi, clo, v);
             continue;
         }
-        // a segment boundary inside the group: a segmented scan per iteration
+        // a segment boundary inside the group: a segmented scan per iteration, over the
+        // lane-major layout (iteration u, lane t: tuple grp + 32 u + t, held by lane 8 u + t / 4)
+        float Am[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int src = 8 * u + (lane >> 2);
+            const float a0 = __shfl_sync(FULL, A[0], src), a1 = __shfl_sync(FULL, A[1], src);
+            const float a2 = __shfl_sync(FULL, A[2], src), a3 = __shfl_sync(FULL, A[3], src);
+            const int e = lane & 3;
+            Am[u] = e == 0 ? a0 : e == 1 ? a1 : e == 2 ? a2 : a3;
+        }
 #pragma unroll
         for (int u = 0; u < kScoreAhead; ++u) {
             const int64_t base = grp + 32 * u;
@@ -130,7 +166,7 @@ __global__ void __launch_bounds__(256) wm_score_kernel(const int32_t* __restrict
                 while (my + 1 < n_seg && seg_off[my + 1] <= t) ++my;
             }
             // segmented inclusive scan over the lanes of each segment run
-            float v = A[u];
+            float v = Am[u];
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
                 const float ov = __shfl_up_sync(FULL, v, o);
@@ -578,13 +614,20 @@ cudaError_t launch_wm_score(const int32_t* tokens, const uint64_t* key, const ui
         // one wave: as many warps as the GPU holds at once, each a contiguous chunk
         // (a multiple of the 128 tokens of one load group)
         const int64_t resident =
-            (int64_t)device_sm_count() * resident_ctas(kOccScore, (const void*)wm_score_kernel, 256) * (256 / 32);
+            (int64_t)device_sm_count() * resident_ctas(kOccScore, (const void*)wm_score_kernel<true>, 256) * (256 / 32);
         const int64_t group = 32 * kScoreAhead;
         const int64_t chunk = ((n + resident - 1) / resident + group - 1) / group * group;
         const int64_t warps = (n + chunk - 1) / chunk;
         const int64_t blocks = (warps * 32 + 255) / 256;
-        wm_score_kernel<<<(unsigned)blocks, 256, 0, stream>>>(tokens, key, ctx, pos, n, n_seg, seg_off, P, out_score,
-                                                              out_sum, chunk);
+        // 16-byte loads and stores need 16-byte aligned arrays (chunks start on multiples of 128 tuples)
+        auto al = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+        const bool vec = al(tokens) && al(key) && al(ctx) && al(pos) && (out_score == nullptr || al(out_score));
+        if (vec)
+            wm_score_kernel<true><<<(unsigned)blocks, 256, 0, stream>>>(tokens, key, ctx, pos, n, n_seg, seg_off, P,
+                                                                        out_score, out_sum, chunk);
+        else
+            wm_score_kernel<false><<<(unsigned)blocks, 256, 0, stream>>>(tokens, key, ctx, pos, n, n_seg, seg_off, P,
+                                                                         out_score, out_sum, chunk);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }

@@ -111,3 +111,31 @@ def test_gamma_and_chernoff_for_one_segment_of_m_tokens(M):
     want = oracle.gamma_tail_logp(M, float(sa.item()))
     assert abs(la.item() - want) <= logp_tol_gamma(M, float(sa.item()), want)
     _check_chernoff(lu.item(), M, float(su.item()))
+
+
+@pytest.mark.parametrize("kind,param", [(pps.SCORE_AARONSON, 0.0), (pps.SCORE_U, 0.0), (pps.SCORE_LI, 0.5)])
+def test_one_key_per_text(kind, param):
+    # the tokens of one text share the watermark key: groups of 128 tuples with one key take the
+    # kernel's uniform-key path; texts of 128 and 300 tokens (boundaries inside groups too), a
+    # ragged tail, and a view whose arrays are not 16-byte aligned (scalar loads)
+    n = 40000 + 37
+    tok, _, ctx, pos = _tuples(n, 90 + kind)
+    rng = np.random.default_rng(91)
+    lens = np.where(np.arange(n // 128 + 2) % 3 == 0, 300, 128)
+    seg = np.concatenate([[0], np.cumsum(lens)])
+    seg = seg[seg < n]
+    seg = np.concatenate([seg, [n]]).astype(np.int64)
+    text_key = rng.integers(0, 2 ** 64, len(seg) - 1, dtype=np.uint64)
+    key = np.repeat(text_key, np.diff(seg))
+    tg = torch.as_tensor(tok).cuda()
+    kg, cg, pg = dev_ids(key, ctx, pos)
+    for off in (0, 1):
+        # off = 1: views one element in, so no array starts on a 16-byte boundary
+        t, kk, cc, pp = tok[off:], key[off:], ctx[off:], pos[off:]
+        sg = np.maximum(seg - off, 0)
+        sg[0] = 0
+        sc, sums, _ = pps.wm_detect(tg[off:], kg[off:], cg[off:], pg[off:], torch.as_tensor(sg).cuda(), kind, param)
+        torch.cuda.synchronize()
+        osc, osums, _ = oracle.wm_detect(t, kk, cc, pp, sg, kind, param)
+        np.testing.assert_allclose(sc.cpu().numpy(), osc, rtol=2e-5, atol=2e-6 * max(1.0, np.abs(osc).max()))
+        np.testing.assert_allclose(sums.cpu().numpy(), osums, rtol=2e-5, atol=1e-4)
