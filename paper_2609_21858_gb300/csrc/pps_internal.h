@@ -84,6 +84,30 @@ struct RaceArgs {
     uint32_t* seq_cnt;   // [n_seq]
 };
 
+// Programmatic dependent launch.  A kernel launched with launch_pdl may start
+// while the previous kernel on its stream drains; it calls pdl_wait() before it
+// reads anything a previous kernel wrote (the wait returns once that kernel has
+// completed and its memory is visible; without the attribute it is a no-op) and
+// pdl_launch_dependents() to let the next kernel start launching in turn.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... Args, typename... Act>
+inline cudaError_t launch_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                              Act&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Act&&>(args)...);
+}
+
 size_t workspace_bytes(int64_t n_rows, int32_t n_seq);
 void workspace_carve(void* ws, int64_t n_rows, int32_t n_seq, Partial** partials, uint32_t** row_cnt,
                      uint32_t** seq_cnt);

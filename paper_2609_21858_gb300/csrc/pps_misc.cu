@@ -402,6 +402,8 @@ __global__ void tree_expand_kernel(int32_t n_seq, int32_t K, int32_t gamma, int3
                                    const int32_t* __restrict__ row_k, uint64_t* next_key, uint64_t* next_ctx,
                                    uint32_t* next_pos, int32_t* next_k, int32_t* child_node, uint64_t* node_key,
                                    uint64_t* node_ctx, uint32_t* node_pos) {
+    pdl_wait();  // the lists and row ids of the previous launch
+    pdl_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int64_t b = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (b >= n_seq) return;
@@ -463,6 +465,8 @@ __global__ void hetero_expand_kernel(int32_t n_seq, int32_t B, int32_t gamma, in
                                      uint32_t* next_pos, int32_t* next_owner, int32_t* list_tok, int32_t* list_nd,
                                      int32_t* child_node, uint64_t* node_key, uint64_t* node_ctx,
                                      uint32_t* node_pos) {
+    pdl_wait();  // the lists and row ids of the previous launch
+    pdl_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int64_t s = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (s >= n_seq) return;
@@ -645,10 +649,10 @@ cudaError_t launch_tree_expand(int32_t n_seq, int32_t K, int32_t gamma, int32_t 
                                uint64_t* node_ctx, uint32_t* node_pos, cudaStream_t stream) {
     if (n_seq == 0) return cudaSuccess;
     const int64_t blocks = ((int64_t)n_seq * 32 + 255) / 256;
-    tree_expand_kernel<<<(unsigned)blocks, 256, 0, stream>>>(n_seq, K, gamma, depth, tok, mult, ndist, key, ctx, pos,
-                                                              row_k, next_key, next_ctx, next_pos, next_k, child_node,
-                                                              node_key, node_ctx, node_pos);
-    return cudaGetLastError();
+    const cudaError_t e = launch_pdl(tree_expand_kernel, dim3((unsigned)blocks), dim3(256), 0, stream, n_seq, K, gamma,
+                                     depth, tok, mult, ndist, key, ctx, pos, row_k, next_key, next_ctx, next_pos,
+                                     next_k, child_node, node_key, node_ctx, node_pos);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_hetero_expand(int32_t n_seq, int32_t B, int32_t gamma, int32_t depth, const int32_t* tok,
@@ -658,10 +662,10 @@ cudaError_t launch_hetero_expand(int32_t n_seq, int32_t B, int32_t gamma, int32_
                                  uint64_t* node_ctx, uint32_t* node_pos, cudaStream_t stream) {
     if (n_seq == 0) return cudaSuccess;
     const int64_t blocks = ((int64_t)n_seq * 32 + 255) / 256;
-    hetero_expand_kernel<<<(unsigned)blocks, 256, 0, stream>>>(n_seq, B, gamma, depth, tok, key, ctx, pos, owner,
-                                                                next_key, next_ctx, next_pos, next_owner, list_tok,
-                                                                list_nd, child_node, node_key, node_ctx, node_pos);
-    return cudaGetLastError();
+    const cudaError_t e = launch_pdl(hetero_expand_kernel, dim3((unsigned)blocks), dim3(256), 0, stream, n_seq, B,
+                                     gamma, depth, tok, key, ctx, pos, owner, next_key, next_ctx, next_pos, next_owner,
+                                     list_tok, list_nd, child_node, node_key, node_ctx, node_pos);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_hetero_block(int64_t n, int32_t B, const int32_t* tok, const uint64_t* key, const uint64_t* ctx,

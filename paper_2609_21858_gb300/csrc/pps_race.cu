@@ -59,6 +59,9 @@
 #ifndef PPS_BLOCK_MIN_BLOCKS
 #define PPS_BLOCK_MIN_BLOCKS 12  // the same for proposal rows of the augmented race (16 spills)
 #endif
+#ifndef PPS_VF_MAXK
+#define PPS_VF_MAXK 4  // draft rows with lists up to this long stream like verify rows (one test per vector)
+#endif
 #ifndef PPS_SEG_CAP
 #define PPS_SEG_CAP 30  // at most this many warp segments per row (small launches; keeps <= 32 partial lists)
 #endif
@@ -1400,6 +1403,8 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
     __shared__ uint32_t s_queue[kQueueCap];
     __shared__ float s_mk[32 * 32];  // staging of the partial lists merged by merge_rounds
     __shared__ int s_mi[32 * 32];
+    pdl_wait();  // the previous kernel's outputs (row ids, lists) and the workspace it used
+    pdl_launch_dependents();
     const int64_t NW = a.G;
     const int64_t gw = blockIdx.x;
     const int64_t g0 = gw * a.total / NW, g1 = (gw + 1) * a.total / NW;
@@ -1426,10 +1431,11 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
         }
         WarpList L;
         L.reset(kp, kr);
-        // A one-token draft list is a target race: such rows stream like verify rows (one filter
-        // test per vector).  A row cut between warps shares its filter bound (verify, one-token
-        // draft and proposal rows: on K-list draft rows the shared bound saves too little).
-        const bool one = VERIFY || (!BLK && kr == 1);
+        // A one-token draft list is a target race, and a list of a few tokens is close to one:
+        // such rows stream like verify rows (one filter test per vector; measured: lists of up
+        // to 4 gain, lists of 8 lose).  A row cut between warps shares its filter bound (verify,
+        // short-list draft and proposal rows: on longer lists the shared bound saves too little).
+        const bool one = VERIFY || (!BLK && kr <= PPS_VF_MAXK);
         uint32_t* slot = nullptr;
         if constexpr (PPS_ROWBOUND)
             if ((one || BLK) && a.row_bound && (v0 > 0 || v1 < nv)) slot = a.row_bound + r;
@@ -1475,31 +1481,32 @@ int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk, int64_t
 
 cudaError_t launch_race(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream) {
     dim3 grid(a.G), block(kThreads);
+    cudaError_t e = cudaSuccess;
     const bool blk = !verify && a.row_block != nullptr;
     if (dtype == 1) {
         if (verify) {
-            if (vec) race_kernel<1, true, true, false><<<grid, block, 0, stream>>>(a);
-            else race_kernel<1, true, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(race_kernel<1, true, true, false>, grid, block, 0, stream, a);
+            else e = launch_pdl(race_kernel<1, true, false, false>, grid, block, 0, stream, a);
         } else if (blk) {
-            if (vec) race_kernel<1, false, true, true><<<grid, block, 0, stream>>>(a);
-            else race_kernel<1, false, false, true><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(race_kernel<1, false, true, true>, grid, block, 0, stream, a);
+            else e = launch_pdl(race_kernel<1, false, false, true>, grid, block, 0, stream, a);
         } else {
-            if (vec) race_kernel<1, false, true, false><<<grid, block, 0, stream>>>(a);
-            else race_kernel<1, false, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(race_kernel<1, false, true, false>, grid, block, 0, stream, a);
+            else e = launch_pdl(race_kernel<1, false, false, false>, grid, block, 0, stream, a);
         }
     } else {
         if (verify) {
-            if (vec) race_kernel<0, true, true, false><<<grid, block, 0, stream>>>(a);
-            else race_kernel<0, true, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(race_kernel<0, true, true, false>, grid, block, 0, stream, a);
+            else e = launch_pdl(race_kernel<0, true, false, false>, grid, block, 0, stream, a);
         } else if (blk) {
-            if (vec) race_kernel<0, false, true, true><<<grid, block, 0, stream>>>(a);
-            else race_kernel<0, false, false, true><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(race_kernel<0, false, true, true>, grid, block, 0, stream, a);
+            else e = launch_pdl(race_kernel<0, false, false, true>, grid, block, 0, stream, a);
         } else {
-            if (vec) race_kernel<0, false, true, false><<<grid, block, 0, stream>>>(a);
-            else race_kernel<0, false, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(race_kernel<0, false, true, false>, grid, block, 0, stream, a);
+            else e = launch_pdl(race_kernel<0, false, false, false>, grid, block, 0, stream, a);
         }
     }
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 // Rows stay whole where the grid allows (a segment's candidate count grows
@@ -1532,31 +1539,32 @@ int trunc_grid(int64_t total, int64_t n_rows, int dtype, bool verify, bool vec, 
 
 cudaError_t launch_trunc(const RaceArgs& a, int dtype, bool verify, bool vec, cudaStream_t stream) {
     dim3 grid(a.G), block(kThreads);
+    cudaError_t e = cudaSuccess;
     const bool blk = !verify && a.row_block != nullptr;
     if (dtype == 1) {
         if (verify) {
-            if (vec) trunc_kernel<1, true, true, false><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<1, true, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(trunc_kernel<1, true, true, false>, grid, block, 0, stream, a);
+            else e = launch_pdl(trunc_kernel<1, true, false, false>, grid, block, 0, stream, a);
         } else if (blk) {
-            if (vec) trunc_kernel<1, false, true, true><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<1, false, false, true><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(trunc_kernel<1, false, true, true>, grid, block, 0, stream, a);
+            else e = launch_pdl(trunc_kernel<1, false, false, true>, grid, block, 0, stream, a);
         } else {
-            if (vec) trunc_kernel<1, false, true, false><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<1, false, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(trunc_kernel<1, false, true, false>, grid, block, 0, stream, a);
+            else e = launch_pdl(trunc_kernel<1, false, false, false>, grid, block, 0, stream, a);
         }
     } else {
         if (verify) {
-            if (vec) trunc_kernel<0, true, true, false><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<0, true, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(trunc_kernel<0, true, true, false>, grid, block, 0, stream, a);
+            else e = launch_pdl(trunc_kernel<0, true, false, false>, grid, block, 0, stream, a);
         } else if (blk) {
-            if (vec) trunc_kernel<0, false, true, true><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<0, false, false, true><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(trunc_kernel<0, false, true, true>, grid, block, 0, stream, a);
+            else e = launch_pdl(trunc_kernel<0, false, false, true>, grid, block, 0, stream, a);
         } else {
-            if (vec) trunc_kernel<0, false, true, false><<<grid, block, 0, stream>>>(a);
-            else trunc_kernel<0, false, false, false><<<grid, block, 0, stream>>>(a);
+            if (vec) e = launch_pdl(trunc_kernel<0, false, true, false>, grid, block, 0, stream, a);
+            else e = launch_pdl(trunc_kernel<0, false, false, false>, grid, block, 0, stream, a);
         }
     }
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace pps

@@ -801,6 +801,8 @@ __global__ void __launch_bounds__(kThreads, PPS_TRUNC_MIN_BLOCKS) trunc_kernel(c
     __shared__ int s_ci[kCandCap];
     __shared__ uint4 s_qv[kTQueueCap];
     __shared__ uint32_t s_qi[kTQueueCap];
+    pdl_wait();  // the previous kernel's outputs and the workspace it used
+    pdl_launch_dependents();
     const int64_t NW = a.G;
     const int64_t gw = blockIdx.x;
     const int64_t g0 = gw * a.total / NW, g1 = (gw + 1) * a.total / NW;
