@@ -772,7 +772,61 @@ __device__ __forceinline__ void emit_row(const RaceArgs& a, int64_t r, double dk
     int tok = mine ? li : -1;
     int mult = mine ? 1 : 0;
     int sample = tok;
-    if (a.iid) {
+    if (a.iid && kr <= 8) {
+        // The same samples with the kr x kr candidates laid out at once: arrival j = e + 1 of
+        // token t (its t-th list entry) sits in lane 8 (t mod 4) + e of slot t / 4.  Each lane
+        // forms its arrival time, the 8-lane group its cumulative sums in arrival order (a
+        // chain of shuffles, so G_{t,j} is summed exactly as the one-at-a-time version sums
+        // it) and its scores; kr rounds of a warp argmin over (score, token, arrival) then
+        // give the samples.  A token's later arrivals order after its earlier ones, so the
+        // global kr smallest are the samples the one-at-a-time version finds.
+        mult = 0;
+        sample = -1;
+        double h2[2];
+        int t2[2], j2[2];
+#pragma unroll
+        for (int sl = 0; sl < 2; ++sl) {
+            const int t = 4 * sl + (lane >> 3), e = lane & 7;
+            const int tt = __shfl_sync(FULL, li, t);
+            const bool valid = t < nuse && e < kr;
+            const double E = valid ? exp1_f64(word_of(key, ctx, pos, tt, e + 1)) : 0.0;
+            double G = E;
+#pragma unroll
+            for (int st = 1; st < 8; ++st) {
+                const double prev = __shfl_up_sync(FULL, G, 1);
+                if (e == st) G = prev + E;
+            }
+            const double ld = valid ? (double)lp(tt) : 0.0;
+            h2[sl] = valid ? log(G) - ld / (double)a.T : (double)INFINITY;
+            t2[sl] = valid ? tt : INT_MAX;
+            j2[sl] = e + 1;
+        }
+        for (int m = 0; m < kr; ++m) {
+            const int ls = (h2[1] < h2[0] || (h2[1] == h2[0] && (t2[1] < t2[0] || (t2[1] == t2[0] && j2[1] < j2[0])))) ? 1 : 0;
+            double bh = ls ? h2[1] : h2[0];
+            int bt = ls ? t2[1] : t2[0], bj = ls ? j2[1] : j2[0], bo = 2 * lane + ls;
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+                const double oh = __shfl_xor_sync(FULL, bh, off);
+                const int ot = __shfl_xor_sync(FULL, bt, off);
+                const int oj = __shfl_xor_sync(FULL, bj, off);
+                const int oo = __shfl_xor_sync(FULL, bo, off);
+                if (oh < bh || (oh == bh && (ot < bt || (ot == bt && oj < bj)))) {
+                    bh = oh;
+                    bt = ot;
+                    bj = oj;
+                    bo = oo;
+                }
+            }
+            if (bt == INT_MAX) break;  // fewer usable tokens than samples
+            if (lane == m) sample = bt;
+            if (mine && tok == bt) ++mult;
+            if ((bo >> 1) == lane) {
+                if (bo & 1) h2[1] = (double)INFINITY, t2[1] = INT_MAX;
+                else h2[0] = (double)INFINITY, t2[0] = INT_MAX;
+            }
+        }
+    } else if (a.iid) {
         // multi-arrival scores ln(G_{t,j}) - l_t/T of the nuse tokens, j = 1..kr;
         // the kr smallest (ties by token, then arrival) are the samples
         mult = 0;
