@@ -14,7 +14,7 @@ CSRC = os.path.join(PKG, "csrc")
 OUT = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT, "libpps.so")
 SOURCES = ["pps_race.cu", "pps_misc.cu", "pps_api.cu"]
-HEADERS = ["pps_device.cuh", "pps_internal.h", "pps_trunc.cuh"]
+HEADERS = ["pps_device.cuh", "pps_internal.h", "pps_trunc.cuh", "pps_lmhead.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
