@@ -90,6 +90,26 @@ __device__ __forceinline__ bool lex_less_d(double ak, int ai, double bk, int bi)
     return ak < bk || (ak == bk && ai < bi);
 }
 
+// fp32 key -> unsigned integer with the same order (-0 taken as +0), and back,
+// so that a warp argmin of (key, token) is two redux.min instructions.
+__device__ __forceinline__ uint32_t ord_key(float f) {
+    const uint32_t b = __float_as_uint(f + 0.0f);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float unord_key(uint32_t u) {
+    return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
+}
+// Warp argmin of (key, token) by lexicographic order; tokens are non-negative
+// (INT_MAX: empty).  Returns the winning token (INT_MAX when every lane is
+// empty) and its key in bk.
+__device__ __forceinline__ int warp_argmin(float k, int t, float& bk) {
+    const uint32_t u = ord_key(k);
+    const uint32_t mu = __reduce_min_sync(FULL, u);
+    const uint32_t mt = __reduce_min_sync(FULL, u == mu ? (uint32_t)t : 0xffffffffu);
+    bk = unord_key(mu);
+    return (int)mt;
+}
+
 // ---------------------------------------------------------------- warp lists
 // A warp list holds entries (k, i) sorted ascending by (k, i), entry m in
 // lane m; lanes >= kp hold (+inf, INT_MAX).
@@ -902,29 +922,17 @@ __device__ __noinline__ bool iid_fast(const RaceArgs& a, int64_t r, float lk, in
     int j = 1, mult = 0, sample = -1, nsel = 0;
     float selh = kInf;
     for (int m = 0; m < kr; ++m) {
-        // warp argmin of (h, tok, j)
-        float bh = h;
-        int bt = mine ? tok : INT_MAX, bj = j, bl = lane;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) {
-            const float oh = __shfl_xor_sync(FULL, bh, off);
-            const int ot = __shfl_xor_sync(FULL, bt, off);
-            const int oj = __shfl_xor_sync(FULL, bj, off);
-            const int ol = __shfl_xor_sync(FULL, bl, off);
-            if (oh < bh || (oh == bh && (ot < bt || (ot == bt && oj < bj)))) {
-                bh = oh;
-                bt = ot;
-                bj = oj;
-                bl = ol;
-            }
-        }
+        // warp argmin of (h, tok): each lane holds a distinct token, so the
+        // winner's lane is the one holding bt
+        float bh;
+        const int bt = warp_argmin(h, mine ? tok : INT_MAX, bh);
         if (bt == INT_MAX) break;  // fewer usable tokens than samples
         if (lane == m) {
             sample = bt;
             selh = bh;
         }
         ++nsel;
-        if (lane == bl) {
+        if (mine && tok == bt) {
             ++mult;
             ++j;
             if (j <= kr) {
@@ -1334,13 +1342,21 @@ __device__ __forceinline__ void merge_partials(const RaceArgs& a, int64_t r, int
 }
 
 // Merge by selection rounds, for at most 32 partial lists: list j is staged in
-// column j of s_k / s_i (entry e at [e * 32 + j], e < kp; one 16-byte load
-// per four entries, all lanes at once), lane j holds the head of list j, and
-// each of kp rounds moves the warp's smallest head (key, token) to entry m of
-// the merged list and advances its lane.  One warp argmin per output entry
-// replaces one dependent bitonic merge per list.  Tokens are unique across the
-// lists (disjoint segments of one row), so only the owner's head matches the
+// row j of s_k / s_i (entry e at [j * 32 + e], e < kp) by asynchronous 16-byte
+// copies that every lane issues for its whole list before one wait (one L2
+// round trip for the lot), lane j holds the head of list j, and each of kp
+// rounds moves the warp's smallest head (key, token) to entry m of the merged
+// list and advances its lane.  One warp argmin per output entry replaces one
+// dependent bitonic merge per list.  Tokens are unique across the lists
+// (disjoint segments of one row), so only the owner's head matches the
 // winner.  The smallest head left over is the smallest listed key dropped.
+// s_k and s_i are 16-byte aligned.
+__device__ __forceinline__ void copy16_async(void* smem, const void* gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
+                 "l"(gmem)
+                 : "memory");
+}
+
 __device__ __noinline__ void merge_rounds(const RaceArgs& a, int64_t r, int64_t first_w, int P, int kp, int lane,
                                           float* s_k, int* s_i, float& lk, int& li, float& theta_drop) {
     float th = kInf;
@@ -1348,36 +1364,20 @@ __device__ __noinline__ void merge_rounds(const RaceArgs& a, int64_t r, int64_t 
         const Partial* Q = a.partials + (first_w + lane + r);
         th = __ldcg(&Q->theta_drop);
         for (int e = 0; e < kp; e += 4) {
-            const float4 k4 = __ldcg(reinterpret_cast<const float4*>(Q->key + e));
-            const int4 i4 = __ldcg(reinterpret_cast<const int4*>(Q->idx + e));
-            s_k[(e + 0) * 32 + lane] = k4.x;
-            s_k[(e + 1) * 32 + lane] = k4.y;
-            s_k[(e + 2) * 32 + lane] = k4.z;
-            s_k[(e + 3) * 32 + lane] = k4.w;
-            s_i[(e + 0) * 32 + lane] = i4.x;
-            s_i[(e + 1) * 32 + lane] = i4.y;
-            s_i[(e + 2) * 32 + lane] = i4.z;
-            s_i[(e + 3) * 32 + lane] = i4.w;
+            copy16_async(s_k + lane * 32 + e, Q->key + e);
+            copy16_async(s_i + lane * 32 + e, Q->idx + e);
         }
     }
+    asm volatile("cp.async.wait_all;" ::: "memory");
     __syncwarp();
     int h = 0;
-    float hk = lane < P ? s_k[lane] : kInf;
-    int hi = lane < P ? s_i[lane] : INT_MAX;
+    float hk = lane < P ? s_k[lane * 32] : kInf;
+    int hi = lane < P ? s_i[lane * 32] : INT_MAX;
     lk = kInf;
     li = INT_MAX;
     for (int m = 0; m < kp; ++m) {
-        float bk = hk;
-        int bi = hi;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float ok = __shfl_xor_sync(FULL, bk, o);
-            const int oi = __shfl_xor_sync(FULL, bi, o);
-            if (lex_less(ok, oi, bk, bi)) {
-                bk = ok;
-                bi = oi;
-            }
-        }
+        float bk;
+        const int bi = warp_argmin(hk, hi, bk);
         if (bi == INT_MAX) break;  // fewer listed entries than kp (warp-uniform)
         if (lane == m) {
             lk = bk;
@@ -1385,8 +1385,8 @@ __device__ __noinline__ void merge_rounds(const RaceArgs& a, int64_t r, int64_t 
         }
         if (hi == bi) {
             ++h;
-            hk = h < kp ? s_k[h * 32 + lane] : kInf;
-            hi = h < kp ? s_i[h * 32 + lane] : INT_MAX;
+            hk = h < kp ? s_k[lane * 32 + h] : kInf;
+            hi = h < kp ? s_i[lane * 32 + h] : INT_MAX;
         }
     }
     float d = fminf(hk, th);
@@ -1397,9 +1397,9 @@ __device__ __noinline__ void merge_rounds(const RaceArgs& a, int64_t r, int64_t 
 }
 
 template <int DT, bool VERIFY, bool BLK>
-__device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_t gw, int64_t NW, int64_t v0,
-                                            int64_t v1, const WarpList L, int kr, int kp, Blk bk, uint32_t* scratch,
-                                            float* s_mk, int* s_mi) {
+__device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_t gw, int64_t NW, int64_t nb,
+                                            int64_t v0, int64_t v1, const WarpList L, int kr, int kp, Blk bk,
+                                            uint32_t* scratch, float* s_mk, int* s_mi) {
     const int lane = threadIdx.x & 31;
     const int64_t nv = a.nv;
     float lk = L.lk;
@@ -1415,8 +1415,9 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
         if (lane == 0) P->theta_drop = theta_drop;
         __threadfence();
         __syncwarp();
-        const int64_t first_w = warp_of(r * nv, a.total, NW);
-        const int64_t last_w = warp_of(r * nv + nv - 1, a.total, NW);
+        const int64_t units = a.n_rows * nb;
+        const int64_t first_w = warp_of(r * nb, units, NW);
+        const int64_t last_w = warp_of(r * nb + nb - 1, units, NW);
         unsigned last = 0;
         if (lane == 0) {
             unsigned t = atomicAdd(a.row_cnt + r, 1u);
@@ -1446,28 +1447,35 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
 
 // ---------------------------------------------------------------- the kernel
 //
-// Every warp is an independent worker: warp gw of NW streams the flattened
-// vector slice [gw*total/NW, (gw+1)*total/NW).  A row cut between warps is
-// merged and finished by the warp that arrives last at the row's counter; a
-// sequence's walk is run by the warp that finishes its last node.  No warp
-// ever waits for another and the kernel has no block-wide barrier.
+// Every warp is an independent worker.  A row is cut into nb units of one
+// fast-loop iteration (the last may be shorter), and warp gw of NW streams the
+// units [gw*U/NW, (gw+1)*U/NW) of the U = n_rows * nb units in row order, so
+// that a segment ends on an iteration boundary and only a row's ragged end
+// takes the scalar tail.  A row cut between warps is merged and finished by
+// the warp that arrives last at the row's counter; a sequence's walk is run by
+// the warp that finishes its last node.  No warp ever waits for another and
+// the kernel has no block-wide barrier.
 
 template <int DT, bool VERIFY, bool VEC, bool BLK>
 __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RACE_MIN_BLOCKS) race_kernel(const RaceArgs a) {
     __shared__ uint32_t s_queue[kQueueCap];
-    __shared__ float s_mk[32 * 32];  // staging of the partial lists merged by merge_rounds
-    __shared__ int s_mi[32 * 32];
+    __shared__ __align__(16) float s_mk[32 * 32];  // staging of the partial lists merged by merge_rounds
+    __shared__ __align__(16) int s_mi[32 * 32];
     pdl_wait();  // the previous kernel's outputs (row ids, lists) and the workspace it used
     pdl_launch_dependents();
     const int64_t NW = a.G;
     const int64_t gw = blockIdx.x;
-    const int64_t g0 = gw * a.total / NW, g1 = (gw + 1) * a.total / NW;
     const float c = a.c;
     const int64_t nv = a.nv;
     const size_t esz = DT == 1 ? 2 : 4;
+    constexpr int64_t kUnit = (DT == 1 ? 32 : 64) * PPS_UNITS_VERIFY;  // vectors per unit (one fast iteration)
+    const int64_t nb = (nv + kUnit - 1) / kUnit;
+    const int64_t units = a.n_rows * nb;
+    const int64_t u0 = gw * units / NW, u1 = (gw + 1) * units / NW;
 
-    for (int64_t r = g0 / nv; g0 < g1 && r < a.n_rows && r * nv < g1; ++r) {
-        const int64_t v0 = max(g0, r * nv) - r * nv, v1 = min(g1, (r + 1) * nv) - r * nv;
+    for (int64_t r = u0 / nb; u0 < u1 && r < a.n_rows && r * nb < u1; ++r) {
+        const int64_t v0 = (max(u0, r * nb) - r * nb) * kUnit;
+        const int64_t v1 = min((min(u1, (r + 1) * nb) - r * nb) * kUnit, nv);
         int kr = 1;
         if (!VERIFY) {
             kr = a.row_k ? __ldg(a.row_k + r) : a.K;
@@ -1500,7 +1508,7 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
             stream_segment<DT, VEC, BLK, VERIFY || DT == 0, VERIFY ? PPS_UNITS_VERIFY : PPS_UNITS>(
                 L, row, a.V, v0, v1, c, key, ctx, pos, s_queue, bk, slot);
 
-        finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, v0, v1, L, kr, kp, bk, s_queue, s_mk, s_mi);
+        finish_segment<DT, VERIFY, BLK>(a, r, gw, NW, nb, v0, v1, L, kr, kp, bk, s_queue, s_mk, s_mi);
     }
 }
 
@@ -1528,6 +1536,13 @@ int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk, int64_t
     int64_t by_size = (total + kMinVecsPerWarp - 1) / kMinVecsPerWarp;
     if (by_size < g) g = by_size;
     if (PPS_SEG_CAP > 0 && n_rows > 0 && n_rows * PPS_SEG_CAP < g) g = n_rows * PPS_SEG_CAP;
+    if (n_rows > 0) {
+        // every warp gets at least one unit (one fast iteration of a row), so every
+        // warp a row's counter waits for streams part of it
+        const int64_t unit = (dtype == 1 ? 32 : 64) * PPS_UNITS_VERIFY;
+        const int64_t units = n_rows * ((total / n_rows + unit - 1) / unit);
+        if (units < g) g = units;
+    }
     if (g > kGridMax) g = kGridMax;
     if (g < 1) g = 1;
     return (int)g;
