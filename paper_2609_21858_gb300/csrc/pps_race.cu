@@ -1163,6 +1163,9 @@ __device__ __noinline__ void finalize_row(const RaceArgs& a, int64_t r, float lk
     finalize_row_lp<DT, VERIFY, BLK>(a, r, lk, li, theta_drop, kr, kp, lane, dense_logits<DT>(a, r), bk, scratch);
 }
 
+// vectors per unit of the streaming kernel's row partition (see race_kernel)
+__host__ __device__ constexpr int64_t race_unit(int dt) { return dt == 1 ? 32 * PPS_UNITS_VERIFY : 1; }
+
 __device__ __forceinline__ int64_t warp_of(int64_t g, int64_t total, int64_t NW) {
     // largest w with floor(w*total/NW) <= g
     return ((g + 1) * NW - 1) / total;
@@ -1447,11 +1450,14 @@ __device__ __noinline__ void finish_segment(const RaceArgs& a, int64_t r, int64_
 
 // ---------------------------------------------------------------- the kernel
 //
-// Every warp is an independent worker.  A row is cut into nb units of one
-// fast-loop iteration (the last may be shorter), and warp gw of NW streams the
-// units [gw*U/NW, (gw+1)*U/NW) of the U = n_rows * nb units in row order, so
-// that a segment ends on an iteration boundary and only a row's ragged end
-// takes the scalar tail.  A row cut between warps is merged and finished by
+// Every warp is an independent worker.  A row is cut into nb units of
+// race_unit(DT) vectors (the last may be shorter), and warp gw of NW streams the
+// units [gw*U/NW, (gw+1)*U/NW) of the U = n_rows * nb units in row order.  For
+// bf16 rows a unit is one fast-loop iteration, so that a segment ends on an
+// iteration boundary and only a row's ragged end takes the scalar tail
+// (measured on the bench tree: verify 0.282 -> 0.272 ms, draft 0.248 ->
+// 0.235 ms); fp32 rows keep units of one vector (iteration units made the
+// fp32 tree slower, 7.35 -> 7.73 ms).  A row cut between warps is merged and finished by
 // the warp that arrives last at the row's counter; a sequence's walk is run by
 // the warp that finishes its last node.  No warp ever waits for another and
 // the kernel has no block-wide barrier.
@@ -1468,7 +1474,7 @@ __global__ void __launch_bounds__(kThreads, BLK ? PPS_BLOCK_MIN_BLOCKS : PPS_RAC
     const float c = a.c;
     const int64_t nv = a.nv;
     const size_t esz = DT == 1 ? 2 : 4;
-    constexpr int64_t kUnit = (DT == 1 ? 32 : 64) * PPS_UNITS_VERIFY;  // vectors per unit (one fast iteration)
+    constexpr int64_t kUnit = race_unit(DT);
     const int64_t nb = (nv + kUnit - 1) / kUnit;
     const int64_t units = a.n_rows * nb;
     const int64_t u0 = gw * units / NW, u1 = (gw + 1) * units / NW;
@@ -1539,7 +1545,7 @@ int race_grid(int64_t total, int dtype, bool verify, bool vec, bool blk, int64_t
     if (n_rows > 0) {
         // every warp gets at least one unit (one fast iteration of a row), so every
         // warp a row's counter waits for streams part of it
-        const int64_t unit = (dtype == 1 ? 32 : 64) * PPS_UNITS_VERIFY;
+        const int64_t unit = race_unit(dtype);
         const int64_t units = n_rows * ((total / n_rows + unit - 1) / unit);
         if (units < g) g = units;
     }
