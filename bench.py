@@ -32,7 +32,6 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "verified rows/s and GB/s vs HBM peak at V=128256, K=8, B=64 (1xGB300)"
-WIDE_MULS_PER_TOKEN = 4.5
 WIDE_MULS_PER_SM_CLK = 32
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "race_kernel_zipf_k8_traffic.txt")
 TRUNC_TRAFFIC_FILE = os.path.join(ROOT, "profiles", "trunc_kernel_zipf_k8_top50_traffic.txt")
@@ -251,6 +250,10 @@ def main():
     ap.add_argument("--top-p", type=float, default=1.0, help="then to its top-p set (with --top-k)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--philox-rounds", type=int, default=10, choices=[7, 10],
+                    help="keyed source of the run: Philox4x32-10 (libpps.so) or -7 (libpps_r7.so)")
+    ap.add_argument("--no-philox7", action="store_true",
+                    help="default workload: skip the second measurement with the Philox4x32-7 build")
     ap.add_argument("--eager", action="store_true",
                     help="tree workloads: launch every call from Python instead of replaying a CUDA graph")
     args = ap.parse_args()
@@ -265,7 +268,11 @@ def main():
         return
 
     from paper_2609_21858_gb300 import pps
+    pps.use_library(args.philox_rounds)
     pps.lib()
+    if args.philox_rounds != 10 and not args.no_cpu_baseline:
+        import oracle
+        oracle.set_philox_rounds(args.philox_rounds)
     dev = torch.device("cuda", local)
     if args.workload == "detector":
         run_detector(args, rank, world, dev)
@@ -375,7 +382,8 @@ def main():
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     clk = (clocks.get("sm_mhz") or 2070.0) * 1e6
     mul_peak = sms * WIDE_MULS_PER_SM_CLK * clk / 1e12
-    mul_ach = tok_verify * WIDE_MULS_PER_TOKEN / (t_verify / 1e3) / 1e12
+    muls_per_token = (2 * args.philox_rounds - 2) / 4  # rounds 1-2 hoisted: 2 R - 2 products per 4 tokens
+    mul_ach = tok_verify * muls_per_token / (t_verify / 1e3) / 1e12
     traffic = None
     if args.workload == "zipf_k8" and args.n_seq is None:
         if args.top_k == 0:
@@ -471,6 +479,49 @@ def main():
         if whole:
             parity = step_parity(wl, keep, dout, vout)
 
+    # ---- the same step with the Philox4x32-7 keyed source (libpps_r7.so): a second number beside
+    # the default's, with every row compared with the oracle at 7 rounds
+    mean_acc = float(vout["accept_len"].float().mean().item())
+    philox7 = None
+    if (args.workload == "zipf_k8" and args.n_seq is None and args.top_k == 0 and args.philox_rounds == 10
+            and not args.no_philox7 and flush is None):
+        pps.use_library(7)
+        for _ in range(3):
+            step(q, p)
+        torch.cuda.synchronize(dev)
+        evs7 = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+        s7, e7 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier(world)
+        s7.record(stream)
+        for k in range(args.steps):
+            step(q, p, evs7[k])
+        e7.record(stream)
+        torch.cuda.synchronize(dev)
+        ms7 = max_over_ranks(s7.elapsed_time(e7), world) / args.steps
+        td7 = statistics.mean(e[0].elapsed_time(e[1]) for e in evs7)
+        tv7 = statistics.mean(e[1].elapsed_time(e[2]) for e in evs7)
+        ph7 = philox_only_rate(dev) if rank == 0 else None
+        par7 = None
+        if rank == 0 and not args.no_cpu_baseline and parity is not None:
+            import oracle
+            oracle.set_philox_rounds(7)
+            keep7 = {}
+            run7, _, _, _ = oracle_sample(wl, t.n_draft, t.n_nodes, keep=keep7)
+            run7()
+            par7 = step_parity(wl, keep7, dout, vout)
+            oracle.set_philox_rounds(10)
+        philox7 = {"keyed_source": "Philox4x32-7 (libpps_r7.so; an option beside the default)",
+                   "value": rows_per_step * world / (ms7 / 1e3), "unit": "rows/s", "ms_per_step": ms7,
+                   "roofline": {"bound": "hbm", "achieved": bytes_verify / (tv7 / 1e3) / 1e9, "peak": peak,
+                                "unit": "GB/s", "frac": bytes_verify / (tv7 / 1e3) / 1e9 / peak, "ms": tv7,
+                                "kernel": "race_kernel (pps_verify_tree)"},
+                   "roofline_draft": {"frac": bytes_draft / (td7 / 1e3) / 1e9 / peak, "ms": td7},
+                   "philox_only_tok_s": ph7,
+                   "frac_of_philox_only": tok_verify / (tv7 / 1e3) / ph7 if ph7 else None,
+                   "mean_accept_len": float(vout["accept_len"].float().mean().item()),
+                   "parity": par7}
+        pps.use_library(10)
+
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": args.steps,
@@ -501,13 +552,15 @@ def main():
                              "frac": mul_ach / mul_peak,
                              "peak_kind": f"derived, not measured: {sms} SMs x {WIDE_MULS_PER_SM_CLK} "
                                           f"32x32->64 multiplies/clk x {clk / 1e6:.0f} MHz (median sampled SM clock)",
-                             "work": f"{WIDE_MULS_PER_TOKEN} wide multiplies per token x {tok_verify} tokens",
+                             "work": f"{muls_per_token} wide multiplies per token x {tok_verify} tokens",
                              "tok_s": tok_verify / (t_verify / 1e3), "philox_only_tok_s": philox_tok_s,
                              "frac_of_philox_only": (tok_verify / (t_verify / 1e3) / philox_tok_s
                                                      if philox_tok_s else None)},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": 2 * args.steps, "clocks": clocks,
-            "mean_accept_len": float(vout["accept_len"].float().mean().item()),
+            "mean_accept_len": mean_acc,
             "parity": parity,
+            "keyed_source": f"Philox4x32-{args.philox_rounds}",
+            "philox7": philox7,
         }
         print(json.dumps(line))
 
@@ -805,13 +858,14 @@ def run_hetero(args, rank, world, dev):
     hz = (clocks.get("sm_mhz") or 2070.0) * 1e6
     mul_peak = sms * WIDE_MULS_PER_SM_CLK * hz / 1e12
     tok_draft = n_prop * V
-    mul_ach = tok_draft * WIDE_MULS_PER_TOKEN / (t_draft / 1e3) / 1e12
+    muls_per_token = (2 * args.philox_rounds - 2) / 4
+    mul_ach = tok_draft * muls_per_token / (t_draft / 1e3) / 1e12
     trunc = f", top-k {tk}, top-p {tp}" if tk > 0 else ""
     roof_alu = {"bound": "alu", "achieved": mul_ach, "peak": mul_peak, "unit": "T wide-mul/s",
                 "frac": mul_ach / mul_peak,
                 "peak_kind": f"derived, not measured: {sms} SMs x {WIDE_MULS_PER_SM_CLK} 32x32->64 "
                              f"multiplies/clk x {hz / 1e6:.0f} MHz (median sampled SM clock)",
-                "work": f"{WIDE_MULS_PER_TOKEN} wide multiplies per token x {tok_draft} tokens"}
+                "work": f"{muls_per_token} wide multiplies per token x {tok_draft} tokens"}
     gbs_d = n_prop * V * 2 / (t_draft / 1e3) / 1e9
     kern = "trunc_kernel" if tk > 0 else "race_kernel"
     roof = {"bound": "hbm", "achieved": gbs_d, "peak": peak, "unit": "GB/s", "frac": gbs_d / peak,

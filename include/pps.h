@@ -79,6 +79,15 @@ typedef struct {
 const char* pps_version(void);
 const char* pps_status_string(pps_status s);
 
+/* Rounds of the keyed source's Philox4x32 in this build of the library: 10
+ * (libpps.so, Philox4x32-10 of Salmon et al., SC'11: every word, list, winner
+ * and score of the other entry points follows it) or 7 (libpps_r7.so, built
+ * with PPS_PHILOX_ROUNDS=7: the same counters and keys, three rounds fewer; a
+ * different keyed source, so its outputs differ from libpps.so's).  The
+ * paper's method needs a keyed pseudorandom function (Sec. 3.1); which
+ * variant a deployment uses is fixed when it picks the library. */
+int pps_philox_rounds(void);
+
 /* Bytes of workspace pps_draft_list / pps_verify_tree need for n_rows rows and
  * n_seq sequences (n_seq = 0 for pps_draft_list).  The workspace holds
  * per-row partial candidate lists, arrival counters and the shared filter

@@ -55,6 +55,10 @@ def lib():
             i64, i32, f64 = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
             L.orc_philox4x32_10.argtypes = [u32p, u32p, u32p]
             L.orc_philox4x32_10.restype = None
+            L.orc_philox4x32.argtypes = [u32p, u32p, i32, u32p]
+            L.orc_philox4x32.restype = None
+            L.orc_set_philox_rounds.argtypes = [i32]
+            L.orc_set_philox_rounds.restype = i32
             L.orc_word.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32, i64, i32]
             L.orc_word.restype = ctypes.c_uint32
             L.orc_uniform.argtypes = [ctypes.c_uint32]
@@ -134,6 +138,20 @@ def philox4x32_10(ctr, key):
     out = np.zeros(4, np.uint32)
     lib().orc_philox4x32_10(_ptr(c, ctypes.c_uint32), _ptr(k, ctypes.c_uint32), _ptr(out, ctypes.c_uint32))
     return out
+
+
+def philox4x32(ctr, key, rounds: int):
+    c = _c(ctr, np.uint32)
+    k = _c(key, np.uint32)
+    out = np.zeros(4, np.uint32)
+    lib().orc_philox4x32(_ptr(c, ctypes.c_uint32), _ptr(k, ctypes.c_uint32), int(rounds), _ptr(out, ctypes.c_uint32))
+    return out
+
+
+def set_philox_rounds(rounds: int = 0) -> int:
+    """Set (rounds > 0) and return the Philox round count of the keyed source (10 by default;
+    7 for the library built with PPS_PHILOX_ROUNDS=7).  Process-wide."""
+    return int(lib().orc_set_philox_rounds(int(rounds)))
 
 
 def word(key: int, ctx: int, pos: int, token: int, arrival: int = 1) -> int:

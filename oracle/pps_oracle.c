@@ -18,6 +18,12 @@
  *                      paper only asks for a keyed pseudorandom function
  *                      F_{ctx,k} (Sec. 3.1, Eq. 1) / keyed source G(k,c)
  *                      (Alg. 3); Philox is the reading taken here.
+ *   orc_philox4x32     the same with R rounds (Philox4x32-R); the keyed source
+ *                      uses R = orc_set_philox_rounds() (10, or 7 for the
+ *                      cheaper variant a library build can select).  Pinned
+ *                      through the 10-round known answers: R rounds followed by
+ *                      10 - R rounds under the key advanced by R Weyl steps are
+ *                      the 10-round function.
  *   orc_word           the keyed source Pi_k(c): counter (token>>2, pos,
  *                      ctx_lo, ctx_hi), key (key_lo ^ (j-1)*0x9E3779B9, key_hi)
  *                      for arrival j, output lane token&3.
@@ -94,11 +100,13 @@
 #define ORC_PHILOX_W0 0x9E3779B9u
 #define ORC_PHILOX_W1 0xBB67AE85u
 
-void orc_philox4x32_10(const uint32_t ctr_in[4], const uint32_t key_in[2], uint32_t out[4])
+/* Philox4x32 with `rounds` rounds (the same round function and key schedule;
+ * Philox4x32-R of Salmon et al. for R = rounds). */
+void orc_philox4x32(const uint32_t ctr_in[4], const uint32_t key_in[2], int rounds, uint32_t out[4])
 {
     uint32_t x0 = ctr_in[0], x1 = ctr_in[1], x2 = ctr_in[2], x3 = ctr_in[3];
     uint32_t k0 = key_in[0], k1 = key_in[1];
-    for (int round = 0; round < 10; ++round) {
+    for (int round = 0; round < rounds; ++round) {
         if (round > 0) { /* key schedule: bump before every round but the first */
             k0 += ORC_PHILOX_W0;
             k1 += ORC_PHILOX_W1;
@@ -116,6 +124,21 @@ void orc_philox4x32_10(const uint32_t ctr_in[4], const uint32_t key_in[2], uint3
     out[0] = x0; out[1] = x1; out[2] = x2; out[3] = x3;
 }
 
+void orc_philox4x32_10(const uint32_t ctr_in[4], const uint32_t key_in[2], uint32_t out[4])
+{
+    orc_philox4x32(ctr_in, key_in, 10, out);
+}
+
+/* Rounds of the keyed source's Philox: 10 (the published default), or the
+ * cheaper variant a library build selects (7).  Process-wide; set it before
+ * any oracle computation.  r <= 0 only queries.  Returns the setting. */
+static int orc_rounds = 10;
+int orc_set_philox_rounds(int r)
+{
+    if (r > 0 && r <= 16) orc_rounds = r;
+    return orc_rounds;
+}
+
 /* Keyed source: the 32-bit word of token `token`, arrival j >= 1, at the
  * context labelled (ctx, pos) under watermark key `key`. */
 uint32_t orc_word(uint64_t key, uint64_t ctx, uint32_t pos, int64_t token, int32_t arrival)
@@ -128,7 +151,7 @@ uint32_t orc_word(uint64_t key, uint64_t ctx, uint32_t pos, int64_t token, int32
     uint32_t tweak = (uint32_t)(arrival - 1) * ORC_PHILOX_W0; /* 0 for the first arrival */
     k[0] = (uint32_t)(key & 0xFFFFFFFFull) ^ tweak;
     k[1] = (uint32_t)(key >> 32);
-    orc_philox4x32_10(ctr, k, out);
+    orc_philox4x32(ctr, k, orc_rounds, out);
     return out[token & 3];
 }
 

@@ -32,31 +32,47 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
+# Library variants: the default (Philox4x32-10) and the cheaper keyed source
+# (Philox4x32-7), each from the same sources with its own objects.
+VARIANTS = {"": [], "_r7": ["-DPPS_PHILOX_ROUNDS=7"]}
+
+
+def lib_path(variant: str = "") -> str:
+    return os.path.join(OUT, f"libpps{variant}.so")
+
+
 def build(force: bool = False, verbose: bool = False) -> str:
     os.makedirs(OUT, exist_ok=True)
     hdrs = [os.path.join(CSRC, h) for h in HEADERS] + [os.path.join(ROOT, "include", "pps.h")]
     flags = ["-std=c++17", "-O3", "-lineinfo", "-Xcompiler", "-fPIC", "-I" + os.path.join(ROOT, "include")] + ARCH
     flags += os.environ.get("PPS_NVCC_FLAGS", "").split()  # extra flags for experiments (e.g. -DPPS_RACE_MIN_BLOCKS=4)
 
-    def compile_one(src):
+    def compile_one(job):
+        variant, src = job
         s = os.path.join(CSRC, src)
-        o = os.path.join(OUT, src.replace(".cu", ".o"))
+        d = os.path.join(OUT, "obj" + variant)
+        os.makedirs(d, exist_ok=True)
+        o = os.path.join(d, src.replace(".cu", ".o"))
         if force or _stale(o, [s] + hdrs):
-            cmd = [nvcc()] + flags + ["-c", s, "-o", o]
+            cmd = [nvcc()] + flags + VARIANTS[variant] + ["-c", s, "-o", o]
             if verbose:
                 print(" ".join(cmd), flush=True)
             subprocess.run(cmd, check=True)
         return o
 
-    with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        objs = list(ex.map(compile_one, SOURCES))
-    if force or _stale(LIB, objs):
-        tmp = LIB + f".tmp{os.getpid()}"
-        cmd = [nvcc()] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs
-        if verbose:
-            print(" ".join(cmd), flush=True)
-        subprocess.run(cmd, check=True)
-        os.replace(tmp, LIB)
+    jobs = [(v, src) for v in VARIANTS for src in SOURCES]
+    with ThreadPoolExecutor(max_workers=len(jobs)) as ex:
+        objs = list(ex.map(compile_one, jobs))
+    for i, v in enumerate(VARIANTS):
+        vobjs = objs[i * len(SOURCES):(i + 1) * len(SOURCES)]
+        target = lib_path(v)
+        if force or _stale(target, vobjs):
+            tmp = target + f".tmp{os.getpid()}"
+            cmd = [nvcc()] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + vobjs
+            if verbose:
+                print(" ".join(cmd), flush=True)
+            subprocess.run(cmd, check=True)
+            os.replace(tmp, target)
     return LIB
 
 

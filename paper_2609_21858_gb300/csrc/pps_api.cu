@@ -129,7 +129,9 @@ using namespace pps;
 
 extern "C" {
 
-const char* pps_version(void) { return "libpps 0.1 (sm_103a)"; }
+#define PPS_STR2(x) #x
+#define PPS_STR(x) PPS_STR2(x)
+const char* pps_version(void) { return "libpps 0.1 (sm_103a, Philox4x32-" PPS_STR(PPS_PHILOX_ROUNDS) ")"; }
 
 const char* pps_status_string(pps_status s) {
     switch (s) {
@@ -142,6 +144,8 @@ const char* pps_status_string(pps_status s) {
     }
     return "unknown status";
 }
+
+int pps_philox_rounds(void) { return PPS_PHILOX_ROUNDS; }
 
 size_t pps_workspace_size(int64_t n_rows, int64_t vocab, int32_t K, int32_t n_seq) {
     (void)vocab;

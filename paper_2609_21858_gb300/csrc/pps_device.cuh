@@ -48,6 +48,12 @@ __device__ __forceinline__ float key_err_bound(float k) { return kErrAbs + kErrR
 __device__ __forceinline__ float filter_slack(float t) { return t + 4.0f * key_err_bound(t); }
 
 // ------------------------------------------------------------------ Philox
+//
+// PPS_PHILOX_ROUNDS: rounds of the keyed source's Philox4x32.  10 (Salmon et
+// al.'s default) unless the library is built with 7, the smallest count they
+// report free of Crush failures (libpps_r7.so; pps_philox_rounds() tells a
+// caller which one it loaded).
+static_assert(PPS_PHILOX_ROUNDS >= 3 && PPS_PHILOX_ROUNDS <= 16, "two hoisted rounds and at least one more");
 
 __device__ __forceinline__ void mulhilo(uint32_t a, uint32_t b, uint32_t& hi, uint32_t& lo) {
     uint64_t p = (uint64_t)a * (uint64_t)b;
@@ -55,10 +61,10 @@ __device__ __forceinline__ void mulhilo(uint32_t a, uint32_t b, uint32_t& hi, ui
     lo = (uint32_t)p;
 }
 
-// full Philox4x32-10 on counter (x0..x3), key (k0, k1)
+// full Philox4x32 (PPS_PHILOX_ROUNDS rounds) on counter (x0..x3), key (k0, k1)
 __device__ __forceinline__ uint4 philox(uint32_t x0, uint32_t x1, uint32_t x2, uint32_t x3, uint32_t k0, uint32_t k1) {
 #pragma unroll
-    for (int r = 0; r < 10; ++r) {
+    for (int r = 0; r < PPS_PHILOX_ROUNDS; ++r) {
         if (r) {
             k0 += kPhiloxW0;
             k1 += kPhiloxW1;
@@ -103,7 +109,7 @@ struct RowPhilox {
     uint32_t r2_f;            // lo(M1 * ctx_lo) ^ (k0 + W0)             (round 2, word 0 xor term)
     uint32_t r2_gh;           // hi(M0 * y0) ^ (k1 + W1), y0 = hi(M1*ctx_lo) ^ pos ^ k0   (round 2, word 2)
     uint32_t r2_lo0;          // lo(M0 * y0)                             (round 2, word 3)
-    uint32_t rk0[8], rk1[8];  // keys of rounds 3..10
+    uint32_t rk0[PPS_PHILOX_ROUNDS - 2], rk1[PPS_PHILOX_ROUNDS - 2];  // keys of rounds 3..
 
     // Called by all 32 lanes of a warp with the same row.  The warp reductions
     // (of equal values) mark the row constants as warp-uniform, so the
@@ -131,7 +137,7 @@ struct RowPhilox {
         r2_f = lo1 ^ (k0 + kPhiloxW0);
         r2_gh = hi ^ (k1 + kPhiloxW1);
 #pragma unroll
-        for (int r = 0; r < 8; ++r) {
+        for (int r = 0; r < PPS_PHILOX_ROUNDS - 2; ++r) {
             rk0[r] = k0 + (uint32_t)(r + 2) * kPhiloxW0;
             rk1[r] = k1 + (uint32_t)(r + 2) * kPhiloxW1;
         }
@@ -152,7 +158,7 @@ struct RowPhilox {
         uint32_t x2 = y3 ^ r2_gh;
         uint32_t x3 = r2_lo0;
 #pragma unroll
-        for (int r = 0; r < 8; ++r) {
+        for (int r = 0; r < PPS_PHILOX_ROUNDS - 2; ++r) {
             uint32_t a0, b0, a1, b1;
             mulhilo(kPhiloxM0, x0, a0, b0);
             mulhilo(kPhiloxM1, x2, a1, b1);

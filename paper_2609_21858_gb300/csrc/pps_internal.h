@@ -3,6 +3,12 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
+// Rounds of the keyed source's Philox4x32 (pps_device.cuh): 10 unless the
+// library is built with -DPPS_PHILOX_ROUNDS=7 (libpps_r7.so).
+#ifndef PPS_PHILOX_ROUNDS
+#define PPS_PHILOX_ROUNDS 10
+#endif
+
 namespace pps {
 
 constexpr int kThreads = 32;            // one warp per CTA: per-row values are CTA-uniform

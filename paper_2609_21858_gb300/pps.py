@@ -12,7 +12,18 @@ import threading
 import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "_lib", "libpps.so")
+
+
+def library_path(rounds: int = 10) -> str:
+    """The build of libpps whose keyed source is Philox4x32 with `rounds` rounds: 10
+    (libpps.so, the default) or 7 (libpps_r7.so)."""
+    if rounds not in (7, 10):
+        raise ValueError("libpps is built for Philox4x32-10 and Philox4x32-7 only")
+    return os.path.join(_HERE, "_lib", "libpps.so" if rounds == 10 else "libpps_r7.so")
+
+
+# PPS_PHILOX_ROUNDS=7 in the environment selects the Philox4x32-7 build at import
+LIB_PATH = library_path(int(os.environ.get("PPS_PHILOX_ROUNDS", "10")))
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_SIZE = 0, 1, 2, 3, 4, 5
 NOALLOC_MAX_ROWS = 4096  # PPS_NOALLOC_MAX_ROWS of include/pps.h (tests/test_abi.py checks the two agree)
@@ -38,6 +49,20 @@ class PPSError(RuntimeError):
         self.code = code
 
 
+def use_library(rounds: int = 10):
+    """Switch the binding to the build for Philox4x32-`rounds` (the next call loads it).
+    Device memory (workspaces, outputs) carries over; results follow the new keyed source."""
+    global _lib, LIB_PATH
+    with _lock:
+        LIB_PATH = library_path(rounds)
+        _lib = None
+
+
+def philox_rounds() -> int:
+    """Rounds of the keyed source of the loaded library (pps_philox_rounds)."""
+    return int(lib().pps_philox_rounds())
+
+
 def lib():
     """Load libpps.so (raises if it was not built)."""
     global _lib
@@ -50,6 +75,8 @@ def lib():
             vp, i64, i32, f32, u64, sz = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_float,
                                           ctypes.c_uint64, ctypes.c_size_t)
             L.pps_version.restype = ctypes.c_char_p
+            L.pps_philox_rounds.argtypes = []
+            L.pps_philox_rounds.restype = ctypes.c_int
             L.pps_status_string.argtypes = [ctypes.c_int]
             L.pps_status_string.restype = ctypes.c_char_p
             L.pps_workspace_size.argtypes = [i64, i64, i32, i32]

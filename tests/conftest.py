@@ -11,6 +11,12 @@ if ROOT not in sys.path:
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a) and the built libpps.so")
     config.addinivalue_line("markers", "slow: long-running statistical check")
+    # PPS_PHILOX_ROUNDS=7: the binding loads libpps_r7.so (the Philox4x32-7 keyed source), and the
+    # oracle's keyed source takes the same round count
+    rounds = os.environ.get("PPS_PHILOX_ROUNDS")
+    if rounds:
+        import oracle
+        oracle.set_philox_rounds(int(rounds))
 
 
 def pytest_terminal_summary(terminalreporter):

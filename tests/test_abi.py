@@ -30,6 +30,19 @@ def test_library_exports_every_declared_symbol():
     assert "sm_103a" in pps.version()
 
 
+def test_both_keyed_source_builds_export_every_symbol_and_report_their_rounds():
+    # libpps.so: Philox4x32-10; libpps_r7.so: the same sources built with PPS_PHILOX_ROUNDS=7
+    # (loading the libraries and these two queries need no GPU)
+    for rounds in (10, 7):
+        L = ctypes.CDLL(pps.library_path(rounds))
+        for n in _declared():
+            assert hasattr(L, n), (rounds, n)
+        L.pps_philox_rounds.restype = ctypes.c_int
+        L.pps_version.restype = ctypes.c_char_p
+        assert L.pps_philox_rounds() == rounds
+        assert f"Philox4x32-{rounds}".encode() in L.pps_version()
+
+
 def _ids0():
     return pps.RowIds(None, None, None)
 

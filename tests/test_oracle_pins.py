@@ -39,6 +39,20 @@ def test_philox_known_answers(ctr, key, out):
 
 
 @pytest.mark.parametrize("ctr,key,out", _kat())
+@pytest.mark.parametrize("rounds", [1, 3, 5, 7, 9])
+def test_philox_r_rounds_continue_into_the_known_answers(ctr, key, out, rounds):
+    # Philox4x32-R is the first R rounds of the 10-round function: its output, taken
+    # through the remaining 10 - R rounds under the key advanced by R Weyl steps (the
+    # schedule bumps the key before every round but the first), gives the published
+    # 10-round answer.  Pins the round count the keyed source uses at 7 rounds.
+    w0, w1 = 0x9E3779B9, 0xBB67AE85
+    head = oracle.philox4x32(ctr, key, rounds)
+    k2 = [(key[0] + rounds * w0) & 0xFFFFFFFF, (key[1] + rounds * w1) & 0xFFFFFFFF]
+    assert [int(x) for x in oracle.philox4x32(head, k2, 10 - rounds)] == out
+    assert [int(x) for x in oracle.philox4x32(ctr, key, 10)] == out
+
+
+@pytest.mark.parametrize("ctr,key,out", _kat())
 def test_word_layout_reaches_known_answers(ctr, key, out):
     # word(token) = lane token&3 of the block at counter (token>>2, pos, ctx_lo, ctx_hi), key (key_lo, key_hi)
     k64 = key[0] | (key[1] << 32)
