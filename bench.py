@@ -682,7 +682,7 @@ def run_detector(args, rank, world, dev):
             "detection": {"tpr_at_1pct_fpr": float(np.mean(wm <= alpha)), "fpr_null": float(np.mean(null <= alpha)),
                           "anlppt_watermarked": float(np.mean(-wm / 128.0)),
                           "anlppt_null": float(np.mean(-null / 128.0)), "segments": int(n_seg)},
-            "gpu_launches": 2 * args.steps, "clocks": clocks,
+            "gpu_launches": 2 * args.steps, "clocks": clocks, "keyed_source": f"Philox4x32-{args.philox_rounds}",
         }))
 
 
@@ -749,6 +749,7 @@ def run_dynamic(args, rank, world, dev):
             "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
                          "traffic": None, "peak_kind": peak_kind, "algorithmic_bytes": nbytes},
             "gpu_launches": args.steps * (2 * gamma + 1), "clocks": clocks,
+            "keyed_source": f"Philox4x32-{args.philox_rounds}",
             "mean_accept_len": float(vout["accept_len"].float().mean().item()),
             "mean_draft_nodes_per_seq": float((b.row_k[:b.n_draft] > 0).sum().item()) / n_seq,
         }))
@@ -889,6 +890,7 @@ def run_hetero(args, rank, world, dev):
             "roofline_verify": {"bound": "hbm", "achieved": b.n_nodes * V * 2 / (t_verify / 1e3) / 1e9,
                                 "peak": peak, "peak_kind": peak_kind, "ms": t_verify},
             "gpu_launches": args.steps * (2 * gamma + 1), "clocks": clocks,
+            "keyed_source": f"Philox4x32-{args.philox_rounds}",
             "mean_accept_len": float(vout["accept_len"].float().mean().item()),
             "mean_nodes_per_seq": float((b.node_ctx != 0).sum().item()) / n_seq,
         }))
@@ -1031,6 +1033,7 @@ def run_lmhead(args, rank, world, dev):
                         "same_outputs": same,
                         "logits_bytes_avoided": int((t.n_nodes + t.n_draft) * V * 4 * 2)},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": 4 * args.steps, "clocks": clocks,
+            "keyed_source": f"Philox4x32-{args.philox_rounds}",
             "mean_accept_len": float(vout["accept_len"].float().mean().item()),
         }))
 
