@@ -919,6 +919,13 @@ __device__ __noinline__ bool iid_fast(const RaceArgs& a, int64_t r, float lk, in
     const float lt = mine ? lp(li) : 0.0f;
     float y = mine ? neg_log2_u(word_of(key, ctx, pos, li, 1)) : 0.0f;
     float h = mine ? lk : kInf;  // arrival 1's score is the list key itself
+    // every lane's second arrival up front (independent chains); the rounds below then
+    // extend a dependent chain only for third and later arrivals
+    float y2 = 0.0f, h2 = kInf;
+    if (kr > 1 && mine) {
+        y2 = y + neg_log2_u(word_of(key, ctx, pos, tok, 2));
+        h2 = fmaf(-lt, a.c, lg2_approx(y2));
+    }
     int j = 1, mult = 0, sample = -1, nsel = 0;
     float selh = kInf;
     for (int m = 0; m < kr; ++m) {
@@ -935,7 +942,10 @@ __device__ __noinline__ bool iid_fast(const RaceArgs& a, int64_t r, float lk, in
         if (mine && tok == bt) {
             ++mult;
             ++j;
-            if (j <= kr) {
+            if (j == 2 && j <= kr) {
+                y = y2;
+                h = h2;
+            } else if (j <= kr) {
                 y += neg_log2_u(word_of(key, ctx, pos, tok, j));
                 h = fmaf(-lt, a.c, lg2_approx(y));
             } else {
