@@ -264,6 +264,9 @@ def main():
     if args.impl == "reference":
         if rank != 0:
             return
+        if args.philox_rounds != 10:
+            import oracle
+            oracle.set_philox_rounds(args.philox_rounds)
         run_reference(args, world)
         return
 

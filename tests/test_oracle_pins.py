@@ -52,6 +52,24 @@ def test_philox_r_rounds_continue_into_the_known_answers(ctr, key, out, rounds):
     assert [int(x) for x in oracle.philox4x32(ctr, key, 10)] == out
 
 
+def test_keyed_word_follows_the_round_setting():
+    # the keyed source's word at 7 rounds is lane token & 3 of Philox4x32-7 on the same
+    # counter and key; the setting is process-wide, so it is restored whatever happens
+    key, ctx, pos, tok = 0x0123456789ABCDEF, 0xFEDCBA9876543210, 77, 12345
+    ctr = [tok >> 2, pos, ctx & 0xFFFFFFFF, ctx >> 32]
+    k = [key & 0xFFFFFFFF, key >> 32]
+    assert oracle.set_philox_rounds(0) == 10
+    w10 = oracle.word(key, ctx, pos, tok)
+    try:
+        assert oracle.set_philox_rounds(7) == 7
+        w7 = oracle.word(key, ctx, pos, tok)
+        assert w7 == int(oracle.philox4x32(ctr, k, 7)[tok & 3])
+    finally:
+        assert oracle.set_philox_rounds(10) == 10
+    assert w10 == int(oracle.philox4x32_10(ctr, k)[tok & 3]) and w7 != w10
+    assert oracle.word(key, ctx, pos, tok) == w10
+
+
 @pytest.mark.parametrize("ctr,key,out", _kat())
 def test_word_layout_reaches_known_answers(ctr, key, out):
     # word(token) = lane token&3 of the block at counter (token>>2, pos, ctx_lo, ctx_hi), key (key_lo, key_hi)
