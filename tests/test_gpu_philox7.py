@@ -1,8 +1,8 @@
 """The cheaper keyed source: libpps_r7.so (Philox4x32-7, built from the same sources with
 PPS_PHILOX_ROUNDS=7) against the oracle at 7 rounds.  The parity, truncation, tree,
-non-identical-proposal, LM-head, detector and acceptance suites run again in a child process
-with PPS_PHILOX_ROUNDS=7, which makes the binding load libpps_r7.so and the oracle's keyed
-source take 7 rounds (tests/conftest.py).  The full-size suite stays on the default build (the
+non-identical-proposal, LM-head, detector, acceptance and word-statistics suites run again in a
+child process with PPS_PHILOX_ROUNDS=7, which makes the binding load libpps_r7.so and the
+oracle's keyed source take 7 rounds (tests/conftest.py).  The full-size suite stays on the default build (the
 bench line's `philox7` compares every row of the bench step at 7 rounds)."""
 import os
 import subprocess
@@ -31,7 +31,7 @@ def test_parity_suites_with_the_seven_round_keyed_source():
     cmd = [sys.executable, "-m", "pytest", "-x", "-q", "-m", "gpu", "-p", "no:cacheprovider",
            "tests/test_gpu_parity.py", "tests/test_gpu_trunc.py", "tests/test_gpu_tree.py",
            "tests/test_gpu_hetero.py", "tests/test_gpu_lmhead.py", "tests/test_gpu_detect.py",
-           "tests/test_gpu_accept.py"]
+           "tests/test_gpu_accept.py", "tests/test_gpu_words_stats.py"]
     r = subprocess.run(cmd, cwd=ROOT, env=env, capture_output=True, text=True, timeout=1800)
     tail = (r.stdout[-4000:] + "\n" + r.stderr[-2000:])
     print(tail)
