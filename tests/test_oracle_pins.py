@@ -31,6 +31,18 @@ def _kat():
     return rows
 
 
+@pytest.fixture(params=[10, 7], ids=["philox10", "philox7"])
+def keyed_rounds(request):
+    """The distributional pins below run on both keyed sources (Philox4x32-10 and the 7-round
+    option); the oracle's process-wide round setting is restored afterwards."""
+    old = oracle.set_philox_rounds(0)
+    oracle.set_philox_rounds(request.param)
+    try:
+        yield request.param
+    finally:
+        oracle.set_philox_rounds(old)
+
+
 # ---------------------------------------------------------------- Philox / words
 
 @pytest.mark.parametrize("ctr,key,out", _kat())
@@ -172,7 +184,7 @@ def test_target_winner_brute_force_ratio_domain():
 
 
 @pytest.mark.parametrize("V", [2, 5])
-def test_target_winner_distributed_as_p(V):
+def test_target_winner_distributed_as_p(V, keyed_rounds):
     # exactness of the race: y(c) ~ P for every fixed logits row (Thm A.1; batched-algorithm exactness thm)
     rng = np.random.default_rng(10 + V)
     n = 60000
@@ -212,7 +224,7 @@ def test_distinct_list_brute_force():
     assert np.all(d["mult"] == 1) and np.all(d["ndist"] == K)
 
 
-def test_distinct_list_is_plackett_luce():
+def test_distinct_list_is_plackett_luce(keyed_rounds):
     # the K smallest of E_i/q_i come out in Plackett-Luce order of q
     rng = np.random.default_rng(7)
     V, K, n = 4, 2, 60000
@@ -257,7 +269,7 @@ def test_iid_list_brute_force_and_prefix_property():
         assert list(d["tok"][r]) == list(dd["tok"][r])
 
 
-def test_iid_labels_are_iid_q():
+def test_iid_labels_are_iid_q(keyed_rounds):
     # direct finite-support MPFR exactness: the K labels are iid ~ Q
     rng = np.random.default_rng(11)
     V, K, n = 3, 2, 60000
@@ -465,7 +477,7 @@ def test_drafter_invariance():
 
 # ---------------------------------------------------------------- watermark score
 
-def test_null_scores_are_exp1():
+def test_null_scores_are_exp1(keyed_rounds):
     # tokens independent of the key: U ~ Unif(0,1), A ~ Exp(1) (App. D.1)
     rng = np.random.default_rng(50)
     n = 30000
@@ -479,7 +491,7 @@ def test_null_scores_are_exp1():
     assert seg[1] == 0.0 and seg[0] + seg[2] == pytest.approx(tot[0], rel=1e-12)
 
 
-def test_watermarked_pivot_law_and_mean():
+def test_watermarked_pivot_law_and_mean(keyed_rounds):
     # the winner's pivot r = u_y has CDF sum_v p_v x^(1/p_v) (App. D.3), and E[A] >= 1 + (pi^2/6-1) H(p)
     rng = np.random.default_rng(52)
     V, n = 5, 40000
