@@ -30,6 +30,25 @@ def test_library_exports_every_declared_symbol():
     assert "sm_103a" in pps.version()
 
 
+def test_binding_selects_the_keyed_source_build():
+    # the binding loads libpps.so (Philox4x32-10) unless told otherwise, and use_library switches
+    # builds (loading a library and asking its rounds need no GPU)
+    import os as _os
+    assert _os.path.basename(pps.library_path(10)) == "libpps.so"
+    assert _os.path.basename(pps.library_path(7)) == "libpps_r7.so"
+    with pytest.raises(ValueError):
+        pps.library_path(8)
+    default = 10 if not _os.environ.get("PPS_PHILOX_ROUNDS") else int(_os.environ["PPS_PHILOX_ROUNDS"])
+    try:
+        pps.use_library(7)
+        assert pps.philox_rounds() == 7 and "Philox4x32-7" in pps.version()
+        pps.use_library(10)
+        assert pps.philox_rounds() == 10 and "Philox4x32-10" in pps.version()
+    finally:
+        pps.use_library(default)
+    assert pps.philox_rounds() == default
+
+
 def test_both_keyed_source_builds_export_every_symbol_and_report_their_rounds():
     # libpps.so: Philox4x32-10; libpps_r7.so: the same sources built with PPS_PHILOX_ROUNDS=7
     # (loading the libraries and these two queries need no GPU)
