@@ -486,8 +486,11 @@ def main():
     # the default's, with every row compared with the oracle at 7 rounds
     mean_acc = float(vout["accept_len"].float().mean().item())
     philox7 = None
-    if (args.workload == "zipf_k8" and args.n_seq is None and args.top_k == 0 and args.philox_rounds == 10
-            and not args.no_philox7 and flush is None):
+    want7 = (args.workload == "zipf_k8" and args.n_seq is None and args.top_k == 0 and args.philox_rounds == 10
+             and not args.no_philox7 and flush is None)
+    if want7 and not os.path.exists(pps.library_path(7)):
+        philox7 = {"unavailable": "libpps_r7.so was not built (build() makes both libraries)"}
+    elif want7:
         pps.use_library(7)
         for _ in range(3):
             step(q, p)
